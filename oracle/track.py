@@ -1,0 +1,213 @@
+"""The TRACK method in fp64: guidance, scheduler, disagreement, policy, calibration, sampling.
+
+Test infrastructure only (see the package docstring).  Paper references are to
+"Accelerating Video Diffusion via Training-Free Trajectory Routing" (TRACK).
+"""
+from __future__ import annotations
+
+import itertools
+import math
+
+import numpy as np
+
+# ---------------------------------------------------------------------------
+# Scheduler timesteps and the scheduler update (Sec. 3.1, Eq. 2)
+# ---------------------------------------------------------------------------
+
+
+def schedule(n_steps: int, shift: float) -> np.ndarray:
+    """Decreasing noise levels sigma_0 > ... > sigma_N as fp32 values (N+1 of them).
+
+    Sec. 3.1 only requires a decreasing timestep sequence t_0 > ... > t_{N-1};
+    the paper leaves the sampler to each pipeline.  Reading used here: the
+    flow-matching grid with shift s, sigma_hat_i = 1 - i/N and
+    sigma_i = s*sigma_hat_i / (1 + (s-1)*sigma_hat_i), computed in fp64 and
+    exchanged as fp32 (so sigma_0 = 1 and sigma_N = 0).
+    """
+    if n_steps < 1:
+        raise ValueError("n_steps must be >= 1")
+    i = np.arange(n_steps + 1, dtype=np.float64)
+    sh = 1.0 - i / n_steps
+    sig = shift * sh / (1.0 + (shift - 1.0) * sh)
+    return sig.astype(np.float32)
+
+
+def model_timestep(sigma) -> np.float32:
+    """Model timestep t_i fed to the denoiser: fp32(1000 * sigma_i) (reading; paper silent)."""
+    return np.float32(np.float32(1000.0) * np.float32(sigma))
+
+
+def euler_update(x, p, sigma_t, sigma_next):
+    """Scheduler update S of Eq. 2 for a flow-matching velocity p, with empty history h_i.
+
+    x_{t_{i+1}} = x_{t_i} + (sigma_{i+1} - sigma_i) * p.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    return x + (float(sigma_next) - float(sigma_t)) * np.asarray(p, dtype=np.float64)
+
+
+# ---------------------------------------------------------------------------
+# Guidance (Eq. 1)
+# ---------------------------------------------------------------------------
+
+
+def guided(f_cond, f_uncond, w):
+    """Eq. 1: p = f(x, t, empty) + w * (f(x, t, tau) - f(x, t, empty)).
+
+    With w == 1 the unconditional branch cancels exactly; the caller may then
+    pass f_uncond=None and the conditional prediction is returned unchanged.
+    """
+    f_cond = np.asarray(f_cond, dtype=np.float64)
+    if float(w) == 1.0:
+        return f_cond.copy()
+    f_uncond = np.asarray(f_uncond, dtype=np.float64)
+    return f_uncond + float(w) * (f_cond - f_uncond)
+
+
+# ---------------------------------------------------------------------------
+# Disagreement (Eq. 4) and mean score (Eq. 5)
+# ---------------------------------------------------------------------------
+
+
+def disagreement(p_large, p_small, eps: float = 1e-8) -> float:
+    """Eq. 4: r = ||p_S - p_L||_2 / max(||p_L||_2, eps), norms over the whole latent of one sample."""
+    pl = np.asarray(p_large, dtype=np.float64).ravel()
+    ps = np.asarray(p_small, dtype=np.float64).ravel()
+    num = math.sqrt(float(np.dot(ps - pl, ps - pl)))
+    den = max(math.sqrt(float(np.dot(pl, pl))), eps)
+    return num / den
+
+
+def mean_score(r) -> np.ndarray:
+    """Eq. 5: q_k = (1/M) sum_j r_{j,k}; r has shape [M, N].  Returned as fp32."""
+    r = np.asarray(r, dtype=np.float64)
+    M = r.shape[0]
+    acc = np.zeros(r.shape[1], dtype=np.float64)
+    for j in range(M):            # summed in calibration-sample order
+        acc = acc + r[j]
+    return (acc / M).astype(np.float32)
+
+
+# ---------------------------------------------------------------------------
+# Policy: relaxation (Eq. 6-7) and top-K switching (Sec. 3.2.3)
+# ---------------------------------------------------------------------------
+
+
+def relaxed_objective(beta, q, c0) -> float:
+    """Eq. 6 objective sum_k (W_k - C0) * beta_k with W_k = q_k^2."""
+    q = np.asarray(q, dtype=np.float64)
+    return float(np.sum((q * q - c0) * np.asarray(beta, dtype=np.float64)))
+
+
+def threshold_policy(q, c0) -> np.ndarray:
+    """Eq. 7: beta_k = 1 where W_k < C0, 0 where W_k > C0 (0 chosen where W_k == C0)."""
+    q = np.asarray(q, dtype=np.float64)
+    return (q * q < c0).astype(np.uint8)
+
+
+def topk_policy(q, k: int) -> np.ndarray:
+    """Top-K switching (Sec. 3.2.3): route the K steps with the lowest q_k to the small model.
+
+    Returns uint8[N] with 1 = small (S), 0 = large (L).  Ranking is on q itself
+    (equivalent to W = q^2 for q >= 0).  Ties at the K/K+1 boundary, where the
+    paper allows any optimal choice, go to the lower step index.
+    """
+    q = np.asarray(q, dtype=np.float32)
+    n = q.shape[0]
+    if not (0 <= k <= n):
+        raise ValueError("K must satisfy 0 <= K <= N")
+    if np.any(np.isnan(q)) or np.any(q < 0):
+        raise ValueError("scores must be non-negative numbers")
+    order = sorted(range(n), key=lambda i: (float(q[i]), i))
+    pol = np.zeros(n, dtype=np.uint8)
+    for i in order[:k]:
+        pol[i] = 1
+    return pol
+
+
+def brute_force_topk(q, k: int) -> np.ndarray:
+    """Exhaustive search over all C(N, K) subsets for the minimum of sum_{k in set} q_k^2.
+
+    Among optimal subsets the lexicographically smallest sorted index tuple wins.
+    Only for small N (test pin of ``topk_policy``).
+    """
+    q = [float(v) for v in np.asarray(q, dtype=np.float32)]
+    n = len(q)
+    best, best_set = None, None
+    for combo in itertools.combinations(range(n), k):
+        cost = sum(q[i] * q[i] for i in combo)
+        if best is None or cost < best or (cost == best and combo < best_set):
+            best, best_set = cost, combo
+    pol = np.zeros(n, dtype=np.uint8)
+    for i in best_set:
+        pol[i] = 1
+    return pol
+
+
+def first_k_policy(n: int, k: int) -> np.ndarray:
+    """Equal-budget baseline First-K (Sec. 4.5, Table 2): the first K steps go to the small model."""
+    pol = np.zeros(n, dtype=np.uint8)
+    pol[:k] = 1
+    return pol
+
+
+def last_k_policy(n: int, k: int) -> np.ndarray:
+    """Equal-budget baseline Last-K (Sec. 4.5, Table 2): the last K steps go to the small model."""
+    pol = np.zeros(n, dtype=np.uint8)
+    if k:
+        pol[n - k:] = 1
+    return pol
+
+
+# ---------------------------------------------------------------------------
+# Denoiser evaluation, calibration (Sec. 3.2.1) and routed sampling (Eq. 3)
+# ---------------------------------------------------------------------------
+
+
+def guided_prediction(model, x, sigma, cond, uncond, w, counter=None):
+    """p_m(x_t, t) of Eq. 1 for one sample, evaluating f_m on tau (and on the negative prompt if w != 1)."""
+    t = model_timestep(sigma)
+    f_c = model.forward(x, t, cond)
+    if counter is not None:
+        counter[model.name] = counter.get(model.name, 0) + 1
+    if float(w) == 1.0:
+        return guided(f_c, None, w)
+    f_u = model.forward(x, t, uncond)
+    if counter is not None:
+        counter[model.name] += 1
+    return guided(f_c, f_u, w)
+
+
+def calibrate(large, small, x_T, conds, unconds, w, sigmas, eps: float = 1e-8):
+    """Reference-trajectory calibration (Sec. 3.2.1) followed by Eq. 4 scoring.
+
+    For every calibration sample j the trajectory is rolled out with the large
+    model only.  Before each update both models are evaluated on the same
+    latent x_{t_k}, timestep, conditioning and guidance; r[j, k] records their
+    relative disagreement and the large model's prediction advances x.
+    Returns (r [M, N] float64, final latents [M, ...] float64).
+    """
+    M = len(x_T)
+    N = len(sigmas) - 1
+    r = np.zeros((M, N), dtype=np.float64)
+    finals = []
+    for j in range(M):
+        x = np.asarray(x_T[j], dtype=np.float64)
+        u = None if unconds is None else unconds[j]
+        for k in range(N):
+            p_l = guided_prediction(large, x, sigmas[k], conds[j], u, w)
+            p_s = guided_prediction(small, x, sigmas[k], conds[j], u, w)
+            r[j, k] = disagreement(p_l, p_s, eps)
+            x = euler_update(x, p_l, sigmas[k], sigmas[k + 1])
+        finals.append(x)
+    return r, np.stack(finals)
+
+
+def sample_routed(large, small, policy, x_T, cond, uncond, w, sigmas, counter=None):
+    """Eq. 3: x_{t_{i+1}} = S(x_{t_i}, p_{pi(i)}(x_{t_i}, t_i), t_i, h_i), one denoiser per step."""
+    x = np.asarray(x_T, dtype=np.float64)
+    for i in range(len(sigmas) - 1):
+        m = small if policy[i] else large
+        p = guided_prediction(m, x, sigmas[i], cond, uncond, w, counter)
+        x = euler_update(x, p, sigmas[i], sigmas[i + 1])
+    return x

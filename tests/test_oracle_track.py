@@ -1,0 +1,252 @@
+"""Pins of the oracle's method functions (Eq. 1-7, Sec. 3.2.1, Sec. 3.3) against what the paper fixes.
+
+Each test checks the oracle against something other than itself: closed forms,
+invariants, special cases and brute force.  No GPU is needed.
+"""
+import itertools
+import math
+
+import numpy as np
+import pytest
+
+import synth
+from oracle import dit, track
+
+# ---------------------------------------------------------------------------
+# Scheduler grid and update (Eq. 2 instance)
+# ---------------------------------------------------------------------------
+
+
+@pytest.mark.parametrize("n", [1, 2, 4, 8, 30, 50])
+@pytest.mark.parametrize("shift", [1.0, 3.0, 5.0])
+def test_schedule_endpoints_and_decreasing(n, shift):
+    s = track.schedule(n, shift)
+    assert s.dtype == np.float32 and s.shape == (n + 1,)
+    assert s[0] == 1.0 and s[-1] == 0.0
+    assert np.all(np.diff(s.astype(np.float64)) < 0)
+
+
+def test_schedule_shift_one_is_uniform():
+    s = track.schedule(8, 1.0)
+    assert np.array_equal(s, np.float32([1, 0.875, 0.75, 0.625, 0.5, 0.375, 0.25, 0.125, 0]))
+
+
+def test_schedule_shift_scales_the_odds():
+    # The shifted grid multiplies the noise odds sigma/(1-sigma) of the uniform grid by s.
+    n, s = 10, 5.0
+    sig = track.schedule(n, s).astype(np.float64)[1:-1]
+    u = 1.0 - np.arange(1, n) / n
+    assert np.allclose(sig / (1 - sig), s * u / (1 - u), rtol=1e-6)
+    # mid-grid closed form: sigma_hat = 1/2 -> s/(s+1)
+    assert abs(float(track.schedule(8, s)[4]) - s / (s + 1)) < 1e-7
+
+
+def test_euler_constant_field_sums_the_grid():
+    # sum of (sigma_{i+1} - sigma_i) over the grid is sigma_N - sigma_0 = -1
+    sig = track.schedule(7, 5.0)
+    x = np.array([0.3, -1.0, 2.0])
+    c = np.array([1.5, -0.25, 4.0])
+    for i in range(7):
+        x = track.euler_update(x, c, sig[i], sig[i + 1])
+    assert np.allclose(x, np.array([0.3, -1.0, 2.0]) - c, atol=1e-12)
+
+
+def test_euler_integrates_the_straight_path_exactly():
+    # x_sigma = (1 - sigma) x0 + sigma eps has constant velocity eps - x0;
+    # starting from eps at sigma_0 = 1, Euler lands on x0 at sigma_N = 0.
+    rng = np.random.default_rng(0)
+    x0, eps = rng.normal(size=50), rng.normal(size=50)
+    sig = track.schedule(13, 5.0)
+    x = eps.copy()
+    for i in range(13):
+        x = track.euler_update(x, eps - x0, sig[i], sig[i + 1])
+    assert np.allclose(x, x0, atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# Guidance (Eq. 1)
+# ---------------------------------------------------------------------------
+
+
+def test_cfg_special_cases():
+    rng = np.random.default_rng(1)
+    fc, fu = rng.normal(size=20), rng.normal(size=20)
+    assert np.array_equal(track.guided(fc, None, 1.0), fc)          # w = 1: uncond not needed
+    assert np.array_equal(track.guided(fc, fu * np.nan, 1.0), fc)   # ... and not read
+    assert np.allclose(track.guided(fc, fu, 0.0), fu)                # w = 0: unconditional
+    assert np.allclose(track.guided(fc, fc, 7.5), fc)                # equal branches
+    # affine in w with slope f_c - f_u
+    assert np.allclose(track.guided(fc, fu, 3.0) - track.guided(fc, fu, 2.0), fc - fu)
+
+
+# ---------------------------------------------------------------------------
+# Disagreement (Eq. 4) and mean score (Eq. 5)
+# ---------------------------------------------------------------------------
+
+
+def test_disagreement_special_cases():
+    rng = np.random.default_rng(2)
+    pl = rng.normal(size=(4, 3, 5))
+    assert track.disagreement(pl, pl) == 0.0
+    assert track.disagreement(pl, np.zeros_like(pl)) == pytest.approx(1.0, abs=1e-15)
+    assert track.disagreement(pl, 2 * pl) == pytest.approx(1.0, abs=1e-14)
+    assert track.disagreement(pl, -pl) == pytest.approx(2.0, abs=1e-14)
+    ps = rng.normal(size=pl.shape)
+    r = track.disagreement(pl, ps)
+    assert track.disagreement(3.5 * pl, 3.5 * ps) == pytest.approx(r, rel=1e-14)
+    assert r >= 0
+    # p_L = 0: the denominator is clamped to eps
+    assert track.disagreement(np.zeros(6), np.full(6, 0.5), eps=1e-3) == pytest.approx(
+        math.sqrt(6 * 0.25) / 1e-3, rel=1e-14)
+
+
+def test_disagreement_brute_force():
+    rng = np.random.default_rng(3)
+    pl, ps = rng.normal(size=17), rng.normal(size=17)
+    num = 0.0
+    den = 0.0
+    for a, b in zip(pl.tolist(), ps.tolist()):
+        num += (b - a) * (b - a)
+        den += a * a
+    assert track.disagreement(pl, ps) == pytest.approx(math.sqrt(num) / math.sqrt(den), rel=1e-13)
+
+
+def test_mean_score_hand_values():
+    q = track.mean_score([[1.0, 2.0, 0.5], [3.0, 4.0, 0.25]])
+    assert q.dtype == np.float32
+    assert np.array_equal(q, np.float32([2.0, 3.0, 0.375]))
+
+
+# ---------------------------------------------------------------------------
+# Policy (Eq. 6-7 and top-K)
+# ---------------------------------------------------------------------------
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_topk_matches_brute_force(seed):
+    rng = np.random.default_rng(seed)
+    n = int(rng.integers(1, 11))
+    q = rng.uniform(0, 1, size=n).astype(np.float32)
+    if seed % 2:                      # many ties
+        q = np.round(q * 3).astype(np.float32) / 3
+    for k in range(n + 1):
+        assert np.array_equal(track.topk_policy(q, k), track.brute_force_topk(q, k)), (q, k)
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_topk_equals_threshold_solution(seed):
+    # Choosing C0 strictly between the K-th and (K+1)-th smallest W = q^2 makes the
+    # threshold solution of Eq. 7 select exactly the top-K set, and it is optimal for Eq. 6.
+    rng = np.random.default_rng(100 + seed)
+    n = 12
+    q = rng.uniform(0, 1, size=n).astype(np.float32)
+    w = np.sort(q.astype(np.float64) ** 2)
+    for k in range(1, n):
+        c0 = 0.5 * (w[k - 1] + w[k])
+        pol = track.topk_policy(q, k)
+        assert np.array_equal(track.threshold_policy(q, c0), pol)
+        best = track.relaxed_objective(pol, q, c0)
+        for combo in itertools.combinations(range(n), k):
+            beta = np.zeros(n)
+            beta[list(combo)] = 1
+            assert track.relaxed_objective(beta, q, c0) >= best - 1e-15
+
+
+def test_topk_extremes_and_errors():
+    q = np.float32([0.3, 0.1, 0.2])
+    assert np.array_equal(track.topk_policy(q, 0), [0, 0, 0])
+    assert np.array_equal(track.topk_policy(q, 3), [1, 1, 1])
+    assert np.array_equal(track.topk_policy(q, 1), [0, 1, 0])
+    assert np.array_equal(track.topk_policy(np.float32([0.5, 0.5, 0.5]), 2), [1, 1, 0])
+    for bad_k in (-1, 4):
+        with pytest.raises(ValueError):
+            track.topk_policy(q, bad_k)
+    with pytest.raises(ValueError):
+        track.topk_policy(np.float32([0.1, np.nan]), 1)
+    with pytest.raises(ValueError):
+        track.topk_policy(np.float32([0.1, -0.2]), 1)
+
+
+def test_topk_on_paper_shaped_score_maps():
+    n, k = 50, 25
+    i = np.arange(n)
+    # U-shaped map with its minimum in the latter half (Sec. 4.4, Fig. 3): a contiguous middle block
+    u = (0.6 * ((i - 31) / 31.0) ** 2 + 0.05).astype(np.float32)
+    sel = np.flatnonzero(track.topk_policy(u, k))
+    assert np.all(np.diff(sel) == 1) and sel[0] > 0 and sel[-1] < n - 1
+    assert sel.mean() > n / 2 - 1
+    # monotone decreasing map (distilled pipelines, App. B): the last K steps
+    m = np.linspace(1.0, 0.1, n).astype(np.float32)
+    assert np.array_equal(track.topk_policy(m, k), track.last_k_policy(n, k))
+
+
+# ---------------------------------------------------------------------------
+# Calibration and routed sampling with a tiny denoiser pair
+# ---------------------------------------------------------------------------
+
+ARCH_L = synth.Arch(dim=32, layers=2, heads=2, ffn=64, text_dim=24, text_len=5,
+                    frames=2, height=4, width=6)
+ARCH_S = synth.Arch(dim=16, layers=1, heads=1, ffn=32, text_dim=24, text_len=5,
+                    frames=2, height=4, width=6)
+
+
+@pytest.fixture(scope="module")
+def pair():
+    L = dit.DiT(ARCH_L, synth.make_weights(ARCH_L, 11), name="L")
+    S = dit.DiT(ARCH_S, synth.make_weights(ARCH_S, 12), name="S")
+    return L, S
+
+
+@pytest.fixture(scope="module")
+def samples():
+    return synth.calibration_inputs(ARCH_L, 0, 2, with_uncond=True)
+
+
+def test_calibration_follows_the_all_large_trajectory(pair, samples):
+    # Sec. 3.2.1: the large model's prediction advances the trajectory, so the
+    # calibration latents are those of all-large sampling, bit for bit.
+    L, S = pair
+    x, c, u = samples
+    sig = track.schedule(4, 5.0)
+    r, finals = track.calibrate(L, S, x, c, u, 5.0, sig)
+    assert r.shape == (2, 4) and np.all(r > 0)
+    for j in range(2):
+        ref = track.sample_routed(L, S, np.zeros(4, np.uint8), x[j], c[j], u[j], 5.0, sig)
+        assert np.array_equal(finals[j], ref)
+
+
+def test_identical_pair_has_zero_disagreement(samples):
+    L = dit.DiT(ARCH_L, synth.make_weights(ARCH_L, 11), name="L")
+    S = dit.DiT(ARCH_L, synth.make_weights(ARCH_L, 11), name="S")
+    x, c, u = samples
+    r, _ = track.calibrate(L, S, x, c, u, 5.0, track.schedule(3, 5.0))
+    assert np.all(r == 0.0)
+
+
+def test_routed_sampling_extremes_and_one_model_per_step(pair, samples):
+    L, S = pair
+    x, c, u = samples
+    sig = track.schedule(5, 5.0)
+    all_l = track.sample_routed(L, S, np.zeros(5, np.uint8), x[0], c[0], u[0], 5.0, sig)
+    assert np.array_equal(track.sample_routed(L, S, track.topk_policy(np.ones(5, np.float32), 0),
+                                              x[0], c[0], u[0], 5.0, sig), all_l)
+    all_s = track.sample_routed(L, S, np.ones(5, np.uint8), x[0], c[0], u[0], 5.0, sig)
+    ref_s = track.sample_routed(S, L, np.zeros(5, np.uint8), x[0], c[0], u[0], 5.0, sig)
+    assert np.array_equal(all_s, ref_s)
+    pol = np.uint8([0, 1, 1, 0, 1])
+    cnt = {}
+    track.sample_routed(L, S, pol, x[0], c[0], u[0], 5.0, sig, counter=cnt)
+    assert cnt == {"L": 2 * 2, "S": 3 * 2}     # cond + uncond of exactly one model per step
+    cnt = {}
+    track.sample_routed(L, S, pol, x[0], c[0], None, 1.0, sig, counter=cnt)
+    assert cnt == {"L": 2, "S": 3}             # w = 1: no unconditional pass
+
+
+def test_mutation_flipped_disagreement_ratio_is_caught():
+    # A plausible slip (normalising by the small model's norm) fails the p_S = 0 pin.
+    def wrong(pl, ps, eps=1e-8):
+        pl, ps = np.ravel(pl), np.ravel(ps)
+        return math.sqrt(np.dot(ps - pl, ps - pl)) / max(math.sqrt(np.dot(ps, ps)), eps)
+    pl = np.ones(4)
+    assert track.disagreement(pl, np.zeros(4)) == pytest.approx(1.0)
+    assert wrong(pl, np.zeros(4)) != pytest.approx(1.0)
