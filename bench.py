@@ -1,0 +1,394 @@
+"""Benchmark of TRACK's routed denoising hot path on GB300.
+
+One benchmark step is one routed sampling trajectory (Eq. 3) of one request on
+the mid workload: a 1536-wide 30-block large DiT and a 768-wide 12-block small
+DiT (bf16, weights generated on the device), latent 16x9x30x52 (3510 tokens),
+text 512x4096, 4 flow-matching Euler steps, no CFG, and the policy that top-K
+(K=2) derives from a calibration run (Sec. 3.2.1, Eq. 4-5) on 8 seeds, which is
+executed and timed once before the timed region.  Each step projects its
+request's text, runs the 4 routed denoiser evaluations and the fused guidance +
+Euler updates.
+
+Printed metric: routed denoise steps/s (whole job over all ranks), plus the
+all-large latency and the routed speedup, DiT TFLOPS, the roofline of the
+dominant kernel class measured with CUDA events inside the timed region, an
+end-to-end number through the C ABI with host buffers, clocks sampled during
+the timed region, and the oracle's CPU throughput on a bounded sample.
+
+    python bench.py [--steps K] [--warmup W] [--gpus N] [--impl ours|reference]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+WORKLOAD = "mid"
+METRIC = "routed denoise steps/s"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    try:
+        with open(PEAKS_FILE) as f:
+            p = json.load(f)
+        return p, "measured"
+    except Exception:
+        return FALLBACK_PEAKS, "fallback"
+
+
+def forward_flops(arch, batch):
+    """Algorithmic FLOPs of one denoiser evaluation of `batch` sequences (text work excluded)."""
+    L, d, F, Lt, l = arch.tokens, arch.dim, arch.ffn, arch.text_len, arch.layers
+    per = l * (2 * L * (6 * d * d + 2 * d * F) + 4 * L * L * d + 4 * L * Lt * d) + 4 * L * 64 * d
+    return batch * per
+
+
+def text_flops(arch, batch):
+    """Once per request and model: text projection and the blocks' cross-attention K/V."""
+    Lt, d, Dt, l = arch.text_len, arch.dim, arch.text_dim, arch.layers
+    return batch * (2 * Lt * Dt * d + 2 * Lt * d * d + l * 2 * Lt * d * 2 * d)
+
+
+class ClockSampler:
+    """Samples SM clocks and throttle reasons with nvidia-smi while running."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        try:
+            for line in open(self.path):
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 8 and parts[0].replace(".", "").isdigit():
+                    rows.append(parts)
+        except Exception:
+            pass
+        finally:
+            try:
+                os.unlink(self.path)
+            except Exception:
+                pass
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        sm = [float(r[0]) for r in rows]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[4 + i].lower() == "active"})
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": float(rows[0][1]),
+                "power_w_max": max(float(r[2]) for r in rows if r[2].replace(".", "").isdigit()),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ---------------------------------------------------------------- CPU oracle sample
+class OracleSample:
+    """The oracle on a bounded sample of the workload: one full-size DiT block of each
+    model (fp64 numpy), timed and extrapolated to one routed trajectory."""
+
+    def __init__(self, wl):
+        from oracle import dit
+
+        self.wl = wl
+        rng = np.random.default_rng(0)
+        self.parts = {}
+        for which, arch, seed in (("large", wl.large, synth.SEED_LARGE),
+                                  ("small", wl.small, synth.SEED_SMALL)):
+            specs = [s for s in synth.weight_specs(arch)
+                     if not s.name.startswith("blk") or s.name.startswith("blk0.")]
+            w = {s.name: synth.make_tensor(s, seed) for s in specs}
+            m = dit.DiT(synth.Arch(**{**arch.__dict__, "layers": 1}), w, "bf16")
+            x = rng.normal(size=(arch.tokens, arch.dim))
+            _, e0 = m.time_embedding(np.float32(500.0))
+            c = m.text_projection(synth.draw(1, 0, (arch.text_len, arch.text_dim), 1.0))
+            self.parts[which] = (m, x, e0, c, arch.layers)
+        self.description = (
+            f"one full-size DiT block of each model (oracle, fp64 numpy, {wl.large.tokens} tokens) "
+            f"per step, extrapolated x layers x routed evaluations ({wl.steps - wl.k} large + "
+            f"{wl.k} small); embedding, head and text work not included")
+
+    def seconds_per_trajectory(self):
+        t = {}
+        for which, (m, x, e0, c, layers) in self.parts.items():
+            t0 = time.perf_counter()
+            m.block(0, x, e0, c)
+            t[which] = (time.perf_counter() - t0) * layers
+        guided = 1 if self.wl.cfg == 1.0 else 2
+        return guided * ((self.wl.steps - self.wl.k) * t["large"] + self.wl.k * t["small"])
+
+
+def cpu_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads") for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    return os.cpu_count()
+
+
+# ---------------------------------------------------------------- reference arm
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    wl = synth.WORKLOADS[WORKLOAD]
+    sampler = OracleSample(wl)
+    for _ in range(args.warmup):
+        sampler.seconds_per_trajectory()
+    times = [sampler.seconds_per_trajectory() for _ in range(args.steps)]
+    desc = sampler.description
+    sec = float(np.mean(times))
+    value = wl.steps / sec
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "steps/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": sec * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": wl.description, "global_batch": 1, "seq_len": wl.large.tokens},
+        "cpu_baseline": {"value": value, "unit": "steps/s", "cores": cpu_threads(),
+                         "kind": "oracle", "sample": desc},
+        "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+# ---------------------------------------------------------------- our arm
+def run_ours(args):
+    import torch
+    import torch.distributed as tdist
+
+    import paper_2609_30096_gb300 as T
+    from paper_2609_30096_gb300 import _build
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        tdist.init_process_group("nccl")
+    _build.build()
+
+    wl = synth.WORKLOADS[WORKLOAD]
+    B = wl.batch
+    w = wl.cfg
+    sig = T.track_schedule(wl.steps, wl.shift)
+    L = T.track_model_create_seeded(wl.large, synth.SEED_LARGE, T.BF16)
+    S = T.track_model_create_seeded(wl.small, synth.SEED_SMALL, T.BF16)
+    uses_uncond = w != 1.0
+
+    # --- offline calibration on wl.calib_seeds seeds (batched), untimed in the step
+    xc, cc, uc = synth.calibration_inputs(wl.large, 0, wl.calib_seeds, uses_uncond)
+    dev = torch.device("cuda", local)
+    xcd = torch.from_numpy(xc).to(dev)
+    ccd = torch.from_numpy(cc).to(dev)
+    ucd = torch.from_numpy(uc).to(dev) if uses_uncond else None
+    stream = torch.cuda.current_stream()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    r = T.track_calibrate(L, S, xcd, ccd, ucd, w, sig)
+    ev1.record(stream)
+    T.track_sync()
+    calib_ms = ev0.elapsed_time(ev1)
+    q = T.track_mean_score(r.cpu().numpy().T)
+    policy = T.track_policy_topk(q, wl.k)
+    del xcd, ccd, ucd, r
+
+    # --- request inputs: per-rank disjoint evaluation seeds
+    x0, c0, u0 = synth.evaluation_inputs(wl.large, rank * B, B, uses_uncond)
+    xh = torch.from_numpy(x0).pin_memory()
+    ch = torch.from_numpy(c0).pin_memory()
+    uh = torch.from_numpy(u0).pin_memory() if uses_uncond else None
+    xd = torch.empty_like(xh, device=dev)
+    cd = ch.to(dev)
+    ud = uh.to(dev) if uses_uncond else None
+    out_h = torch.empty_like(xh).pin_memory()
+
+    x_init = xh.to(dev)
+
+    def step_device(pol):
+        xd.copy_(x_init)                          # on-device reset of the latent
+        T.track_invalidate_ctx(L)
+        T.track_invalidate_ctx(S)
+        T.track_sample(L, S, pol, sig, xd, cd, ud, w)
+
+    def step_e2e(pol):
+        xd.copy_(xh, non_blocking=True)           # host -> device: latent and text
+        cd.copy_(ch, non_blocking=True)
+        if uses_uncond:
+            ud.copy_(uh, non_blocking=True)
+        T.track_invalidate_ctx(L)
+        T.track_invalidate_ctx(S)
+        T.track_sample(L, S, pol, sig, xd, cd, ud, w)
+        out_h.copy_(xd, non_blocking=True)        # device -> host: the sample
+
+    def timed(fn, pol, steps, profile=False):
+        if world > 1:
+            tdist.barrier()
+        torch.cuda.synchronize()
+        T.track_profile_enable(profile)
+        n0 = T.track_launch_count()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(steps):
+            fn(pol)
+        b.record(stream)
+        torch.cuda.synchronize()
+        T.track_profile_enable(False)
+        T.track_sync()
+        ms = a.elapsed_time(b)
+        launches = T.track_launch_count() - n0
+        if world > 1:
+            t = torch.tensor([ms], device=dev)
+            tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+            if world > 1:
+                tdist.barrier()
+            ms = float(t.item())
+        return ms, launches
+
+    for _ in range(args.warmup):
+        step_device(policy)
+    torch.cuda.synchronize()
+    T.track_profile_read()                         # drop any stale records
+
+    with ClockSampler(local) as clk:
+        ms, launches = timed(step_device, policy, args.steps, profile=True)
+    clocks = clk.summary()
+    prof = T.track_profile_read()
+
+    all_l = np.zeros(wl.steps, np.uint8)
+    for _ in range(max(1, args.warmup // 2)):
+        step_device(all_l)
+    ms_all_large, _ = timed(step_device, all_l, args.steps)
+    for _ in range(max(1, args.warmup // 2)):
+        step_e2e(policy)
+    ms_e2e, _ = timed(step_e2e, policy, args.steps)
+
+    per_step_ms = ms / args.steps
+    value = world * wl.steps * B * args.steps / (ms / 1e3)
+    e2e_value = world * wl.steps * B * args.steps / (ms_e2e / 1e3)
+    n_small = int(policy.sum())
+    n_large = wl.steps - n_small
+    guided = 1 if w == 1.0 else 2
+    fl = (n_large * forward_flops(wl.large, guided * B) + n_small * forward_flops(wl.small, guided * B)
+          + (text_flops(wl.large, guided * B) if n_large else 0)
+          + (text_flops(wl.small, guided * B) if n_small else 0))
+    tflops = fl / (per_step_ms / 1e3) / 1e12
+
+    peaks, src = load_peaks()
+    gm, gf, gn = prof["gemm"]
+    am, af, an = prof["attention"]
+    dominant = "gemm" if gm >= am else "attention"
+    dm, dflops, dn = prof[dominant]
+    achieved = (dflops / dn) / (dm / dn / 1e3) / 1e12 if dn else None
+    peak = peaks["bf16_tflops"]
+    traffic = None
+    roof = {"bound": "tensor", "kernel": "bf16 GEMM (tcgen05)" if dominant == "gemm"
+            else "flash attention (bf16 mma.sync)",
+            "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+            "frac": achieved / peak if achieved else None, "traffic": traffic,
+            "peak_source": f"{src} bf16 burst (sustained {peaks.get('bf16_tflops_sustained')})",
+            "launches": int(dn), "avg_launch_ms": dm / dn if dn else None,
+            "share_of_step": dm / ms if ms else None,
+            "other": {("attention" if dominant == "gemm" else "gemm"):
+                      {"ms": am if dominant == "gemm" else gm,
+                       "tflops": ((af / (am / 1e3)) if dominant == "gemm" and am
+                                  else (gf / (gm / 1e3)) if gm else 0) / 1e12}}}
+
+    cpu = None
+    if rank == 0 and not args.skip_cpu:
+        sampler = OracleSample(wl)
+        sec = sampler.seconds_per_trajectory()
+        cpu = {"value": wl.steps / sec, "unit": "steps/s", "cores": cpu_threads(), "kind": "oracle",
+               "sample": sampler.description}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_step_ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic",
+            "config": {"workload": wl.description, "global_batch": world * B,
+                       "seq_len": wl.large.tokens, "parallelism": f"replicas x{world}",
+                       "l2": "inputs larger than L2: every step streams 2.8 GB of large-model "
+                             "and 0.24 GB of small-model bf16 weights through the 126 MB L2",
+                       "policy": "".join("S" if p else "L" for p in policy)},
+            "routed_ms": per_step_ms, "all_large_ms": ms_all_large / args.steps,
+            "speedup_vs_all_large": (ms_all_large / ms) if ms else None,
+            "ideal_flop_speedup": wl.steps / (n_large + n_small *
+                                              forward_flops(wl.small, 1) / forward_flops(wl.large, 1)),
+            "dit_tflops": tflops, "dit_frac_of_bf16_peak": tflops / peak,
+            "calibration_ms": calib_ms, "calibration_seeds": wl.calib_seeds,
+            "score_map": [float(v) for v in q],
+            "roofline": roof,
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_value, "unit": "steps/s",
+                    "h2d_bytes_per_step": int(xh.numel() * 4 + ch.numel() * 4 +
+                                              (uh.numel() * 4 if uses_uncond else 0)),
+                    "d2h_bytes_per_step": int(xh.numel() * 4)},
+            "gpu_launches": int(launches),
+            "clocks": clocks,
+        }
+        print(json.dumps(line))
+    if world > 1:
+        tdist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--skip-cpu", action="store_true", help="omit the oracle CPU baseline")
+    args = ap.parse_args()
+    args.warmup = max(3, args.warmup)     # at least three untimed warm-up steps
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

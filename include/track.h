@@ -1,0 +1,246 @@
+/*
+ * track.h - C ABI of the GB300 (sm_103a) implementation of TRACK's routed
+ * denoising hot path ("Accelerating Video Diffusion via Training-Free
+ * Trajectory Routing").
+ *
+ * Conventions for every entry point:
+ *  - Every function returns an int status (TRACK_OK = 0 or a TRACK_E* code)
+ *    unless stated otherwise.  No function aborts, prints or throws; the text
+ *    of the last error on the calling thread is returned by track_last_error().
+ *  - "device" pointers are CUDA device memory owned by the caller, 16-byte
+ *    aligned, and are read/written in stream order on the given stream
+ *    (a cudaStream_t passed as void*; NULL means the legacy default stream).
+ *    Calls return once the work is enqueued; asynchronous device errors
+ *    surface at the next call that synchronizes, or at track_sync().
+ *  - "host" pointers are ordinary host memory, read/written before return.
+ *  - Latents are fp32 [B, C, F, H, W] (C = 16), contiguous.  Text
+ *    conditioning is fp32 [B, Lt, Dtxt], contiguous.
+ *  - Models with dtype TRACK_BF16 keep weight matrices and activations in
+ *    bf16 and accumulate in fp32 on the tensor cores; TRACK_FP32 models run
+ *    true fp32 (FFMA) arithmetic throughout (no TF32).
+ */
+#ifndef TRACK_H
+#define TRACK_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ------------------------------------------------------ */
+#define TRACK_OK 0
+#define TRACK_EINVAL 1       /* bad argument (NULL, shape, range, NaN score ...) */
+#define TRACK_ENOMEM 2       /* device or host allocation failed */
+#define TRACK_ECUDA 3        /* a CUDA runtime/driver call failed */
+#define TRACK_EUNSUPPORTED 4 /* valid request this build does not support */
+#define TRACK_ETIMEOUT 5     /* a device pipeline wait ran out (kernel gave up) */
+
+#define TRACK_FP32 0
+#define TRACK_BF16 1
+
+/* Epilogues of track_linear (Y = X W^T + b, then): */
+#define TRACK_EPI_STORE 0      /* Y stored in the model dtype                     */
+#define TRACK_EPI_GELU 1       /* GELU_tanh(Y) stored in the model dtype          */
+#define TRACK_EPI_RESID_GATE 2 /* fp32 R[m,n] += gate[n] * Y[m,n]                 */
+#define TRACK_EPI_RESID 3      /* fp32 R[m,n] += Y[m,n]                           */
+
+typedef void* track_stream; /* a cudaStream_t */
+
+/*
+ * Architecture of one denoiser f_m (the black box of Eq. 1).  The paper fixes
+ * no internals (Sec. 3.1, "Compatible model pairs": the pair shares latent,
+ * output shape, conditioning interface and prediction target; architectures
+ * may differ).  This library implements a Wan-style video DiT: patch 1x2x2,
+ * adaLN-modulated self-attention with 3D RoPE and RMSNorm(q, k) over the model
+ * width, cross-attention to the projected text, GELU_tanh MLP, modulated head.
+ * Requirements: dim % heads == 0, head_dim = dim/heads in {64, 128},
+ * in_ch * 4 == 64, frames/height/width divisible by the patch, dim, ffn and
+ * text_dim multiples of 64, freq_dim == 256.
+ */
+typedef struct track_arch {
+  int dim;      /* model width d                      */
+  int layers;   /* transformer blocks                 */
+  int heads;    /* attention heads                    */
+  int ffn;      /* MLP hidden width                   */
+  int text_dim; /* Dtxt, width of the text input      */
+  int text_len; /* Lt, text tokens per sample         */
+  int in_ch;    /* latent channels C (16)             */
+  int frames;   /* latent F                           */
+  int height;   /* latent H                           */
+  int width;    /* latent W                           */
+  int patch_f, patch_h, patch_w; /* must be 1, 2, 2   */
+  int freq_dim; /* timestep sinusoid width (256)      */
+  int dtype;    /* TRACK_FP32 or TRACK_BF16           */
+  float eps;    /* LayerNorm / RMSNorm epsilon (1e-6) */
+} track_arch;
+
+typedef struct track_model track_model;
+
+/* ---- library ----------------------------------------------------------- */
+
+/* Text of the last error on this thread ("" if none).  Never NULL. */
+const char* track_last_error(void);
+
+/* ABI version of this header (returns the integer, not a status). */
+int track_abi_version(void);
+
+/* Waits for all work on stream s and reports device-side errors: TRACK_ECUDA
+ * for a CUDA error, TRACK_ETIMEOUT if a kernel abandoned a pipeline wait
+ * (the flag is cleared by this call). */
+int track_sync(track_stream s);
+
+/* Number of kernels this library has launched since load (returns the count). */
+int64_t track_launch_count(void);
+
+/* Kernel timing: while enabled, GEMM and attention launches inside
+ * track_denoise/track_denoise_step/track_calibrate/track_sample are bracketed
+ * by CUDA events on their stream.  track_profile_read synchronizes those
+ * events and returns, per class (0 = GEMM, 1 = attention), the summed event
+ * time in ms, the summed algorithmic FLOPs and the number of launches, then
+ * clears the records.  Arrays are host, length 2. */
+int track_profile_enable(int enable);
+int track_profile_read(double* ms, double* flops, int64_t* launches);
+
+/* ---- models (Sec. 3.1 "Compatible model pairs") --------------------------- */
+
+/* Number of canonical weight tensors of arch (returns the count, or -1). */
+int track_weight_count(const track_arch* arch);
+
+/* Shape of canonical tensor `index` (rows, cols; cols = 1 for vectors).
+ * Canonical order: pe.W[d,64] pe.b[d] txt.W1[d,Dtxt] txt.b1 txt.W2[d,d] txt.b2
+ * tim.W1[d,256] tim.b1 tim.W2[d,d] tim.b2 mod.W[6d,d] mod.b[6d]; per block:
+ * mod_bias[6,d] q.W[d,d] q.b k.W k.b v.W v.b o.W o.b qn.g kn.g ln3.g ln3.b
+ * cq.W cq.b ck.W ck.b cv.W cv.b co.W co.b cqn.g ckn.g ffn.W1[F,d] ffn.b1[F]
+ * ffn.W2[d,F] ffn.b2[d]; then head_bias[2,d] head.W[64,d] head.b[64].
+ * Matrices are [out, in] row-major. */
+int track_weight_shape(const track_arch* arch, int index, int64_t* rows, int64_t* cols);
+
+/* Creates a model on the current CUDA device from host fp32 weights.
+ * weights[i] points to canonical tensor i (track_weight_count entries).  The
+ * library copies (and, for TRACK_BF16, rounds to nearest-even bf16) every
+ * matrix into device memory it owns; the caller may free the host arrays
+ * after return.  Synchronous.  EINVAL for an unsupported arch. */
+int track_model_create(const track_arch* arch, const float* const* weights, track_model** out);
+
+/* Same, with weights generated on the device by the library's counter-based
+ * generator (SplitMix64 stream per (seed, tensor index); approximately normal
+ * Irwin-Hall-4 draws; matrices N(0, 1/fan_in), biases N(0, 0.02^2), norm gains
+ * 1 + N(0, 0.05^2), LayerNorm offsets N(0, 0.05^2)).  The values are bit-for-bit
+ * those the repository's host generator produces for the same seed. */
+int track_model_create_seeded(const track_arch* arch, uint32_t seed, track_model** out);
+
+int track_model_destroy(track_model* m);
+
+/* Sec. 3.1: 1 if a and b can be interchanged within one trajectory (same
+ * latent shape, text interface and patch), 0 if not, negative on error. */
+int track_models_compatible(const track_model* a, const track_model* b);
+
+/* Drops the model's cache of projected text conditioning.  track_denoise
+ * caches the text projection and the per-block cross-attention keys/values
+ * keyed on the (cond, uncond, B) pointers it was last given; call this when
+ * the data behind the same pointers changes. */
+int track_invalidate_ctx(track_model* m);
+
+/* ---- denoiser and guidance (Eq. 1) --------------------------------------- */
+
+/* v_out = p_m(x_t, t) of Eq. 1 for B samples at model timestep t:
+ *   f(x_t, t, uncond) + cfg_scale * (f(x_t, t, cond) - f(x_t, t, uncond)).
+ * x_t, v_out: device fp32 [B, C, F, H, W]; cond, uncond: device fp32
+ * [B, Lt, Dtxt].  With cfg_scale == 1 the unconditional pass is skipped, v_out
+ * equals f(x_t, t, cond) exactly and uncond may be NULL (else EINVAL).
+ * cond and uncond are batched into one forward of 2B sequences.  v_out must
+ * not alias x_t.  The first call at a new B grows the model's workspace
+ * (cudaMalloc, synchronizing). */
+int track_denoise(track_model* m, const float* x_t, int B, float t, const float* cond,
+                  const float* uncond, float cfg_scale, float* v_out, track_stream s);
+
+/* One scheduler step with this denoiser (Eq. 2/Eq. 3 with the flow-matching
+ * Euler update): evaluates the model at t = 1000 * sigma_t and updates x in
+ * place, x += (sigma_next - sigma_t) * p, with the guidance combine fused into
+ * the update kernel. */
+int track_denoise_step(track_model* m, float* x, int B, float sigma_t, float sigma_next,
+                       const float* cond, const float* uncond, float cfg_scale, track_stream s);
+
+/* Eq. 1 combine on n elements: p = f_u + w * (f_c - f_u) (p = f_c if w == 1). */
+int track_cfg(const float* f_c, const float* f_u, int64_t n, float w, float* p_out,
+              track_stream s);
+
+/* ---- scheduler (Eq. 2, flow-matching Euler instance) ---------------------- */
+
+/* sigmas_out (host, n_steps + 1 floats): sigma_i = s*u/(1+(s-1)*u), u = 1 - i/N,
+ * computed in double and rounded to float; sigma_0 = 1, sigma_N = 0.  The
+ * model timestep of step i is t_i = 1000 * sigma_i. */
+int track_schedule(int n_steps, float shift, float* sigmas_out);
+
+/* In place x += (sigma_next - sigma_t) * v on n device floats (Eq. 2). */
+int track_step(float* x_t, const float* v, int64_t n, float sigma_t, float sigma_next,
+               track_stream s);
+
+/* Fused Eq. 1 + Eq. 2: x += (sigma_next - sigma_t) * (f_u + w (f_c - f_u)).
+ * f_u may be NULL when w == 1 (then p = f_c). */
+int track_cfg_step(float* x, const float* f_c, const float* f_u, int64_t n, float w,
+                   float sigma_t, float sigma_next, track_stream s);
+
+/* ---- calibration score (Eq. 4, Eq. 5) ------------------------------------ */
+
+/* Eq. 4 per sample b: r_b = ||v_S[b] - v_L[b]||_2 / max(||v_L[b]||_2, eps), norms
+ * over the n_per_sample elements of sample b; adds r_b to score_accum[b]
+ * (device, B floats).  Deterministic: identical inputs give bitwise-identical
+ * results (fixed-order two-level reduction, no floating-point atomics).
+ * Uses library-owned device scratch per (device, stream). */
+int track_disagreement(const float* v_L, const float* v_S, int B, int64_t n_per_sample,
+                       float eps, float* score_accum, track_stream s);
+
+/* Eq. 5 on the host: q[k] = (1/M) sum_j r[j*N + k] (r host [M, N]), summed in j
+ * order in double and rounded to float. */
+int track_mean_score(const float* r, int M, int N, float* q_out);
+
+/* ---- policy (Eq. 6, Eq. 7, top-K switching of Sec. 3.2.3) ------------------ */
+
+/* policy_out[k] = 1 (small model) for the K steps with the lowest score, else
+ * 0 (large model).  Ranking is on the fp32 score; ties at the K/K+1 boundary
+ * go to the lower step index.  EINVAL if K < 0, K > N, N < 1 or any score is
+ * NaN or negative.  Host only, bit-exact. */
+int track_policy_topk(const float* score_map, int N, int K, uint8_t* policy_out);
+
+/* ---- loops (Sec. 3.2.1 calibration, Eq. 3 routed sampling) ---------------- */
+
+/* Reference-trajectory calibration for B samples: for k in 0..n_steps-1,
+ * p_L = track_denoise(L), p_S = track_denoise(S) on the same x, then
+ * r_out[k*B + b] = Eq. 4 score, then x += (sigma_{k+1} - sigma_k) * p_L.
+ * x: device [B, ...] in/out (ends as the all-large sample); sigmas: host
+ * (n_steps + 1); r_out: device fp32 [n_steps, B] (overwritten). */
+int track_calibrate(track_model* large, track_model* small, float* x, int B, const float* cond,
+                    const float* uncond, float cfg_scale, const float* sigmas, int n_steps,
+                    float eps, float* r_out, track_stream s);
+
+/* Eq. 3: for i in 0..n_steps-1, the model policy[i] (0 = large, 1 = small)
+ * supplies p and x += (sigma_{i+1} - sigma_i) * p; exactly one model per step.
+ * policy, sigmas: host; x: device in/out. */
+int track_sample(track_model* large, track_model* small, const uint8_t* policy,
+                 const float* sigmas, int n_steps, float* x, int B, const float* cond,
+                 const float* uncond, float cfg_scale, track_stream s);
+
+/* ---- building blocks (the denoiser's kernels, for tests and benchmarks) --- */
+
+/* Y = X W^T + bias with an epilogue (TRACK_EPI_*).  dtype selects the kernel:
+ * TRACK_BF16 -> tcgen05 tensor-core GEMM (X bf16 [M,K], W bf16 [N,K], Y bf16
+ * or fp32 residual), TRACK_FP32 -> FFMA GEMM (all fp32).  out has leading
+ * dimension ldo (elements).  gate: fp32 [N] (RESID_GATE only); bias may be
+ * NULL.  Requires K % 64 == 0 and N % 32 == 0 for TRACK_BF16. */
+int track_linear(int dtype, const void* X, const void* W, const float* bias, int M, int N,
+                 int K, int epilogue, const float* gate, void* out, int ldo, track_stream s);
+
+/* O = softmax(Q K^T / sqrt(hd)) V per (sequence, head), no mask.  Q: [S, H, Lq,
+ * hd], K, V: [S, H, Lk, hd], O: [S, Lq, H, hd], all in dtype (bf16 or fp32);
+ * hd in {64, 128}. */
+int track_attention(int dtype, const void* Q, const void* K, const void* V, int S, int H,
+                    int Lq, int Lk, int hd, void* O, track_stream s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TRACK_H */

@@ -1,0 +1,544 @@
+// HBM-bound and small kernels of the denoiser and of the TRACK method:
+// weight conversion/generation, timestep embedding, adaLN modulation, patch
+// embedding, LayerNorm + modulation, RMSNorm + 3D RoPE + head split, head +
+// unpatchify, guidance (Eq. 1), Euler update (Eq. 2) and the disagreement
+// reduction (Eq. 4).
+#include <cuda_bf16.h>
+#include <math.h>
+
+#include "internal.h"
+
+namespace track {
+
+typedef __nv_bfloat16 bf16;
+
+__device__ __forceinline__ float ldv(const float* p, int64_t i) { return p[i]; }
+__device__ __forceinline__ float ldv(const bf16* p, int64_t i) { return __bfloat162float(p[i]); }
+__device__ __forceinline__ void stv(float* p, int64_t i, float v) { p[i] = v; }
+__device__ __forceinline__ void stv(bf16* p, int64_t i, float v) { p[i] = __float2bfloat16_rn(v); }
+
+static int grid_for(int64_t n, int per_block) {
+  int64_t g = (n + per_block - 1) / per_block;
+  int cap = 8 * num_sms();
+  return (int)(g < 1 ? 1 : (g > cap ? cap : g));
+}
+
+// Block-wide sum of one float per thread (blockDim.x a multiple of 32, <= 1024).
+__device__ float block_sum(float v, float* red) {
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31, nw = blockDim.x >> 5;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  float t = 0.f;
+  for (int i = 0; i < nw; ++i) t += red[i];  // same order in every thread
+  return t;
+}
+
+// ---------------------------------------------------------------- weights
+template <typename T>
+__global__ void k_convert(const float* __restrict__ src, T* __restrict__ dst, int64_t n) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    stv(dst, i, src[i]);
+}
+
+cudaError_t convert_f32(const float* src, void* dst, int dtype, int64_t n, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  const int g = grid_for(n, 256);
+  if (dtype == BF16) k_convert<bf16><<<g, 256, 0, s>>>(src, (bf16*)dst, n);
+  else k_convert<float><<<g, 256, 0, s>>>(src, (float*)dst, n);
+  count_launch();
+  return cudaGetLastError();
+}
+
+// SplitMix64 output mixing (Steele, Lea and Flood 2014).
+__device__ __forceinline__ uint64_t mix64(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// Element i = float(2 * (sum of the four 16-bit lanes of output i) - 262140) * scale
+// (+ offset), each step one correctly rounded fp32 operation.
+template <typename T>
+__global__ void k_seed(T* __restrict__ dst, uint64_t state, int64_t n, float scale, float offset,
+                       int has_offset) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const uint64_t z = mix64(state + (uint64_t)(i + 1) * 0x9E3779B97F4A7C15ull);
+    const int sum = (int)(z & 0xFFFFu) + (int)((z >> 16) & 0xFFFFu) + (int)((z >> 32) & 0xFFFFu) +
+                    (int)(z >> 48);
+    float v = __fmul_rn((float)(2 * sum - 262140), scale);
+    if (has_offset) v = __fadd_rn(v, offset);
+    stv(dst, i, v);
+  }
+}
+
+cudaError_t seed_fill(void* dst, int dtype, uint64_t state, int64_t n, float scale, float offset,
+                      int has_offset, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  const int g = grid_for(n, 256);
+  if (dtype == BF16) k_seed<bf16><<<g, 256, 0, s>>>((bf16*)dst, state, n, scale, offset, has_offset);
+  else k_seed<float><<<g, 256, 0, s>>>((float*)dst, state, n, scale, offset, has_offset);
+  count_launch();
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- timestep embedding
+__global__ void k_sinusoid(float t, float* emb, int dim) {
+  const int half = dim / 2;
+  for (int i = threadIdx.x; i < dim; i += blockDim.x) {
+    const int j = i < half ? i : i - half;
+    const double a = (double)t * pow(10000.0, -(double)j / (double)half);
+    emb[i] = (float)(i < half ? cos(a) : sin(a));
+  }
+}
+
+cudaError_t sinusoid(float t, float* emb, int freq_dim, cudaStream_t s) {
+  k_sinusoid<<<1, 256, 0, s>>>(t, emb, freq_dim);
+  count_launch();
+  return cudaGetLastError();
+}
+
+// One warp per output row: coalesced reads of W's row.
+template <typename T>
+__global__ void k_matvec(const T* __restrict__ W, const float* __restrict__ in,
+                         const float* __restrict__ b, float* __restrict__ out, int rows, int cols,
+                         int silu_in) {
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  float acc = 0.f;
+  const T* w = W + (int64_t)row * cols;
+  for (int k = lane; k < cols; k += 32) {
+    float v = in[k];
+    if (silu_in) v = v / (1.f + expf(-v));
+    acc = fmaf(ldv(w, k), v, acc);
+  }
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  if (lane == 0) out[row] = acc + (b ? b[row] : 0.f);
+}
+
+cudaError_t matvec(const void* W, int dtype, const float* in, const float* b, float* out, int rows,
+                   int cols, int silu_in, cudaStream_t s) {
+  const int g = (rows * 32 + 255) / 256;
+  if (dtype == BF16) k_matvec<bf16><<<g, 256, 0, s>>>((const bf16*)W, in, b, out, rows, cols, silu_in);
+  else k_matvec<float><<<g, 256, 0, s>>>((const float*)W, in, b, out, rows, cols, silu_in);
+  count_launch();
+  return cudaGetLastError();
+}
+
+__global__ void k_modulation(const float* __restrict__ e0, const float* __restrict__ mod_bias,
+                             int layers, const float* __restrict__ e,
+                             const float* __restrict__ head_bias, int d, float* __restrict__ mod_all,
+                             float* __restrict__ head_mod) {
+  const int64_t n1 = (int64_t)layers * 6 * d;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n1 + 2 * d;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    if (i < n1) mod_all[i] = e0[i % (6 * d)] + mod_bias[i];
+    else {
+      const int64_t j = i - n1;
+      head_mod[j] = e[j % d] + head_bias[j];
+    }
+  }
+}
+
+cudaError_t modulation(const float* e0, const float* mod_bias, int layers, const float* e,
+                       const float* head_bias, int d, float* mod_all, float* head_mod,
+                       cudaStream_t s) {
+  const int64_t n = (int64_t)layers * 6 * d + 2 * d;
+  k_modulation<<<grid_for(n, 256), 256, 0, s>>>(e0, mod_bias, layers, e, head_bias, d, mod_all,
+                                                head_mod);
+  count_launch();
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- patch embedding
+// Row r = seq * L + tok; token tok = (f, h', w') row-major; patch vector ordered (c, ph, pw).
+constexpr int PE_TOK = 8;
+
+template <typename T>
+__global__ void __launch_bounds__(256) k_patch_embed(const float* __restrict__ x, int B, int rows,
+                                                     int C, int F, int H, int W,
+                                                     const T* __restrict__ Wpe,
+                                                     const float* __restrict__ bpe, int d,
+                                                     float* __restrict__ xres) {
+  __shared__ float patch[PE_TOK][64];
+  const int Hp = H / 2, Wp = W / 2, L = F * Hp * Wp;
+  const int r0 = blockIdx.x * PE_TOK;
+  for (int i = threadIdx.x; i < PE_TOK * 64; i += blockDim.x) {
+    const int t = i / 64, k = i % 64, r = r0 + t;
+    float v = 0.f;
+    if (r < rows && k < C * 4) {
+      const int seq = r / L, tok = r % L, smp = seq % B;
+      const int f = tok / (Hp * Wp), hp = (tok / Wp) % Hp, wp = tok % Wp;
+      const int c = k / 4, ph = (k / 2) % 2, pw = k % 2;
+      v = x[((((int64_t)smp * C + c) * F + f) * H + 2 * hp + ph) * W + 2 * wp + pw];
+    }
+    patch[t][k] = v;
+  }
+  __syncthreads();
+  const int P = C * 4;
+  for (int n = threadIdx.x; n < d; n += blockDim.x) {
+    float acc[PE_TOK];
+#pragma unroll
+    for (int t = 0; t < PE_TOK; ++t) acc[t] = 0.f;
+    const T* w = Wpe + (int64_t)n * P;
+    for (int k = 0; k < P; ++k) {
+      const float wk = ldv(w, k);
+#pragma unroll
+      for (int t = 0; t < PE_TOK; ++t) acc[t] = fmaf(wk, patch[t][k], acc[t]);
+    }
+    const float bb = bpe[n];
+#pragma unroll
+    for (int t = 0; t < PE_TOK; ++t)
+      if (r0 + t < rows) xres[(int64_t)(r0 + t) * d + n] = acc[t] + bb;
+  }
+}
+
+cudaError_t patch_embed(const float* x, int B, int nseq, int C, int F, int H, int W, const void* Wpe,
+                        int dtype, const float* bpe, int d, float* xres, cudaStream_t s) {
+  const int rows = nseq * F * (H / 2) * (W / 2);
+  const int g = (rows + PE_TOK - 1) / PE_TOK;
+  if (dtype == BF16)
+    k_patch_embed<bf16><<<g, 256, 0, s>>>(x, B, rows, C, F, H, W, (const bf16*)Wpe, bpe, d, xres);
+  else
+    k_patch_embed<float><<<g, 256, 0, s>>>(x, B, rows, C, F, H, W, (const float*)Wpe, bpe, d, xres);
+  count_launch();
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- LayerNorm + modulation
+constexpr int LN_MAXV = 24;  // d <= 24 * blockDim
+
+template <typename T>
+__global__ void __launch_bounds__(256) k_ln_mod(const float* __restrict__ x, int d,
+                                                const float* __restrict__ a,
+                                                const float* __restrict__ b, int mode, float eps,
+                                                T* __restrict__ out) {
+  __shared__ float red[32];
+  const int64_t row = blockIdx.x;
+  const float* xr = x + row * d;
+  float v[LN_MAXV];
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < LN_MAXV; ++i) {
+    const int j = threadIdx.x + i * blockDim.x;
+    v[i] = j < d ? xr[j] : 0.f;
+    s += v[i];
+  }
+  const float mean = block_sum(s, red) / (float)d;
+  float q = 0.f;
+#pragma unroll
+  for (int i = 0; i < LN_MAXV; ++i) {
+    const int j = threadIdx.x + i * blockDim.x;
+    const float c = j < d ? v[i] - mean : 0.f;
+    q = fmaf(c, c, q);
+  }
+  const float var = block_sum(q, red) / (float)d;
+  const float rstd = 1.f / sqrtf(var + eps);
+  T* orow = out + row * d;
+#pragma unroll
+  for (int i = 0; i < LN_MAXV; ++i) {
+    const int j = threadIdx.x + i * blockDim.x;
+    if (j < d) {
+      const float m = mode == 0 ? 1.f + a[j] : a[j];
+      stv(orow, j, fmaf((v[i] - mean) * rstd, m, b[j]));
+    }
+  }
+}
+
+cudaError_t ln_modulate(const float* x, int M, int d, const float* a, const float* b, int mode,
+                        float eps, void* out, int dtype, cudaStream_t s) {
+  if (d > LN_MAXV * 256) return cudaErrorInvalidValue;
+  const int threads = d >= 2048 ? 256 : (d >= 512 ? 128 : 64);
+  if (d > LN_MAXV * threads) return cudaErrorInvalidValue;
+  if (dtype == BF16) k_ln_mod<bf16><<<M, threads, 0, s>>>(x, d, a, b, mode, eps, (bf16*)out);
+  else k_ln_mod<float><<<M, threads, 0, s>>>(x, d, a, b, mode, eps, (float*)out);
+  count_launch();
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- RMSNorm + RoPE + head split
+// One block per row.  For each present section (q, k, v): load d values, optionally
+// RMSNorm over d with gain, optionally rotate (q, k) pairs, write head-major.
+template <typename T>
+__global__ void __launch_bounds__(256) k_qkv_prep(PrepArgs a) {
+  extern __shared__ float buf[];  // d floats
+  __shared__ float red[32];
+  const int r = blockIdx.x;
+  const int seq = r / a.L, l = r % a.L;
+  const T* src = (const T*)a.src + (int64_t)r * a.ld;
+  const int half = a.hd / 2;
+  const int s6 = a.hd / 6;
+  const int nf = (a.hd - 4 * s6) / 2, nh = s6;  // pairs per axis: frame, height (width = nh)
+  const int pf = l / (a.Hp * a.Wp), ph = (l / a.Wp) % a.Hp, pw = l % a.Wp;
+  for (int sec = 0; sec < 3; ++sec) {
+    if (a.dst[sec] == nullptr) continue;  // uniform across the block
+    const T* sp = src + a.off[sec];
+    float ss = 0.f;
+    for (int j = threadIdx.x; j < a.d; j += blockDim.x) {
+      const float v = ldv(sp, j);
+      buf[j] = v;
+      ss = fmaf(v, v, ss);
+    }
+    float rstd = 1.f;
+    if (a.gain[sec] != nullptr) {
+      const float tot = block_sum(ss, red);
+      rstd = 1.f / sqrtf(tot / (float)a.d + a.eps);
+    } else {
+      __syncthreads();
+    }
+    const float* g = a.gain[sec];
+    T* dst = (T*)a.dst[sec];
+    const bool rot = a.rope && sec < 2;
+    for (int p = threadIdx.x; p < a.d / 2; p += blockDim.x) {
+      const int h = p / half, j = p % half;
+      const int e = 2 * j;
+      float x0 = buf[h * a.hd + e], x1 = buf[h * a.hd + e + 1];
+      if (g) {
+        x0 = x0 * rstd * g[h * a.hd + e];
+        x1 = x1 * rstd * g[h * a.hd + e + 1];
+      }
+      if (rot) {
+        int idx;
+        if (j < nf) idx = pf * nf + j;
+        else if (j < nf + nh) idx = a.Fp * nf + ph * nh + (j - nf);
+        else idx = a.Fp * nf + a.Hp * nh + pw * nh + (j - nf - nh);
+        const float2 cs = a.rope_tab[idx];
+        const float y0 = x0 * cs.x - x1 * cs.y;
+        const float y1 = x0 * cs.y + x1 * cs.x;
+        x0 = y0;
+        x1 = y1;
+      }
+      const int64_t o = (((int64_t)seq * a.H + h) * a.L + l) * a.hd + e;
+      stv(dst, o, x0);
+      stv(dst, o + 1, x1);
+    }
+    __syncthreads();  // buf reused by the next section
+  }
+}
+
+cudaError_t qkv_prep(const PrepArgs& a, cudaStream_t s) {
+  const size_t sm = (size_t)a.d * sizeof(float);
+  if (sm > 48 * 1024) return cudaErrorInvalidValue;
+  if (a.dtype == BF16) k_qkv_prep<bf16><<<a.rows, 256, sm, s>>>(a);
+  else k_qkv_prep<float><<<a.rows, 256, sm, s>>>(a);
+  count_launch();
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- head + unpatchify
+template <typename T>
+__global__ void __launch_bounds__(256) k_head(const float* __restrict__ xres, int L, int d,
+                                              const float* __restrict__ head_mod,
+                                              const T* __restrict__ Wh,
+                                              const float* __restrict__ bh, float eps, int C, int F,
+                                              int H, int W, float* __restrict__ out) {
+  extern __shared__ float h[];  // d floats
+  __shared__ float red[32];
+  const int r = blockIdx.x;
+  const float* xr = xres + (int64_t)r * d;
+  float s = 0.f;
+  for (int j = threadIdx.x; j < d; j += blockDim.x) {
+    h[j] = xr[j];
+    s += h[j];
+  }
+  const float mean = block_sum(s, red) / (float)d;
+  float q = 0.f;
+  for (int j = threadIdx.x; j < d; j += blockDim.x) {
+    const float c = h[j] - mean;
+    q = fmaf(c, c, q);
+  }
+  const float rstd = 1.f / sqrtf(block_sum(q, red) / (float)d + eps);
+  for (int j = threadIdx.x; j < d; j += blockDim.x)
+    h[j] = fmaf((h[j] - mean) * rstd, 1.f + head_mod[d + j], head_mod[j]);
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  const int seq = r / L, tok = r % L;
+  const int Hp = H / 2, Wp = W / 2;
+  const int f = tok / (Hp * Wp), hp = (tok / Wp) % Hp, wp = tok % Wp;
+  const int P = C * 4;
+  for (int o = warp; o < P; o += nw) {
+    const T* w = Wh + (int64_t)o * d;
+    float acc = 0.f;
+    for (int j = lane; j < d; j += 32) acc = fmaf(ldv(w, j), h[j], acc);
+    for (int k = 16; k > 0; k >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, k);
+    if (lane == 0) {
+      const int c = o / 4, ph = (o / 2) % 2, pw = o % 2;
+      out[((((int64_t)seq * C + c) * F + f) * H + 2 * hp + ph) * W + 2 * wp + pw] = acc + bh[o];
+    }
+  }
+}
+
+cudaError_t head_unpatchify(const float* xres, int nseq, int L, int d, const float* head_mod,
+                            const void* Whead, int dtype, const float* bhead, float eps, int C,
+                            int F, int H, int W, float* out, cudaStream_t s) {
+  const size_t sm = (size_t)d * sizeof(float);
+  if (sm > 48 * 1024) return cudaErrorInvalidValue;
+  const int rows = nseq * L;
+  if (dtype == BF16)
+    k_head<bf16><<<rows, 256, sm, s>>>(xres, L, d, head_mod, (const bf16*)Whead, bhead, eps, C, F, H,
+                                       W, out);
+  else
+    k_head<float><<<rows, 256, sm, s>>>(xres, L, d, head_mod, (const float*)Whead, bhead, eps, C, F,
+                                        H, W, out);
+  count_launch();
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- guidance and Euler update
+// Explicitly rounded operations (no contraction) so that the fused and the separate
+// kernels produce bitwise-identical latents.
+__device__ __forceinline__ float cfg_val(float fc, float fu, float w) {
+  return __fadd_rn(fu, __fmul_rn(w, __fsub_rn(fc, fu)));
+}
+__device__ __forceinline__ float euler_val(float x, float p, float dsig) {
+  return __fadd_rn(x, __fmul_rn(dsig, p));
+}
+
+// mode 0: p = cfg(fc, fu)                  -> out
+// mode 1: x = x + dsig * v                 (v = fc)
+// mode 2: x = x + dsig * cfg(fc, fu)       (fu == nullptr: p = fc)
+__global__ void k_guide(float* __restrict__ x, const float* __restrict__ fc,
+                        const float* __restrict__ fu, float* __restrict__ out, int64_t n, float w,
+                        float dsig, int mode) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int64_t n4 = n / 4;
+  const bool vec = ((((uintptr_t)x) | ((uintptr_t)fc) | ((uintptr_t)fu) | ((uintptr_t)out)) & 15) == 0;
+  int64_t i0 = 0;
+  if (vec) {
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n4; i += stride) {
+      const float4 c = reinterpret_cast<const float4*>(fc)[i];
+      float4 p = c;
+      if (fu != nullptr && mode != 1) {
+        const float4 u = reinterpret_cast<const float4*>(fu)[i];
+        p = make_float4(cfg_val(c.x, u.x, w), cfg_val(c.y, u.y, w), cfg_val(c.z, u.z, w),
+                        cfg_val(c.w, u.w, w));
+      }
+      if (mode == 0) {
+        reinterpret_cast<float4*>(out)[i] = p;
+      } else {
+        float4 xv = reinterpret_cast<float4*>(x)[i];
+        xv = make_float4(euler_val(xv.x, p.x, dsig), euler_val(xv.y, p.y, dsig),
+                         euler_val(xv.z, p.z, dsig), euler_val(xv.w, p.w, dsig));
+        reinterpret_cast<float4*>(x)[i] = xv;
+      }
+    }
+    i0 = n4 * 4;
+  }
+  for (int64_t i = i0 + blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += stride) {
+    float p = fc[i];
+    if (fu != nullptr && mode != 1) p = cfg_val(p, fu[i], w);
+    if (mode == 0) out[i] = p;
+    else x[i] = euler_val(x[i], p, dsig);
+  }
+}
+
+static cudaError_t launch_guide(float* x, const float* fc, const float* fu, float* out, int64_t n,
+                                float w, float dsig, int mode, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  k_guide<<<grid_for((n + 3) / 4, 256), 256, 0, s>>>(x, fc, fu, out, n, w, dsig, mode);
+  count_launch();
+  return cudaGetLastError();
+}
+
+cudaError_t cfg_combine(const float* fc, const float* fu, int64_t n, float w, float* p,
+                        cudaStream_t s) {
+  return launch_guide(nullptr, fc, w == 1.f ? nullptr : fu, p, n, w, 0.f, 0, s);
+}
+cudaError_t euler_step(float* x, const float* v, int64_t n, float dsig, cudaStream_t s) {
+  return launch_guide(x, v, nullptr, nullptr, n, 1.f, dsig, 1, s);
+}
+cudaError_t cfg_euler(float* x, const float* fc, const float* fu, int64_t n, float w, float dsig,
+                      cudaStream_t s) {
+  return launch_guide(x, fc, w == 1.f ? nullptr : fu, nullptr, n, w, dsig, 2, s);
+}
+
+// ---------------------------------------------------------------- disagreement (Eq. 4)
+// Pass 1: grid (nblk, B); block j of sample b sums (vS - vL)^2 and vL^2 over a fixed
+// strided subset in fp32 and writes both to scratch[(b * nblk + j) * 2 + {0, 1}].
+// Pass 2: one block per sample adds the nblk partials in a fixed order in fp64 and
+// accumulates r_b into accum[b].
+constexpr int DIS_THREADS = 256;
+
+__global__ void __launch_bounds__(DIS_THREADS) k_dis_partial(const float* __restrict__ vL,
+                                                             const float* __restrict__ vS,
+                                                             int64_t n, float* __restrict__ part) {
+  __shared__ float red[32];
+  const int b = blockIdx.y, nblk = gridDim.x;
+  const float* l = vL + (int64_t)b * n;
+  const float* sp = vS + (int64_t)b * n;
+  float sd = 0.f, sl = 0.f;
+  const int64_t stride = (int64_t)nblk * DIS_THREADS;
+  const bool vec = ((((uintptr_t)l) | ((uintptr_t)sp)) & 15) == 0;
+  int64_t i0 = 0;
+  if (vec) {
+    const int64_t n4 = n / 4;
+    for (int64_t i = blockIdx.x * (int64_t)DIS_THREADS + threadIdx.x; i < n4; i += stride) {
+      const float4 a = reinterpret_cast<const float4*>(l)[i];
+      const float4 c = reinterpret_cast<const float4*>(sp)[i];
+      float t;
+      t = c.x - a.x; sd = fmaf(t, t, sd); sl = fmaf(a.x, a.x, sl);
+      t = c.y - a.y; sd = fmaf(t, t, sd); sl = fmaf(a.y, a.y, sl);
+      t = c.z - a.z; sd = fmaf(t, t, sd); sl = fmaf(a.z, a.z, sl);
+      t = c.w - a.w; sd = fmaf(t, t, sd); sl = fmaf(a.w, a.w, sl);
+    }
+    i0 = n4 * 4;
+  }
+  for (int64_t i = i0 + blockIdx.x * (int64_t)DIS_THREADS + threadIdx.x; i < n; i += stride) {
+    const float t = sp[i] - l[i];
+    sd = fmaf(t, t, sd);
+    sl = fmaf(l[i], l[i], sl);
+  }
+  const float td = block_sum(sd, red);
+  const float tl = block_sum(sl, red);
+  if (threadIdx.x == 0) {
+    part[((int64_t)b * nblk + blockIdx.x) * 2 + 0] = td;
+    part[((int64_t)b * nblk + blockIdx.x) * 2 + 1] = tl;
+  }
+}
+
+__global__ void __launch_bounds__(256) k_dis_final(const float* __restrict__ part, int nblk,
+                                                   float eps, float* __restrict__ accum) {
+  __shared__ double rd[256], rl[256];
+  const int b = blockIdx.x;
+  double sd = 0.0, sl = 0.0;
+  for (int j = threadIdx.x; j < nblk; j += 256) {
+    sd += (double)part[((int64_t)b * nblk + j) * 2 + 0];
+    sl += (double)part[((int64_t)b * nblk + j) * 2 + 1];
+  }
+  rd[threadIdx.x] = sd;
+  rl[threadIdx.x] = sl;
+  __syncthreads();
+  for (int w = 128; w > 0; w >>= 1) {
+    if (threadIdx.x < w) {
+      rd[threadIdx.x] += rd[threadIdx.x + w];
+      rl[threadIdx.x] += rl[threadIdx.x + w];
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    const double den = fmax(sqrt(rl[0]), (double)eps);
+    accum[b] += (float)(sqrt(rd[0]) / den);
+  }
+}
+
+int disagreement_blocks(int64_t n_per_sample) {
+  int64_t want = (n_per_sample + DIS_THREADS * 16 - 1) / (DIS_THREADS * 16);
+  const int cap = 2 * num_sms();
+  if (want < 1) want = 1;
+  if (want > cap) want = cap;
+  return (int)want;
+}
+
+cudaError_t disagreement(const float* vL, const float* vS, int B, int64_t n, float eps,
+                         float* accum, float* scratch, int nblk, cudaStream_t s) {
+  if (B <= 0) return cudaSuccess;
+  k_dis_partial<<<dim3(nblk, B), DIS_THREADS, 0, s>>>(vL, vS, n, scratch);
+  k_dis_final<<<B, 256, 0, s>>>(scratch, nblk, eps, accum);
+  count_launch(2);
+  return cudaGetLastError();
+}
+
+}  // namespace track

@@ -1,0 +1,96 @@
+// Internal declarations shared by the CUDA translation units of libtrack.
+// Kernel launchers take device pointers and a stream and return cudaError_t.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace track {
+
+enum Dtype { F32 = 0, BF16 = 1 };
+enum Epi { EPI_STORE = 0, EPI_GELU = 1, EPI_RESID_GATE = 2, EPI_RESID = 3 };
+
+// Error word written by kernels whose pipeline waits ran out (0 = none).
+// One per device, zeroed at first use; read and cleared by track_sync.
+int* device_error_word();
+
+// Counts every kernel launch made by the library.
+void count_launch(int n = 1);
+
+// ---------------------------------------------------------------- GEMM
+struct GemmArgs {
+  int M, N, K;
+  int epi;             // Epi
+  const float* bias;   // [N] or nullptr
+  const float* gate;   // [N] (EPI_RESID_GATE)
+  void* out;           // T [M, ldo] (STORE/GELU) or fp32 [M, ldo] (RESID*)
+  int ldo;
+  int* err;            // device error word
+};
+
+// fp32 FFMA GEMM: out = A[M,K] . W[N,K]^T (+ epilogue), all fp32.
+cudaError_t gemm_f32(const float* A, const float* W, const GemmArgs& g, cudaStream_t s);
+
+// bf16 tcgen05 GEMM: A bf16 [M,K] and W bf16 [N,K], fp32 accumulation in TMEM.
+// Requires K % 64 == 0, N % 32 == 0 and 16-byte aligned A, W and out.
+cudaError_t gemm_bf16_tc(const void* A, const void* W, const GemmArgs& g, cudaStream_t s);
+
+// ---------------------------------------------------------------- attention
+// Q [S,H,Lq,hd], K/V [S,H,Lk,hd] -> O [S,Lq,H,hd].
+cudaError_t attention_f32(const float* Q, const float* K, const float* V, float* O, int S, int H,
+                          int Lq, int Lk, int hd, cudaStream_t s);
+cudaError_t attention_bf16(const void* Q, const void* K, const void* V, void* O, int S, int H,
+                           int Lq, int Lk, int hd, cudaStream_t s);
+
+// ---------------------------------------------------------------- elementwise
+cudaError_t convert_f32(const float* src, void* dst, int dtype, int64_t n, cudaStream_t s);
+cudaError_t seed_fill(void* dst, int dtype, uint64_t state, int64_t n, float scale,
+                      float offset, int has_offset, cudaStream_t s);
+// emb[freq_dim] = [cos(t f_i), sin(t f_i)], f_i = 10000^(-i/(freq_dim/2)) (double precision)
+cudaError_t sinusoid(float t, float* emb, int freq_dim, cudaStream_t s);
+// out[r] = b[r] + sum_k W[r,k] * act(in[k]); act = SiLU if silu_in else identity
+cudaError_t matvec(const void* W, int dtype, const float* in, const float* b, float* out, int rows,
+                   int cols, int silu_in, cudaStream_t s);
+// mod_all[l,6,d] = e0[6,d] + mod_bias[l,6,d];  head_mod[2,d] = e[d] + head_bias[2,d]
+cudaError_t modulation(const float* e0, const float* mod_bias, int layers, const float* e,
+                       const float* head_bias, int d, float* mod_all, float* head_mod,
+                       cudaStream_t s);
+// x_res[s*L + tok, :] = patch(x[s % B], tok) . W_pe^T + b_pe
+cudaError_t patch_embed(const float* x, int B, int nseq, int C, int F, int H, int W,
+                        const void* Wpe, int dtype, const float* bpe, int d, float* xres,
+                        cudaStream_t s);
+// out = LN(x) * (1 + scale) + shift (mode 0) or LN(x) * g + b (mode 1); out in dtype
+cudaError_t ln_modulate(const float* x, int M, int d, const float* a, const float* b, int mode,
+                        float eps, void* out, int dtype, cudaStream_t s);
+// Per row of src [rows, ld]: q/k/v sections at column offsets; optional RMSNorm over d with
+// gain, optional 3D RoPE; write head-major [nseq, H, L, hd].  Row r = seq * L + l.
+struct PrepArgs {
+  const void* src; int ld; int rows; int L; int H; int hd; int d;
+  int off[3];               // column offsets of q, k, v (-1 = absent)
+  const float* gain[3];     // RMSNorm gains (nullptr = no norm)
+  void* dst[3];             // head-major outputs (nullptr = absent)
+  int rope;                 // apply 3D RoPE to q and k
+  const float2* rope_tab;   // [(Fp + Hp + Wp) * hd/2] (cos, sin); see track_api.cu
+  int Fp, Hp, Wp;
+  float eps;
+  int dtype;
+};
+cudaError_t qkv_prep(const PrepArgs& a, cudaStream_t s);
+// Head: LN(x)*(1+scale)+shift, . head_W^T + head_b, unpatchify into out [nseq, C, F, H, W]
+cudaError_t head_unpatchify(const float* xres, int nseq, int L, int d, const float* head_mod,
+                            const void* Whead, int dtype, const float* bhead, float eps, int C,
+                            int F, int H, int W, float* out, cudaStream_t s);
+// Eq. 1 and Eq. 2 on n floats.
+cudaError_t cfg_combine(const float* fc, const float* fu, int64_t n, float w, float* p,
+                        cudaStream_t s);
+cudaError_t euler_step(float* x, const float* v, int64_t n, float dsig, cudaStream_t s);
+cudaError_t cfg_euler(float* x, const float* fc, const float* fu, int64_t n, float w, float dsig,
+                      cudaStream_t s);
+// Eq. 4: partial sums then a fixed-order final combine; scratch holds B*nblk*2 floats.
+int disagreement_blocks(int64_t n_per_sample);
+cudaError_t disagreement(const float* vL, const float* vS, int B, int64_t n, float eps,
+                         float* accum, float* scratch, int nblk, cudaStream_t s);
+
+int num_sms();
+
+}  // namespace track

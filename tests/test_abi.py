@@ -1,0 +1,92 @@
+"""The C ABI without a GPU: the library builds and loads, exports every symbol
+include/track.h declares, and its host-only entry points (schedule, mean score,
+top-K policy, weight layout, argument checks) agree with the oracle."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import synth
+from oracle import track as otrack
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def T():
+    from paper_2609_30096_gb300 import _build
+    _build.build()
+    import paper_2609_30096_gb300 as T
+    T.lib()
+    return T
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "track.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    src = re.sub(r"//[^\n]*", "", src)
+    names = set(re.findall(r"\b(track_[a-z0-9_]+)\s*\(", src))
+    return sorted(names)
+
+
+def test_every_declared_symbol_is_exported(T):
+    names = declared_functions()
+    assert len(names) >= 25
+    raw = ctypes.CDLL(T._LIB_PATH)
+    missing = [n for n in names if not hasattr(raw, n)]
+    assert not missing, missing
+    assert T.track_abi_version() == 1
+
+
+@pytest.mark.parametrize("n,shift", [(1, 5.0), (4, 5.0), (8, 5.0), (50, 5.0), (30, 3.0), (7, 1.0)])
+def test_schedule_matches_oracle_bitwise(T, n, shift):
+    assert np.array_equal(T.track_schedule(n, shift), otrack.schedule(n, shift))
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_policy_topk_bit_exact(T, seed):
+    rng = np.random.default_rng(seed)
+    n = int(rng.integers(1, 60))
+    q = rng.uniform(0, 1, n).astype(np.float32)
+    if seed % 2:
+        q = (np.round(q * 4) / 4).astype(np.float32)        # ties
+    for k in sorted({0, n, int(rng.integers(0, n + 1)), n // 2}):
+        assert np.array_equal(T.track_policy_topk(q, k), otrack.topk_policy(q, k))
+        if n <= 10:
+            assert np.array_equal(T.track_policy_topk(q, k), otrack.brute_force_topk(q, k))
+
+
+def test_policy_topk_rejects_bad_input(T):
+    q = np.float32([0.2, 0.1])
+    for bad in (dict(q=q, k=-1), dict(q=q, k=3), dict(q=np.float32([0.1, np.nan]), k=1),
+                dict(q=np.float32([0.1, -1.0]), k=1)):
+        with pytest.raises(T.TrackError) as e:
+            T.track_policy_topk(bad["q"], bad["k"])
+        assert e.value.code == T.TRACK_EINVAL
+
+
+def test_mean_score_matches_oracle(T):
+    r = np.random.default_rng(3).uniform(0, 2, (16, 50)).astype(np.float32)
+    assert np.array_equal(T.track_mean_score(r), otrack.mean_score(r))
+
+
+@pytest.mark.parametrize("name", ["tiny", "mid", "wan480"])
+def test_weight_layout_matches_generator(T, name):
+    for arch in (synth.WORKLOADS[name].large, synth.WORKLOADS[name].small):
+        specs = synth.weight_specs(arch)
+        assert T.track_weight_count(arch) == len(specs)
+        for s in specs:
+            r, c = T.track_weight_shape(arch, s.tensor_id)
+            assert (r, c) == (s.shape if len(s.shape) == 2 else (s.shape[0], 1)), s.name
+
+
+def test_arch_validation(T):
+    a = synth.WORKLOADS["tiny"].large
+    bad = synth.Arch(dim=96, layers=1, heads=3, ffn=128, text_dim=64, text_len=4,
+                     frames=2, height=4, width=4)       # head_dim 32 unsupported
+    with pytest.raises(T.TrackError):
+        T.track_weight_count(bad)
+    with pytest.raises(T.TrackError):
+        T.track_weight_shape(a, 10 ** 6)

@@ -1,0 +1,244 @@
+"""Kernel-level parity of the CUDA path against the oracle, through the C ABI.
+
+GEMM (tcgen05 bf16 and FFMA fp32, every epilogue, ragged tiles), attention
+(bf16 tensor-core and fp32), guidance / Euler update, the Eq. 4 reduction and
+on-device weight generation.
+"""
+import numpy as np
+import pytest
+
+import synth
+from oracle import dit, track
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def T():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_30096_gb300 import _build
+    _build.build()
+    import paper_2609_30096_gb300 as T
+    return T
+
+
+DEV = "cuda"
+
+
+def rel_l2(a, b):
+    a = np.asarray(a, np.float64)
+    b = np.asarray(b, np.float64)
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-300))
+
+
+def dev_f32(a):
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(DEV)
+
+
+def dev_bf16(a):
+    return dev_f32(a).to(torch.bfloat16)
+
+
+# ---------------------------------------------------------------- GEMM
+GEMM_SHAPES = [
+    (128, 256, 64),      # one tile
+    (200, 384, 128),     # ragged M, N not a multiple of 256 (128-wide tiles)
+    (1, 512, 256),       # a single row
+    (777, 1024, 640),    # ragged M, several 256-wide tiles, K not a power of two
+    (3510, 1536, 1536),  # mid-size output projection (bench shape)
+    (600, 8960, 1536),   # wide N (FFN up-projection)
+    (333, 1536, 8960),   # long K (FFN down-projection)
+]
+
+
+@pytest.mark.parametrize("M,N,K", GEMM_SHAPES)
+@pytest.mark.parametrize("epi", [0, 1, 2, 3])
+def test_linear_bf16_tcgen05(T, M, N, K, epi):
+    rng = np.random.default_rng(M * 7 + N * 3 + K + epi)
+    X = dit.round_bf16(rng.normal(size=(M, K)).astype(np.float32))
+    W = dit.round_bf16((rng.normal(size=(N, K)) / np.sqrt(K)).astype(np.float32))
+    b = rng.normal(size=N).astype(np.float32) * 0.1
+    gate = rng.normal(size=N).astype(np.float32)
+    ref = dit.linear(X, W, b)
+    if epi == T.EPI_GELU:
+        ref = dit.gelu_tanh(ref)
+    if epi in (T.EPI_STORE, T.EPI_GELU):
+        out = torch.zeros((M, N), dtype=torch.bfloat16, device=DEV)
+        T.track_linear(T.BF16, dev_bf16(X), dev_bf16(W), dev_f32(b), epi, out)
+        T.track_sync()
+        got = out.float().cpu().numpy()
+        assert rel_l2(got, ref) < 4e-3
+        assert np.all(np.abs(got - ref) <= 8e-3 * np.abs(ref) + 2e-3 * np.sqrt(np.mean(ref ** 2)))
+    else:
+        r0 = rng.normal(size=(M, N)).astype(np.float32)
+        out = dev_f32(r0)
+        T.track_linear(T.BF16, dev_bf16(X), dev_bf16(W), dev_f32(b), epi, out,
+                       gate=dev_f32(gate) if epi == T.EPI_RESID_GATE else None)
+        T.track_sync()
+        delta = out.cpu().numpy().astype(np.float64) - r0
+        want = ref * gate if epi == T.EPI_RESID_GATE else ref
+        assert rel_l2(delta, want) < 2e-5
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 32, 64), (100, 96, 80), (513, 700, 256)])
+@pytest.mark.parametrize("epi", [0, 1, 2, 3])
+def test_linear_fp32(T, M, N, K, epi):
+    rng = np.random.default_rng(M + N + K + epi)
+    X = rng.normal(size=(M, K)).astype(np.float32)
+    W = (rng.normal(size=(N, K)) / np.sqrt(K)).astype(np.float32)
+    b = rng.normal(size=N).astype(np.float32)
+    gate = rng.normal(size=N).astype(np.float32)
+    r0 = rng.normal(size=(M, N)).astype(np.float32)
+    out = dev_f32(r0)
+    T.track_linear(T.FP32, dev_f32(X), dev_f32(W), dev_f32(b), epi, out,
+                   gate=dev_f32(gate) if epi == 2 else None)
+    T.track_sync()
+    ref = dit.linear(X, W, b)
+    if epi == 1:
+        ref = dit.gelu_tanh(ref)
+    got = out.cpu().numpy().astype(np.float64)
+    if epi == 2:
+        got, ref = got - r0, ref * gate
+    elif epi == 3:
+        got = got - r0
+    assert rel_l2(got, ref) < 2e-6
+
+
+def test_linear_rejects_unsupported_bf16_shape(T):
+    X = torch.zeros((4, 96), dtype=torch.bfloat16, device=DEV)
+    W = torch.zeros((64, 96), dtype=torch.bfloat16, device=DEV)
+    out = torch.zeros((4, 64), dtype=torch.bfloat16, device=DEV)
+    with pytest.raises(T.TrackError) as e:
+        T.track_linear(T.BF16, X, W, None, 0, out)
+    assert e.value.code == T.TRACK_EUNSUPPORTED
+
+
+# ---------------------------------------------------------------- attention
+ATTN_CASES = [  # S, H, Lq, Lk, hd
+    (1, 1, 64, 64, 64),
+    (2, 3, 100, 100, 128),     # ragged query and key tiles
+    (1, 2, 257, 32, 64),       # short keys (tiny cross-attention)
+    (2, 2, 300, 512, 128),     # cross-attention at text length 512
+    (1, 12, 3510, 3510, 128),  # mid-size self-attention (bench shape)
+]
+
+
+def _attn_ref(Q, K, V):
+    S, H, Lq, hd = Q.shape
+    out = np.empty((S, Lq, H, hd))
+    for s in range(S):
+        for h in range(H):
+            out[s, :, h, :] = dit.attention(Q[s, h], K[s, h], V[s, h])
+    return out
+
+
+@pytest.mark.parametrize("S,H,Lq,Lk,hd", ATTN_CASES)
+def test_attention_bf16(T, S, H, Lq, Lk, hd):
+    rng = np.random.default_rng(Lq + Lk + hd)
+    Q = dit.round_bf16(rng.normal(size=(S, H, Lq, hd)).astype(np.float32))
+    K = dit.round_bf16(rng.normal(size=(S, H, Lk, hd)).astype(np.float32))
+    V = dit.round_bf16(rng.normal(size=(S, H, Lk, hd)).astype(np.float32))
+    O = torch.zeros((S, Lq, H, hd), dtype=torch.bfloat16, device=DEV)
+    T.track_attention(T.BF16, dev_bf16(Q), dev_bf16(K), dev_bf16(V), O)
+    T.track_sync()
+    if Lq * Lk > 2_000_000:          # large case: sampled query rows
+        rows = rng.choice(Lq, 64, replace=False)
+        ref = _attn_ref(Q[:, :, rows], K, V)
+        got = O.float().cpu().numpy()[:, rows]
+    else:
+        ref, got = _attn_ref(Q, K, V), O.float().cpu().numpy()
+    assert rel_l2(got, ref) < 1e-2
+
+
+@pytest.mark.parametrize("S,H,Lq,Lk,hd", ATTN_CASES[:4])
+def test_attention_fp32(T, S, H, Lq, Lk, hd):
+    rng = np.random.default_rng(Lq * 3 + Lk + hd)
+    Q, K, V = (rng.normal(size=(S, H, L, hd)).astype(np.float32) for L in (Lq, Lk, Lk))
+    O = torch.zeros((S, Lq, H, hd), dtype=torch.float32, device=DEV)
+    T.track_attention(T.FP32, dev_f32(Q), dev_f32(K), dev_f32(V), O)
+    T.track_sync()
+    assert rel_l2(O.cpu().numpy(), _attn_ref(Q, K, V)) < 2e-6
+
+
+def test_attention_single_key_returns_value_row(T):
+    rng = np.random.default_rng(5)
+    Q = rng.normal(size=(1, 2, 70, 64)).astype(np.float32)
+    K = rng.normal(size=(1, 2, 1, 64)).astype(np.float32)
+    V = dit.round_bf16(rng.normal(size=(1, 2, 1, 64)).astype(np.float32))
+    O = torch.zeros((1, 70, 2, 64), dtype=torch.bfloat16, device=DEV)
+    T.track_attention(T.BF16, dev_bf16(Q), dev_bf16(K), dev_bf16(V), O)
+    T.track_sync()
+    got = O.float().cpu().numpy()
+    for h in range(2):
+        assert np.array_equal(got[0, :, h, :], np.repeat(V[0, h], 70, 0))
+
+
+# ---------------------------------------------------------------- guidance, Euler, Eq. 4
+@pytest.mark.parametrize("n", [1, 3, 4096 + 3, 2_096_640])
+def test_guidance_and_euler(T, n):
+    rng = np.random.default_rng(n)
+    fc, fu, x = (rng.normal(size=n).astype(np.float32) for _ in range(3))
+    w, s0, s1 = 5.0, 0.8333333, 0.625
+    p = T.track_cfg(dev_f32(fc), dev_f32(fu), w)
+    T.track_sync()
+    assert rel_l2(p.cpu().numpy(), track.guided(fc, fu, w)) < 1e-6
+    p1 = T.track_cfg(dev_f32(fc), None, 1.0)
+    assert np.array_equal(p1.cpu().numpy(), fc)                   # w = 1: exactly f_c
+    xa = dev_f32(x)
+    T.track_step(xa, p, s0, s1)                                   # separate
+    xb = dev_f32(x)
+    T.track_cfg_step(xb, dev_f32(fc), dev_f32(fu), w, s0, s1)     # fused
+    T.track_sync()
+    assert torch.equal(xa, xb)
+    ref = track.euler_update(x, track.guided(fc, fu, w), np.float32(s0), np.float32(s1))
+    assert rel_l2(xa.cpu().numpy(), ref) < 1e-6
+
+
+@pytest.mark.parametrize("B,n", [(1, 1), (3, 5), (2, 4097), (8, 33_600), (1, 2_096_640)])
+def test_disagreement(T, B, n):
+    rng = np.random.default_rng(B * 1000 + n)
+    pl = rng.normal(size=(B, n)).astype(np.float32)
+    ps = (pl + 0.3 * rng.normal(size=(B, n))).astype(np.float32)
+    acc = dev_f32(np.full(B, 0.25, np.float32))
+    T.track_disagreement(dev_f32(pl), dev_f32(ps), acc)
+    T.track_sync()
+    got = acc.cpu().numpy() - 0.25                                # accumulates into the output
+    ref = [track.disagreement(pl[b], ps[b]) for b in range(B)]
+    assert np.max(np.abs(got - ref)) < 1e-5
+    again = dev_f32(np.full(B, 0.25, np.float32))
+    T.track_disagreement(dev_f32(pl), dev_f32(ps), again)
+    assert torch.equal(acc, again)                                # deterministic
+
+
+def test_disagreement_special_cases(T):
+    pl = np.random.default_rng(1).normal(size=(2, 1000)).astype(np.float32)
+    acc = torch.zeros(2, device=DEV)
+    T.track_disagreement(dev_f32(pl), dev_f32(pl), acc)
+    T.track_sync()
+    assert np.all(acc.cpu().numpy() == 0.0)                       # identical predictions
+    acc.zero_()
+    T.track_disagreement(dev_f32(pl), torch.zeros(2, 1000, device=DEV), acc)
+    T.track_sync()
+    assert np.allclose(acc.cpu().numpy(), 1.0, atol=1e-6)         # p_S = 0
+    acc.zero_()
+    T.track_disagreement(torch.zeros(2, 1000, device=DEV), dev_f32(pl), acc, eps=1e-3)
+    T.track_sync()
+    ref = np.linalg.norm(pl.astype(np.float64), axis=1) / 1e-3
+    assert np.allclose(acc.cpu().numpy(), ref, rtol=1e-6)         # p_L = 0: eps clamp
+
+
+# ---------------------------------------------------------------- on-device weights
+@pytest.mark.parametrize("dtype", [0, 1])
+def test_seeded_weights_equal_host_generator(T, dtype):
+    wl = synth.WORKLOADS["tiny"]
+    arch = wl.small
+    host = T.track_model_create(arch, list(synth.make_weights(arch, 77).values()), dtype)
+    seeded = T.track_model_create_seeded(arch, 77, dtype)
+    x, c, u = synth.evaluation_inputs(arch, 0, 2, with_uncond=True)
+    xd, cd, ud = dev_f32(x), dev_f32(c), dev_f32(u)
+    a = T.track_denoise(host, xd, 600.0, cd, ud, 5.0)
+    b = T.track_denoise(seeded, xd, 600.0, cd, ud, 5.0)
+    T.track_sync()
+    assert torch.equal(a, b)

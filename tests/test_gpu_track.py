@@ -1,0 +1,210 @@
+"""End-to-end parity of the routed denoising hot path against the oracle (GPU).
+
+Tiny pair (fp32 and bf16 modes): per-step guided predictions of both models
+(teacher-forced on the oracle's all-large trajectory), calibration scores,
+the policy derived from them, routed sampling, and the bit-exact identities
+the paper fixes (calibration follows the all-large trajectory; identical
+models disagree by exactly zero).  Mid pair (bf16, the benchmark workload at
+full size): per-step predictions of both models.
+"""
+import numpy as np
+import pytest
+
+import synth
+from oracle import dit, track
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+TOL = {"fp32": 1e-4, "bf16": 2e-2}      # relative L2 of per-step v
+SCORE_TOL = 1e-3                         # absolute, per-step disagreement
+
+
+@pytest.fixture(scope="module")
+def T():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_30096_gb300 import _build
+    _build.build()
+    import paper_2609_30096_gb300 as T
+    return T
+
+
+def rel_l2(a, b):
+    a = np.asarray(a, np.float64)
+    b = np.asarray(b, np.float64)
+    return float(np.linalg.norm(a - b) / np.linalg.norm(b))
+
+
+def dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).cuda()
+
+
+WL = synth.WORKLOADS["tiny"]
+
+
+class Pair:
+    def __init__(self, T, prec, wl=WL, small_seed=synth.SEED_SMALL, small_arch=None):
+        dtype = T.FP32 if prec == "fp32" else T.BF16
+        small_arch = small_arch or wl.small
+        wL = synth.make_weights(wl.large, synth.SEED_LARGE)
+        wS = synth.make_weights(small_arch, small_seed)
+        self.L = T.track_model_create(wl.large, list(wL.values()), dtype)
+        self.S = T.track_model_create(small_arch, list(wS.values()), dtype)
+        self.oL = dit.DiT(wl.large, wL, prec, name="L")
+        self.oS = dit.DiT(small_arch, wS, prec, name="S")
+
+
+@pytest.fixture(scope="module", params=["fp32", "bf16"])
+def tiny(T, request):
+    return request.param, Pair(T, request.param)
+
+
+@pytest.fixture(scope="module")
+def calib_inputs():
+    return synth.calibration_inputs(WL.large, 0, WL.calib_seeds, with_uncond=True)
+
+
+@pytest.fixture(scope="module")
+def oracle_calibration(tiny, calib_inputs):
+    prec, P = tiny
+    x, c, u = calib_inputs
+    sig = track.schedule(WL.steps, WL.shift)
+    # the all-large reference trajectory of every calibration sample, with r
+    traj = []
+    r = np.zeros((len(x), WL.steps))
+    for j in range(len(x)):
+        xs = [np.asarray(x[j], np.float64)]
+        for k in range(WL.steps):
+            pl = track.guided_prediction(P.oL, xs[-1], sig[k], c[j], u[j], WL.cfg)
+            ps = track.guided_prediction(P.oS, xs[-1], sig[k], c[j], u[j], WL.cfg)
+            r[j, k] = track.disagreement(pl, ps)
+            xs.append(track.euler_update(xs[-1], pl, sig[k], sig[k + 1]))
+        traj.append(xs)
+    return sig, traj, r
+
+
+def test_per_step_prediction_parity(T, tiny, calib_inputs, oracle_calibration):
+    """Teacher-forced: the GPU gets the oracle's x_{t_k}; v of both models within tolerance."""
+    prec, P = tiny
+    x, c, u = calib_inputs
+    sig, traj, _ = oracle_calibration
+    cd, ud = dev(c[:2]), dev(u[:2])
+    for k in range(WL.steps):
+        xk = np.stack([traj[j][k] for j in range(2)]).astype(np.float32)
+        t = float(track.model_timestep(sig[k]))
+        for gm, om in ((P.L, P.oL), (P.S, P.oS)):
+            v = T.track_denoise(gm, dev(xk), t, cd, ud, WL.cfg).cpu().numpy()
+            for j in range(2):
+                ref = track.guided_prediction(om, xk[j], sig[k], c[j], u[j], WL.cfg)
+                err = rel_l2(v[j], ref)
+                assert err < TOL[prec], (prec, om.name, k, j, err)
+
+
+def test_no_cfg_prediction_parity(T, tiny, calib_inputs):
+    prec, P = tiny
+    x, c, _ = calib_inputs
+    v = T.track_denoise(P.L, dev(x[:1]), 900.0, dev(c[:1]), None, 1.0).cpu().numpy()
+    ref = P.oL.forward(x[0], np.float32(900.0), c[0])
+    assert rel_l2(v[0], ref) < TOL[prec]
+
+
+def test_calibration_scores_and_policy(T, tiny, calib_inputs, oracle_calibration):
+    prec, P = tiny
+    x, c, u = calib_inputs
+    sig, traj, r_ref = oracle_calibration
+    xd = dev(x)
+    r = T.track_calibrate(P.L, P.S, xd, dev(c), dev(u), WL.cfg, sig)
+    T.track_sync()
+    r_gpu = r.cpu().numpy().T                                  # [M, N]
+    if prec == "fp32":
+        assert np.max(np.abs(r_gpu - r_ref)) < SCORE_TOL
+        # the calibration latents end on the oracle's all-large sample
+        for j in range(len(x)):
+            assert rel_l2(xd[j].cpu().numpy(), traj[j][-1]) < 1e-3
+    q_gpu = T.track_mean_score(r_gpu)
+    q_ref = track.mean_score(r_ref)
+    if prec == "fp32":
+        assert np.max(np.abs(q_gpu - q_ref)) < SCORE_TOL
+    # policy identical wherever the oracle's K-th / (K+1)-th gap exceeds the score tolerance
+    srt = np.sort(q_ref)
+    if srt[WL.k] - srt[WL.k - 1] > SCORE_TOL and prec == "fp32":
+        assert np.array_equal(T.track_policy_topk(q_gpu, WL.k), track.topk_policy(q_ref, WL.k))
+
+
+def test_calibration_trajectory_is_the_all_large_trajectory(T, tiny, calib_inputs):
+    """Sec. 3.2.1: the large model advances the calibration trajectory, so its latents
+    equal those of all-large routed sampling bit for bit."""
+    prec, P = tiny
+    x, c, u = calib_inputs
+    sig = track.schedule(WL.steps, WL.shift)
+    xa = dev(x)
+    T.track_calibrate(P.L, P.S, xa, dev(c), dev(u), WL.cfg, sig)
+    xb = dev(x)
+    T.track_sample(P.L, P.S, np.zeros(WL.steps, np.uint8), sig, xb, dev(c), dev(u), WL.cfg)
+    T.track_sync()
+    assert torch.equal(xa, xb)
+    xc = dev(x)                                               # K = 0 routed sample
+    T.track_sample(P.L, P.S, T.track_policy_topk(np.ones(WL.steps, np.float32), 0), sig, xc,
+                   dev(c), dev(u), WL.cfg)
+    T.track_sync()
+    assert torch.equal(xb, xc)
+
+
+def test_identical_models_have_zero_disagreement(T, calib_inputs):
+    P = Pair(T, "fp32", small_seed=synth.SEED_LARGE, small_arch=WL.large)
+    x, c, u = calib_inputs
+    r = T.track_calibrate(P.L, P.S, dev(x), dev(c), dev(u), WL.cfg, track.schedule(3, 5.0))
+    T.track_sync()
+    assert np.all(r.cpu().numpy() == 0.0)
+
+
+def test_routed_sampling_follows_the_oracle(T, tiny, calib_inputs, oracle_calibration):
+    prec, P = tiny
+    _, _, r_ref = oracle_calibration
+    pol = track.topk_policy(track.mean_score(r_ref), WL.k)
+    x, c, u = synth.evaluation_inputs(WL.large, 0, 2, with_uncond=True)
+    sig = track.schedule(WL.steps, WL.shift)
+    xd = dev(x)
+    T.track_sample(P.L, P.S, pol, sig, xd, dev(c), dev(u), WL.cfg)
+    T.track_sync()
+    cnt = {}
+    for j in range(2):
+        ref = track.sample_routed(P.oL, P.oS, pol, x[j], c[j], u[j], WL.cfg, sig, counter=cnt)
+        assert rel_l2(xd[j].cpu().numpy(), ref) < (1e-3 if prec == "fp32" else 5e-2)
+    assert cnt == {"L": 2 * 2 * int((pol == 0).sum()), "S": 2 * 2 * int(pol.sum())}
+
+
+def test_argument_errors(T, tiny, calib_inputs):
+    prec, P = tiny
+    x, c, u = calib_inputs
+    with pytest.raises(T.TrackError) as e:
+        T.track_denoise(P.L, dev(x[:1]), 500.0, dev(c[:1]), None, 5.0)   # uncond needed
+    assert e.value.code == T.TRACK_EINVAL
+    other = synth.Arch(dim=128, layers=1, heads=2, ffn=256, text_dim=256, text_len=32,
+                       frames=4, height=8, width=16)
+    M = T.track_model_create_seeded(other, 5, T.FP32)
+    assert not T.track_models_compatible(P.L, M)
+    with pytest.raises(T.TrackError):
+        T.track_sample(P.L, M, np.zeros(2, np.uint8), track.schedule(2, 5.0), dev(x[:1]),
+                       dev(c[:1]), dev(u[:1]), WL.cfg)
+
+
+# ---------------------------------------------------------------- full-size mid workload
+@pytest.mark.slow
+@pytest.mark.parametrize("which", ["large", "small"])
+def test_mid_workload_full_size_per_step(T, which):
+    """The benchmark workload at full size (3510 tokens, 30/12 layers, bf16, no CFG):
+    one denoiser evaluation of each model against the fp64 oracle, with weights
+    generated on the device exactly as the benchmark creates them."""
+    wl = synth.WORKLOADS["mid"]
+    arch = getattr(wl, which)
+    seed = synth.SEED_LARGE if which == "large" else synth.SEED_SMALL
+    m = T.track_model_create_seeded(arch, seed, T.BF16)
+    x, c, _ = synth.evaluation_inputs(arch, 0, 1, with_uncond=False)
+    sig = track.schedule(wl.steps, wl.shift)
+    t = float(track.model_timestep(sig[1]))
+    v = T.track_denoise(m, dev(x), t, dev(c), None, 1.0).cpu().numpy()
+    m.close()
+    ref = dit.DiT(arch, synth.make_weights(arch, seed), "bf16").forward(x[0], np.float32(t), c[0])
+    assert rel_l2(v[0], ref) < TOL["bf16"]
