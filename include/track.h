@@ -239,6 +239,32 @@ int track_linear(int dtype, const void* X, const void* W, const float* bias, int
 int track_attention(int dtype, const void* Q, const void* K, const void* V, int S, int H,
                     int Lq, int Lk, int hd, void* O, track_stream s);
 
+/* ---- allocation-free variant of track_disagreement -------------------------
+ * The paper has no counterpart to this entry point.  It is for callers that
+ * cannot allocate device memory while they run: a process whose device memory
+ * is reserved up front by its own pool allocator (a cudaMalloc in mid-run could
+ * fail), or a latency-critical loop that cannot take the device-wide
+ * synchronization that cudaMalloc/cudaFree imply.
+ *
+ * Computes what track_disagreement computes (Eq. 4 per sample, added to
+ * score_accum[b]), with the same arguments, but allocates nothing: its partial
+ * sums live in one fixed device array of TRACK_STATIC_MAX_SAMPLES x
+ * TRACK_STATIC_MAX_BLOCKS x 2 floats (256 KiB) compiled into the library, which
+ * every GPU that loads the library holds until the process exits.
+ *  - B above TRACK_STATIC_MAX_SAMPLES is rejected with TRACK_EINVAL.
+ *  - The first call on each device looks up the array's device address
+ *    (cudaGetSymbolAddress) with that device current; make that first call
+ *    before any stream capture.
+ *  - Every call shares the one array: calls whose kernels overlap on the GPU
+ *    (two streams with no ordering between them, two host threads) race and
+ *    produce wrong scores.  Calls ordered on one stream are safe; each call
+ *    writes every scratch slot it reads, so nothing is cleared in between.
+ */
+#define TRACK_STATIC_MAX_SAMPLES 64
+#define TRACK_STATIC_MAX_BLOCKS 512
+int track_disagreement_static(const float* v_L, const float* v_S, int B, int64_t n_per_sample,
+                              float eps, float* score_accum, track_stream s);
+
 #ifdef __cplusplus
 }
 #endif

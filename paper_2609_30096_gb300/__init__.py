@@ -71,6 +71,7 @@ def lib():
         "track_step": (_I, [_P, _P, _L, _F, _F, _P]),
         "track_cfg_step": (_I, [_P, _P, _P, _L, _F, _F, _F, _P]),
         "track_disagreement": (_I, [_P, _P, _I, _L, _F, _P, _P]),
+        "track_disagreement_static": (_I, [_P, _P, _I, _L, _F, _P, _P]),
         "track_mean_score": (_I, [_P, _I, _I, _P]),
         "track_policy_topk": (_I, [_P, _I, _I, _P]),
         "track_calibrate": (_I, [_P, _P, _P, _I, _P, _P, _F, _P, _I, _F, _P, _P]),
@@ -276,6 +277,15 @@ def track_disagreement(v_L, v_S, score_accum, eps=1e-8, stream=None):
     B = v_L.shape[0]
     _check(lib().track_disagreement(_ptr(v_L), _ptr(v_S), B, v_L.numel() // B, eps,
                                     _ptr(score_accum), _stream(stream)))
+    return score_accum
+
+
+def track_disagreement_static(v_L, v_S, score_accum, eps=1e-8, stream=None):
+    """track_disagreement with library-held scratch: allocates no device memory
+    (at most 64 samples per call; calls that overlap on the GPU race)."""
+    B = v_L.shape[0]
+    _check(lib().track_disagreement_static(_ptr(v_L), _ptr(v_S), B, v_L.numel() // B, eps,
+                                           _ptr(score_accum), _stream(stream)))
     return score_accum
 
 

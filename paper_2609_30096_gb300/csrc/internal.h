@@ -17,6 +17,9 @@ int* device_error_word();
 // Counts every kernel launch made by the library.
 void count_launch(int n = 1);
 
+// Records msg as this thread's last error (returned by track_last_error); returns code.
+int report_error(int code, const char* msg);
+
 // ---------------------------------------------------------------- GEMM
 struct GemmArgs {
   int M, N, K;

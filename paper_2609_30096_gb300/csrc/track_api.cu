@@ -28,6 +28,8 @@ static int fail(int code, const std::string& msg) {
   return code;
 }
 
+int report_error(int code, const char* msg) { return fail(code, msg); }
+
 #define TRACK_CUDA(expr)                                                              \
   do {                                                                                \
     cudaError_t e_ = (expr);                                                          \
