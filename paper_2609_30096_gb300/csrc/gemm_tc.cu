@@ -156,63 +156,44 @@ __device__ __forceinline__ float gelu_tanh(float u) {
   return 0.5f * u * (1.f + tanhf(0.7978845608028654f * fmaf(0.044715f * u, u * u, u)));
 }
 
-__device__ __forceinline__ void epilogue32(const GemmArgs& g, int row, int col0,
-                                           const uint32_t (&r)[32]) {
-  float v[32];
+// TMA bulk tensor store / reduce-add of a 32-row box staged in shared memory
+// (128-byte rows, 128-byte swizzle), tracked by the issuing thread's bulk group.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* tm, int x, int y, uint32_t src) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];"
+               ::"l"((uint64_t)tm), "r"(x), "r"(y), "r"(src) : "memory");
+}
+__device__ __forceinline__ void tma_reduce_add_2d(const CUtensorMap* tm, int x, int y,
+                                                  uint32_t src) {
+  asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.bulk_group"
+               " [%0, {%1, %2}], [%3];" ::"l"((uint64_t)tm), "r"(x), "r"(y), "r"(src)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// At most one older bulk group of this thread may still be reading shared memory.
+__device__ __forceinline__ void bulk_wait_read_1() {
+  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() {
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+__device__ __forceinline__ void fence_async_shared() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Writes this thread's 128-byte row `row` (8 chunks of 16 bytes) into a staging
+// box in the 128-byte-swizzled layout TMA expects: chunk j at j ^ (row % 8).
+__device__ __forceinline__ void stage_row(uint8_t* box, int row, const uint4 (&chunk)[8]) {
+  uint8_t* base = box + row * 128;
 #pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-  if (g.bias != nullptr) {
-    const float4* b4 = reinterpret_cast<const float4*>(g.bias + col0);
-#pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      const float4 b = b4[q];
-      v[4 * q] += b.x;
-      v[4 * q + 1] += b.y;
-      v[4 * q + 2] += b.z;
-      v[4 * q + 3] += b.w;
-    }
-  }
-  if (g.epi == EPI_STORE || g.epi == EPI_GELU) {
-    if (g.epi == EPI_GELU) {
-#pragma unroll
-      for (int i = 0; i < 32; ++i) v[i] = gelu_tanh(v[i]);
-    }
-    uint4* o = reinterpret_cast<uint4*>((bf16*)g.out + (int64_t)row * g.ldo + col0);
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      uint4 pk;
-      __nv_bfloat162 t;
-      t = __floats2bfloat162_rn(v[8 * q + 0], v[8 * q + 1]);
-      pk.x = *reinterpret_cast<uint32_t*>(&t);
-      t = __floats2bfloat162_rn(v[8 * q + 2], v[8 * q + 3]);
-      pk.y = *reinterpret_cast<uint32_t*>(&t);
-      t = __floats2bfloat162_rn(v[8 * q + 4], v[8 * q + 5]);
-      pk.z = *reinterpret_cast<uint32_t*>(&t);
-      t = __floats2bfloat162_rn(v[8 * q + 6], v[8 * q + 7]);
-      pk.w = *reinterpret_cast<uint32_t*>(&t);
-      o[q] = pk;
-    }
-  } else {
-    float4* o = reinterpret_cast<float4*>((float*)g.out + (int64_t)row * g.ldo + col0);
-    const float4* g4 = reinterpret_cast<const float4*>(g.gate + col0);
-#pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      float4 x = o[q];
-      if (g.epi == EPI_RESID_GATE) {
-        const float4 gg = g4[q];
-        x.x = fmaf(gg.x, v[4 * q], x.x);
-        x.y = fmaf(gg.y, v[4 * q + 1], x.y);
-        x.z = fmaf(gg.z, v[4 * q + 2], x.z);
-        x.w = fmaf(gg.w, v[4 * q + 3], x.w);
-      } else {
-        x.x += v[4 * q];
-        x.y += v[4 * q + 1];
-        x.z += v[4 * q + 2];
-        x.w += v[4 * q + 3];
-      }
-      o[q] = x;
-    }
-  }
+  for (int j = 0; j < 8; ++j)
+    *reinterpret_cast<uint4*>(base + ((j ^ (row & 7)) << 4)) = chunk[j];
+}
+
+__device__ __forceinline__ uint32_t pack2(float a, float b) {
+  __nv_bfloat162 t = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&t);
 }
 
 template <int BN, int STAGES>
@@ -220,19 +201,21 @@ struct TcShape {
   static constexpr uint32_t A_BYTES = BM * BK * 2;
   static constexpr uint32_t B_BYTES = BN * BK * 2;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
-  static constexpr size_t SMEM = 1024 + (size_t)STAGES * (A_BYTES + B_BYTES) + 256;
+  static constexpr uint32_t STG_BYTES = 4 * 2 * 4096;  // two 32x128-byte boxes per epilogue warp
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * (A_BYTES + B_BYTES) + STG_BYTES + 256;
 };
 
 template <int BN, int STAGES>
 __global__ void __launch_bounds__(192, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-              const GemmArgs g) {
+              const __grid_constant__ CUtensorMap tmC, const GemmArgs g) {
   using S = TcShape<BN, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* sA = smem;
   uint8_t* sB = smem + STAGES * S::A_BYTES;
-  uint64_t* bars = (uint64_t*)(sB + STAGES * S::B_BYTES);
+  uint8_t* stg_all = sB + STAGES * S::B_BYTES;  // 1024-byte aligned
+  uint64_t* bars = (uint64_t*)(stg_all + S::STG_BYTES);
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
   uint64_t* accf = bars + 2 * STAGES;
@@ -340,7 +323,10 @@ __global__ void __launch_bounds__(192, 1)
     }
   } else {
     const int quarter = warp & 3;  // TMEM lanes 32*quarter .. 32*quarter+31
-    int acc = 0;
+    uint8_t* stg = stg_all + (warp - 2) * 2 * 4096;
+    const bool bf16_out = g.epi == EPI_STORE || g.epi == EPI_GELU;
+    const int cw = bf16_out ? 64 : 32;  // columns per staged box (128-byte rows)
+    int sb = 0, acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
       const int mt = tile % m_tiles, nt = tile / m_tiles;
@@ -349,14 +335,74 @@ __global__ void __launch_bounds__(192, 1)
       ok = __shfl_sync(0xffffffffu, ok, 0);  // the whole warp takes the same branch
       if (!ok) break;
       tc_fence_after();
-      const int row = mt * BM + quarter * 32 + lane;
+      const int row_base = mt * BM + quarter * 32;
       const uint32_t tbase = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * BN);
 #pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
-        uint32_t r[32];
-        tmem_ld32(tbase + (uint32_t)(c * 32), r);
-        const int col0 = nt * BN + c * 32;
-        if (row < g.M && col0 < g.N) epilogue32(g, row, col0, r);
+      for (int c = 0; c < BN; c += cw) {
+        const int col0 = nt * BN + c;
+        if (row_base >= g.M || col0 >= g.N) continue;  // uniform across the warp
+        uint4 chunk[8];
+        if (bf16_out) {
+          uint32_t r0[32], r1[32];
+          tmem_ld32(tbase + (uint32_t)c, r0);
+          tmem_ld32(tbase + (uint32_t)(c + 32), r1);
+          const float4* b4 = reinterpret_cast<const float4*>(g.bias + col0);
+          const bool gelu = g.epi == EPI_GELU;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            float v[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const int i = 8 * j + e;
+              v[e] = __uint_as_float(i < 32 ? r0[i] : r1[i - 32]);
+            }
+            if (g.bias != nullptr && (j < 4 || col0 + 64 <= g.N)) {  // columns >= N are clipped
+              const float4 ba = b4[2 * j], bb = b4[2 * j + 1];
+              v[0] += ba.x; v[1] += ba.y; v[2] += ba.z; v[3] += ba.w;
+              v[4] += bb.x; v[5] += bb.y; v[6] += bb.z; v[7] += bb.w;
+            }
+            if (gelu) {
+#pragma unroll
+              for (int e = 0; e < 8; ++e) v[e] = gelu_tanh(v[e]);
+            }
+            chunk[j] = make_uint4(pack2(v[0], v[1]), pack2(v[2], v[3]), pack2(v[4], v[5]),
+                                  pack2(v[6], v[7]));
+          }
+        } else {
+          uint32_t r0[32];
+          tmem_ld32(tbase + (uint32_t)c, r0);
+          const float4* b4 = reinterpret_cast<const float4*>(g.bias + col0);
+          const float4* g4 = reinterpret_cast<const float4*>(g.gate + col0);
+          const bool gated = g.epi == EPI_RESID_GATE;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            float4 v = make_float4(__uint_as_float(r0[4 * j]), __uint_as_float(r0[4 * j + 1]),
+                                   __uint_as_float(r0[4 * j + 2]), __uint_as_float(r0[4 * j + 3]));
+            if (g.bias != nullptr) {
+              const float4 b = b4[j];
+              v.x += b.x; v.y += b.y; v.z += b.z; v.w += b.w;
+            }
+            if (gated) {
+              const float4 gg = g4[j];
+              v.x *= gg.x; v.y *= gg.y; v.z *= gg.z; v.w *= gg.w;
+            }
+            chunk[j] = make_uint4(__float_as_uint(v.x), __float_as_uint(v.y),
+                                  __float_as_uint(v.z), __float_as_uint(v.w));
+          }
+        }
+        // The box written two stores ago must have been read out by its TMA.
+        if (lane == 0) bulk_wait_read_1();
+        __syncwarp();
+        uint8_t* box = stg + sb * 4096;
+        stage_row(box, lane, chunk);
+        fence_async_shared();
+        __syncwarp();
+        if (lane == 0) {
+          if (bf16_out) tma_store_2d(&tmC, col0, row_base, su32(box));
+          else tma_reduce_add_2d(&tmC, col0, row_base, su32(box));
+          bulk_commit();
+        }
+        sb ^= 1;
       }
       tc_fence_before();
       __syncwarp();
@@ -366,6 +412,8 @@ __global__ void __launch_bounds__(192, 1)
         acc_phase ^= 1;
       }
     }
+    if (lane == 0) bulk_wait_all();  // this warp's stores have completed
+    __syncwarp();
   }
 
   tc_fence_before();
@@ -395,16 +443,18 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 2-D bf16 tensor map of a row-major [rows, cols] matrix, box [box_rows, 64].
-bool make_tmap(CUtensorMap* tm, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+// 2-D tensor map of a row-major [rows, cols] matrix with leading dimension ld
+// (elements), box [box_rows, box_cols], 128-byte swizzle, zero fill out of bounds.
+bool make_tmap(CUtensorMap* tm, CUtensorMapDataType dt, size_t esize, const void* ptr,
+               uint64_t rows, uint64_t cols, uint64_t ld, uint32_t box_rows, uint32_t box_cols) {
   EncodeTiledFn enc = encode_fn();
   if (enc == nullptr) return false;
   cuuint64_t dims[2] = {cols, rows};
-  cuuint64_t strides[1] = {cols * 2};
-  cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+  cuuint64_t strides[1] = {ld * esize};
+  cuuint32_t box[2] = {box_cols, box_rows};
   cuuint32_t estr[2] = {1, 1};
-  return enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box,
-             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+  return enc(tm, dt, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -412,15 +462,23 @@ template <int BN, int STAGES>
 cudaError_t launch_tc(const void* A, const void* W, const GemmArgs& g, cudaStream_t s) {
   using S = TcShape<BN, STAGES>;
   static_assert(S::SMEM <= 232448, "shared memory budget");
-  CUtensorMap ta, tb;
-  if (!make_tmap(&ta, A, (uint64_t)g.M, (uint64_t)g.K, BM)) return cudaErrorInvalidValue;
-  if (!make_tmap(&tb, W, (uint64_t)g.N, (uint64_t)g.K, BN)) return cudaErrorInvalidValue;
+  CUtensorMap ta, tb, tc;
+  const CUtensorMapDataType BF = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  if (!make_tmap(&ta, BF, 2, A, (uint64_t)g.M, (uint64_t)g.K, (uint64_t)g.K, BM, BK))
+    return cudaErrorInvalidValue;
+  if (!make_tmap(&tb, BF, 2, W, (uint64_t)g.N, (uint64_t)g.K, (uint64_t)g.K, BN, BK))
+    return cudaErrorInvalidValue;
+  const bool bf16_out = g.epi == EPI_STORE || g.epi == EPI_GELU;
+  if (bf16_out ? !make_tmap(&tc, BF, 2, g.out, (uint64_t)g.M, (uint64_t)g.N, (uint64_t)g.ldo, 32, 64)
+               : !make_tmap(&tc, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, g.out, (uint64_t)g.M,
+                            (uint64_t)g.N, (uint64_t)g.ldo, 32, 32))
+    return cudaErrorInvalidValue;
   cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN, STAGES>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)S::SMEM);
   if (e != cudaSuccess) return e;
   const int tiles = ((g.M + BM - 1) / BM) * ((g.N + BN - 1) / BN);
   const int grid = tiles < num_sms() ? tiles : num_sms();
-  k_gemm_tc<BN, STAGES><<<grid, 192, S::SMEM, s>>>(ta, tb, g);
+  k_gemm_tc<BN, STAGES><<<grid, 192, S::SMEM, s>>>(ta, tb, tc, g);
   count_launch();
   return cudaGetLastError();
 }
