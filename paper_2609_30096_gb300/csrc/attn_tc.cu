@@ -1,0 +1,335 @@
+// Flash attention on the sm_103a tensor cores (bf16 in, fp32 accumulate):
+// O = softmax(Q K^T / sqrt(hd)) V per (sequence, head), no mask.
+//
+// One CTA per 128-query tile of one (sequence, head), 192 threads:
+//   warp 0      TMA: the Q tile once, then K and V tiles of 128 keys into a
+//               two-stage ring (3-D tensor maps [S*H, L, hd], 128-byte swizzle,
+//               zero fill past L).
+//   warp 1      allocates TMEM (O: hd columns; S: two 128-column buffers) and
+//               issues, from one thread, S(j+1) = Q K(j+1)^T while the softmax
+//               warps work on S(j), then O += P(j) V(j) once P(j) is ready.
+//               V is the MN-major B operand, so no transposed copy is needed.
+//   warps 2-5   one thread per query row (its TMEM lane): row maximum of S(j)
+//               over the valid keys, lazy rescaling of O (only when the running
+//               maximum grows by more than 2^8, the rescale reading and writing
+//               the row in TMEM), P = exp2(S * log2(e)/sqrt(hd) - m) rounded to
+//               bf16 into 128-byte-swizzled shared memory, and at the end O / l
+//               stored to the token-major output.
+// Every mbarrier wait is bounded (see tc_common.cuh).
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <math.h>
+
+#include "internal.h"
+#include "tc_common.cuh"
+
+namespace track {
+
+namespace {
+
+using namespace tc;
+typedef __nv_bfloat16 bf16;
+
+constexpr int AT_BM = 128;       // query rows per CTA (MMA M)
+constexpr int AT_BN = 128;       // keys per tile
+constexpr int AT_THREADS = 192;  // warp 0 TMA, warp 1 MMA, warps 2-5 softmax
+constexpr uint32_t TM_S0 = 128;  // TMEM column of S buffer 0 (buffer 1 at 256)
+
+template <int HD>
+struct AtShape {
+  static constexpr uint32_t Q_BYTES = AT_BM * HD * 2;   // HD/64 boxes of [128 rows][128 B]
+  static constexpr uint32_t KV_BYTES = AT_BN * HD * 2;  // one K or V tile
+  static constexpr uint32_t P_BYTES = AT_BM * AT_BN * 2;
+  static constexpr int STAGES = 2;
+  static constexpr size_t SMEM = 1024 + Q_BYTES + 2 * STAGES * KV_BYTES + P_BYTES + 256;
+  static constexpr uint32_t TMEM_COLS = 512;
+};
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 t = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&t);
+}
+
+// Lane 0 waits, the whole warp learns the outcome.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          int* err, int code) {
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort_flag, err, code) ? 1 : 0;
+  return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+
+template <int HD>
+__global__ void __launch_bounds__(AT_THREADS, 1)
+    k_attn_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+              const __grid_constant__ CUtensorMap tmV, bf16* __restrict__ O, int H, int Lq, int Lk,
+              float scale_log2, int* err) {
+  using S = AtShape<HD>;
+  constexpr int NB = HD / 64;  // 64-column boxes per row of Q/K/V
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* sQ = smem;
+  uint8_t* sK = sQ + S::Q_BYTES;
+  uint8_t* sV = sK + S::STAGES * S::KV_BYTES;
+  uint8_t* sP = sV + S::STAGES * S::KV_BYTES;
+  uint64_t* bars = (uint64_t*)(sP + S::P_BYTES);
+  uint64_t* q_full = bars;
+  uint64_t* kv_full = bars + 1;   // [2]
+  uint64_t* kv_empty = bars + 3;  // [2]
+  uint64_t* s_full = bars + 5;    // [2]
+  uint64_t* p_full = bars + 7;
+  uint64_t* o_done = bars + 8;
+  uint64_t* done = bars + 9;
+  uint32_t* tmem_slot = (uint32_t*)(bars + 10);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int bh = blockIdx.y, q0 = blockIdx.x * AT_BM;
+  const int nkt = (Lk + AT_BN - 1) / AT_BN;
+
+  if (threadIdx.x == 0) {
+    mbar_init(su32(q_full), 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(su32(&kv_full[i]), 1);
+      mbar_init(su32(&kv_empty[i]), 1);
+      mbar_init(su32(&s_full[i]), 1);
+    }
+    mbar_init(su32(p_full), 4);
+    mbar_init(su32(o_done), 1);
+    mbar_init(su32(done), 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(su32(tmem_slot), S::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmQ) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmK) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmV) : "memory");
+      mbar_expect_tx(su32(q_full), S::Q_BYTES);
+      for (int b = 0; b < NB; ++b)
+        tma_load_3d(su32(sQ + b * AT_BM * 128), &tmQ, b * 64, q0, bh, su32(q_full));
+      uint32_t armed[2] = {0, 0};
+      for (int kt = 0; kt < nkt; ++kt) {
+        const int st = kt & 1;
+        if (!mbar_wait(su32(&kv_empty[st]), ((kt >> 1) & 1) ^ 1, abort_flag, err, 11)) break;
+        mbar_expect_tx(su32(&kv_full[st]), 2 * S::KV_BYTES);
+        for (int b = 0; b < NB; ++b) {
+          tma_load_3d(su32(sK + st * S::KV_BYTES + b * AT_BN * 128), &tmK, b * 64, kt * AT_BN, bh,
+                      su32(&kv_full[st]));
+          tma_load_3d(su32(sV + st * S::KV_BYTES + b * AT_BN * 128), &tmV, b * 64, kt * AT_BN, bh,
+                      su32(&kv_full[st]));
+        }
+        ++armed[st];
+      }
+      // Every copy this thread issued has landed before the CTA may exit.
+      mbar_drain(su32(q_full), 0, err, 15);
+      for (int i = 0; i < 2; ++i)
+        if (armed[i] != 0) mbar_drain(su32(&kv_full[i]), (armed[i] - 1) & 1, err, 15);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idS = idesc_bf16(AT_BM, AT_BN);
+      constexpr uint32_t idO = idesc_bf16_bmn(AT_BM, HD);
+      const uint32_t qa = su32(sQ), pa = su32(sP);
+      auto issue_s = [&](int kt) -> bool {
+        const int st = kt & 1;
+        if (!mbar_wait(su32(&kv_full[st]), (kt >> 1) & 1, abort_flag, err, 12)) return false;
+        tc_fence_after();
+        const uint32_t ka = su32(sK + st * S::KV_BYTES);
+        const uint32_t d = tmem_base + TM_S0 + (uint32_t)(st * AT_BN);
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk)
+          mma_bf16(d, sdesc_sw128(qa + (kk >> 2) * (AT_BM * 128) + (kk & 3) * 32),
+                   sdesc_sw128(ka + (kk >> 2) * (AT_BN * 128) + (kk & 3) * 32), idS,
+                   kk > 0 ? 1u : 0u);
+        mma_commit(su32(&s_full[st]));
+        return true;
+      };
+      bool ok = mbar_wait(su32(q_full), 0, abort_flag, err, 13);
+      if (ok) {
+        tc_fence_after();
+        ok = issue_s(0);
+      }
+      for (int kt = 0; ok && kt < nkt; ++kt) {
+        if (kt + 1 < nkt && !issue_s(kt + 1)) break;
+        if (!mbar_wait(su32(p_full), kt & 1, abort_flag, err, 14)) break;
+        tc_fence_after();
+        const int st = kt & 1;
+        const uint32_t va = su32(sV + st * S::KV_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < AT_BN / 16; ++kk)
+          mma_bf16(tmem_base, sdesc_sw128(pa + (kk >> 2) * (AT_BM * 128) + (kk & 3) * 32),
+                   sdesc_sw128_mn(va + kk * 16 * 128, AT_BN * 128), idO,
+                   (kt > 0 || kk > 0) ? 1u : 0u);
+        mma_commit(su32(&kv_empty[st]));
+        mma_commit(su32(o_done));
+      }
+      // Every MMA this thread issued has completed before TMEM is freed.
+      mma_commit(su32(done));
+      mbar_drain(su32(done), 0, err, 16);
+    }
+  } else {
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;
+    const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
+    const uint32_t tO = tmem_base + lane_off;
+    float m = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int kt = 0; kt < nkt; ++kt) {
+      if (!warp_wait(su32(&s_full[kt & 1]), (kt >> 1) & 1, abort_flag, err, 17)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t tS = tmem_base + lane_off + TM_S0 + (uint32_t)((kt & 1) * AT_BN);
+      const int kbase = kt * AT_BN;
+      uint32_t r[32];
+      float mx = -INFINITY;
+#pragma unroll 1
+      for (int c = 0; c < AT_BN / 32; ++c) {
+        tmem_ld32(tS + c * 32, r);
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (kbase + c * 32 + i < Lk) mx = fmaxf(mx, __uint_as_float(r[i]));
+      }
+      const float mt = mx * scale_log2;
+      if (kt > 0) {
+        // P(kt-1) V(kt-1) must be complete before P is overwritten or O rescaled.
+        if (!warp_wait(su32(o_done), (kt - 1) & 1, abort_flag, err, 18)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const bool need = mt > m + 8.f;
+        if (__any_sync(0xffffffffu, need)) {
+          const float alpha = need ? exp2_approx(m - mt) : 1.f;
+          if (need) {
+            m = mt;
+            l *= alpha;
+          }
+#pragma unroll 1
+          for (int c = 0; c < HD / 32; ++c) {
+            tmem_ld32(tO + c * 32, r);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+            tmem_st32(tO + c * 32, r);
+          }
+          tmem_st_wait();
+        }
+      } else {
+        m = mt;
+      }
+      float rs = 0.f;
+#pragma unroll 1
+      for (int c = 0; c < AT_BN / 32; ++c) {
+        tmem_ld32(tS + c * 32, r);
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int k0 = kbase + c * 32 + 2 * i;
+          const float p0 = k0 < Lk ? exp2_approx(fmaf(__uint_as_float(r[2 * i]), scale_log2, -m)) : 0.f;
+          const float p1 =
+              k0 + 1 < Lk ? exp2_approx(fmaf(__uint_as_float(r[2 * i + 1]), scale_log2, -m)) : 0.f;
+          rs += p0 + p1;
+          pk[i] = pack_bf16x2(p0, p1);
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int cidx = c * 4 + j;  // 16-byte chunk of the row (8 keys)
+          uint8_t* dst = sP + (cidx >> 3) * (AT_BM * 128) + row * 128 + (((cidx & 7) ^ (row & 7)) << 4);
+          *reinterpret_cast<uint4*>(dst) = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
+        }
+      }
+      l += rs;
+      fence_async_shared();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(su32(p_full));
+    }
+    if (ok && warp_wait(su32(o_done), (nkt - 1) & 1, abort_flag, err, 19)) {
+      tc_fence_after();
+      const float inv = 1.f / l;
+      const int qrow = q0 + row;
+      const int s_ = bh / H, h = bh % H;
+      bf16* orow = O + (((int64_t)s_ * Lq + qrow) * H + h) * HD;
+      uint32_t r2[32];
+#pragma unroll 1
+      for (int c = 0; c < HD / 32; ++c) {
+        tmem_ld32(tO + c * 32, r2);
+        if (qrow < Lq) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            uint4 v;
+            v.x = pack_bf16x2(__uint_as_float(r2[8 * j]) * inv, __uint_as_float(r2[8 * j + 1]) * inv);
+            v.y = pack_bf16x2(__uint_as_float(r2[8 * j + 2]) * inv, __uint_as_float(r2[8 * j + 3]) * inv);
+            v.z = pack_bf16x2(__uint_as_float(r2[8 * j + 4]) * inv, __uint_as_float(r2[8 * j + 5]) * inv);
+            v.w = pack_bf16x2(__uint_as_float(r2[8 * j + 6]) * inv, __uint_as_float(r2[8 * j + 7]) * inv);
+            *reinterpret_cast<uint4*>(orow + c * 32 + 8 * j) = v;
+          }
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem_base, S::TMEM_COLS);
+  }
+}
+
+// 3-D tensor map of head-major [SH, L, hd] bf16, box [1, rows, 64].
+bool make_tmap_3d(CUtensorMap* tm, const void* ptr, int hd, int L, int SH, uint32_t rows) {
+  EncodeTiledFn enc = encode_tiled_fn();
+  if (enc == nullptr) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)hd, (cuuint64_t)L, (cuuint64_t)SH};
+  cuuint64_t strides[2] = {(cuuint64_t)hd * 2, (cuuint64_t)L * hd * 2};
+  cuuint32_t box[3] = {64, rows, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int HD>
+cudaError_t launch_attn_tc(const void* Q, const void* K, const void* V, void* O, int S_, int H,
+                           int Lq, int Lk, cudaStream_t s) {
+  using S = AtShape<HD>;
+  static_assert(S::SMEM <= 232448, "shared memory budget");
+  CUtensorMap tq, tk, tv;
+  if (!make_tmap_3d(&tq, Q, HD, Lq, S_ * H, AT_BM) || !make_tmap_3d(&tk, K, HD, Lk, S_ * H, AT_BN) ||
+      !make_tmap_3d(&tv, V, HD, Lk, S_ * H, AT_BN))
+    return cudaErrorInvalidValue;
+  int* err = device_error_word();
+  if (err == nullptr) return cudaErrorMemoryAllocation;
+  cudaError_t e = cudaFuncSetAttribute(k_attn_tc<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)S::SMEM);
+  if (e != cudaSuccess) return e;
+  dim3 grid((Lq + AT_BM - 1) / AT_BM, S_ * H);
+  const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)HD));
+  k_attn_tc<HD><<<grid, AT_THREADS, S::SMEM, s>>>(tq, tk, tv, (bf16*)O, H, Lq, Lk, scale_log2, err);
+  count_launch();
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t attention_bf16_tc(const void* Q, const void* K, const void* V, void* O, int S, int H,
+                              int Lq, int Lk, int hd, cudaStream_t s) {
+  if (S <= 0 || Lq <= 0) return cudaSuccess;
+  if (Lk <= 0 || S * H > 65535) return cudaErrorInvalidValue;
+  if ((((uintptr_t)Q) | ((uintptr_t)K) | ((uintptr_t)V) | ((uintptr_t)O)) & 15)
+    return cudaErrorMisalignedAddress;
+  if (hd == 128) return launch_attn_tc<128>(Q, K, V, O, S, H, Lq, Lk, s);
+  if (hd == 64) return launch_attn_tc<64>(Q, K, V, O, S, H, Lq, Lk, s);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace track

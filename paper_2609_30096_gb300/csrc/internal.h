@@ -44,6 +44,9 @@ cudaError_t attention_f32(const float* Q, const float* K, const float* V, float*
                           int Lq, int Lk, int hd, cudaStream_t s);
 cudaError_t attention_bf16(const void* Q, const void* K, const void* V, void* O, int S, int H,
                            int Lq, int Lk, int hd, cudaStream_t s);
+// tcgen05 / TMEM flash attention (attn_tc.cu); same layouts.
+cudaError_t attention_bf16_tc(const void* Q, const void* K, const void* V, void* O, int S, int H,
+                              int Lq, int Lk, int hd, cudaStream_t s);
 
 // ---------------------------------------------------------------- elementwise
 cudaError_t convert_f32(const float* src, void* dst, int dtype, int64_t n, cudaStream_t s);
