@@ -50,6 +50,25 @@ def load_peaks():
         return FALLBACK_PEAKS, "fallback"
 
 
+def measured_traffic(kernel, flops_per_launch):
+    """DRAM bytes per launch from the committed ncu capture of `kernel`, scaled to a launch
+    of `flops_per_launch` by its FLOPs; None if the kernel's source changed since."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "ncu_traffic.json")) as f:
+            rec = json.load(f)[kernel]
+        m = hashlib.sha1()
+        for src in rec["sources"]:
+            with open(os.path.join(ROOT, "paper_2609_30096_gb300", "csrc", src), "rb") as f:
+                m.update(f.read())
+        if m.hexdigest() != rec["source_sha1"]:
+            return None, "kernel changed since the ncu capture"
+        per_flop = (rec["dram_read_bytes"] + rec["dram_write_bytes"]) / rec["flops"]
+        return per_flop * flops_per_launch, "scaled by FLOPs from " + rec["launch"]
+    except Exception as e:  # noqa: BLE001
+        return None, f"no capture ({type(e).__name__})"
+
+
 def forward_flops(arch, batch):
     """Algorithmic FLOPs of one denoiser evaluation of `batch` sequences (text work excluded)."""
     L, d, F, Lt, l = arch.tokens, arch.dim, arch.ffn, arch.text_len, arch.layers
@@ -322,15 +341,18 @@ def run_ours(args):
     peaks, src = load_peaks()
     gm, gf, gn = prof["gemm"]
     am, af, an = prof["attention"]
+    nm, nb, nn = prof["norm"]
     dominant = "gemm" if gm >= am else "attention"
     dm, dflops, dn = prof[dominant]
     achieved = (dflops / dn) / (dm / dn / 1e3) / 1e12 if dn else None
     peak = peaks["bf16_tflops"]
-    traffic = None
+    traffic, traffic_src = measured_traffic("k_gemm_tc" if dominant == "gemm" else "k_attn_tc",
+                                            dflops / dn if dn else 0.0)
     roof = {"bound": "tensor", "kernel": "bf16 GEMM (tcgen05)" if dominant == "gemm"
             else "flash attention (bf16 mma.sync)",
             "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
             "frac": achieved / peak if achieved else None, "traffic": traffic,
+            "traffic_unit": "bytes per launch", "traffic_source": traffic_src,
             "peak_source": f"{src} bf16 burst (sustained {peaks.get('bf16_tflops_sustained')})",
             "launches": int(dn), "avg_launch_ms": dm / dn if dn else None,
             "share_of_step": dm / ms_prof if ms_prof else None,
@@ -339,7 +361,11 @@ def run_ours(args):
             "other": {("attention" if dominant == "gemm" else "gemm"):
                       {"ms": am if dominant == "gemm" else gm,
                        "tflops": ((af / (am / 1e3)) if dominant == "gemm" and am
-                                  else (gf / (gm / 1e3)) if gm else 0) / 1e12}}}
+                                  else (gf / (gm / 1e3)) if gm else 0) / 1e12},
+                      "norm_kernels": {"ms": nm, "launches": int(nn),
+                                       "gb_per_s": (nb / (nm / 1e3) / 1e9) if nm else None,
+                                       "frac_of_hbm": ((nb / (nm / 1e3) / 1e9) / peaks["hbm_gbs"])
+                                       if nm else None}}}
 
     cpu = None
     if rank == 0 and not args.skip_cpu:
@@ -410,7 +436,7 @@ def run_kernel(args):
             fn = (lambda X=X, W=W, b=b, epi=epi, out=out, gate=gate:
                   T.track_linear(T.BF16, X, W, b, epi, out, gate=gate if epi == 2 else None))
             cases.append((name, f"M={M} N={N} K={K}", 2.0 * M * N * K, fn))
-    else:
+    elif args.kernel == "attention":
         Q, Kt, V = (rnd(args.batch, H, a.tokens, hd) for _ in range(3))
         Kc, Vc = rnd(args.batch, H, a.text_len, hd), rnd(args.batch, H, a.text_len, hd)
         O = torch.empty(args.batch, a.tokens, H, hd, device="cuda", dtype=torch.bfloat16)
@@ -420,6 +446,22 @@ def run_kernel(args):
         cases.append(("cross_attention", f"S={args.batch} H={H} Lq={a.tokens} Lk={a.text_len}",
                       4.0 * args.batch * H * a.tokens * a.text_len * hd,
                       lambda: T.track_attention(T.BF16, Q, Kc, Vc, O)))
+    elif args.kernel == "hbm":
+        # HBM-bound kernels of the public C ABI, algorithmic bytes per call: fused
+        # guidance + Euler update 16 B/elem (read f_c, f_u, x; write x), Eq. 4
+        # reduction 8 B/elem (read p_L, p_S).  The normalization kernels inside the
+        # denoiser are measured in place by the full benchmark.
+        n480 = 16 * 21 * 60 * 104
+        for label, n in (("480p latent x2 (CFG batch)", 2 * n480), ("1 Gi elements", 1 << 30)):
+            fc, fu, xx = (torch.randn(n, device="cuda") for _ in range(3))
+            cases.append(("cfg_euler", f"{label}: n={n}", 16.0 * n,
+                          lambda fc=fc, fu=fu, xx=xx: T.track_cfg_step(xx, fc, fu, 5.0, 0.5, 0.45)))
+            B = 2 if n == 2 * n480 else 8
+            acc = torch.zeros(B, device="cuda")
+            cases.append(("disagreement", f"{label}: B={B} n={n // B}", 8.0 * n,
+                          lambda fc=fc, fu=fu, acc=acc, B=B: T.track_disagreement(
+                              fc.view(B, -1), fu.view(B, -1), acc)))
+            del xx
     peaks, src = load_peaks()
     out = []
     for name, shape, flops, fn in cases:
@@ -433,6 +475,11 @@ def run_kernel(args):
         e1.record()
         T.track_sync()
         ms = e0.elapsed_time(e1) / args.steps
+        if args.kernel == "hbm":
+            gbs = flops / (ms / 1e3) / 1e9
+            out.append({"kernel": name, "shape": shape, "ms": ms, "gb_per_s": gbs,
+                        "frac_of_hbm": gbs / peaks["hbm_gbs"], "peak_source": src})
+            continue
         tf = flops / (ms / 1e3) / 1e12
         out.append({"kernel": name, "shape": shape, "ms": ms, "tflops": tf,
                     "frac_of_bf16_peak": tf / peaks["bf16_tflops"], "peak_source": src})
@@ -448,7 +495,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--skip-cpu", action="store_true", help="omit the oracle CPU baseline")
-    ap.add_argument("--kernel", choices=["gemm", "attention"], default=None,
+    ap.add_argument("--kernel", choices=["gemm", "attention", "hbm"], default=None,
                     help="time one kernel class alone at the workload's shapes")
     ap.add_argument("--batch", type=int, default=1, help="sequences for --kernel")
     args = ap.parse_args()

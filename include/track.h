@@ -94,12 +94,14 @@ int track_sync(track_stream s);
 /* Number of kernels this library has launched since load (returns the count). */
 int64_t track_launch_count(void);
 
-/* Kernel timing: while enabled, GEMM and attention launches inside
- * track_denoise/track_denoise_step/track_calibrate/track_sample are bracketed
- * by CUDA events on their stream.  track_profile_read synchronizes those
- * events and returns, per class (0 = GEMM, 1 = attention), the summed event
- * time in ms, the summed algorithmic FLOPs and the number of launches, then
- * clears the records.  Arrays are host, length 2. */
+/* Kernel timing: while enabled, the GEMM, attention and normalization
+ * launches inside track_denoise/track_denoise_step/track_calibrate/track_sample
+ * are bracketed by CUDA events on their stream.  track_profile_read
+ * synchronizes those events and returns, per class (0 = GEMM, 1 = attention,
+ * 2 = LayerNorm-modulate and RMSNorm/RoPE/head split), the summed event time in
+ * ms, the summed algorithmic work (FLOPs for classes 0 and 1, bytes moved for
+ * class 2) and the number of launches, then clears the records.  Arrays are
+ * host, length 3. */
 int track_profile_enable(int enable);
 int track_profile_read(double* ms, double* flops, int64_t* launches);
 

@@ -141,12 +141,14 @@ def track_profile_enable(enable: bool):
 
 
 def track_profile_read():
-    """{'gemm': (ms, flops, launches), 'attention': (...)} since the last read."""
-    ms = (ctypes.c_double * 2)()
-    fl = (ctypes.c_double * 2)()
-    n = (ctypes.c_int64 * 2)()
+    """{'gemm': (ms, flops, launches), 'attention': (ms, flops, launches),
+    'norm': (ms, bytes, launches)} since the last read."""
+    ms = (ctypes.c_double * 3)()
+    fl = (ctypes.c_double * 3)()
+    n = (ctypes.c_int64 * 3)()
     _check(lib().track_profile_read(ms, fl, n))
-    return {"gemm": (ms[0], fl[0], n[0]), "attention": (ms[1], fl[1], n[1])}
+    return {"gemm": (ms[0], fl[0], n[0]), "attention": (ms[1], fl[1], n[1]),
+            "norm": (ms[2], fl[2], n[2])}
 
 
 # ---------------------------------------------------------------- models

@@ -209,121 +209,170 @@ cudaError_t patch_embed(const float* x, int B, int nseq, int C, int F, int H, in
 }
 
 // ---------------------------------------------------------------- LayerNorm + modulation
-constexpr int LN_MAXV = 24;  // d <= 24 * blockDim
+__device__ __forceinline__ float warp_sum(float v) {
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
 
+__device__ __forceinline__ void store4(float* p, float a, float b, float c, float d) {
+  *reinterpret_cast<float4*>(p) = make_float4(a, b, c, d);
+}
+__device__ __forceinline__ void store4(bf16* p, float a, float b, float c, float d) {
+  __nv_bfloat162 lo = __floats2bfloat162_rn(a, b), hi = __floats2bfloat162_rn(c, d);
+  *reinterpret_cast<uint2*>(p) =
+      make_uint2(*reinterpret_cast<uint32_t*>(&lo), *reinterpret_cast<uint32_t*>(&hi));
+}
+
+// One warp per row, 16-byte loads; mean and variance in two passes over the row
+// (the second and third reads hit L1).
 template <typename T>
-__global__ void __launch_bounds__(256) k_ln_mod(const float* __restrict__ x, int d,
+__global__ void __launch_bounds__(256) k_ln_mod(const float* __restrict__ x, int M, int d,
                                                 const float* __restrict__ a,
                                                 const float* __restrict__ b, int mode, float eps,
                                                 T* __restrict__ out) {
-  __shared__ float red[32];
-  const int64_t row = blockIdx.x;
-  const float* xr = x + row * d;
-  float v[LN_MAXV];
+  const int lane = threadIdx.x & 31;
+  const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (row >= M) return;
+  const float4* xr = reinterpret_cast<const float4*>(x + row * d);
+  const int n4 = d >> 2;
   float s = 0.f;
-#pragma unroll
-  for (int i = 0; i < LN_MAXV; ++i) {
-    const int j = threadIdx.x + i * blockDim.x;
-    v[i] = j < d ? xr[j] : 0.f;
-    s += v[i];
+  for (int i = lane; i < n4; i += 32) {
+    const float4 v = xr[i];
+    s += (v.x + v.y) + (v.z + v.w);
   }
-  const float mean = block_sum(s, red) / (float)d;
+  const float mean = warp_sum(s) / (float)d;
   float q = 0.f;
-#pragma unroll
-  for (int i = 0; i < LN_MAXV; ++i) {
-    const int j = threadIdx.x + i * blockDim.x;
-    const float c = j < d ? v[i] - mean : 0.f;
-    q = fmaf(c, c, q);
+  for (int i = lane; i < n4; i += 32) {
+    const float4 v = xr[i];
+    float t;
+    t = v.x - mean; q = fmaf(t, t, q);
+    t = v.y - mean; q = fmaf(t, t, q);
+    t = v.z - mean; q = fmaf(t, t, q);
+    t = v.w - mean; q = fmaf(t, t, q);
   }
-  const float var = block_sum(q, red) / (float)d;
-  const float rstd = 1.f / sqrtf(var + eps);
+  const float rstd = 1.f / sqrtf(warp_sum(q) / (float)d + eps);
+  const float4* a4 = reinterpret_cast<const float4*>(a);
+  const float4* b4 = reinterpret_cast<const float4*>(b);
   T* orow = out + row * d;
-#pragma unroll
-  for (int i = 0; i < LN_MAXV; ++i) {
-    const int j = threadIdx.x + i * blockDim.x;
-    if (j < d) {
-      const float m = mode == 0 ? 1.f + a[j] : a[j];
-      stv(orow, j, fmaf((v[i] - mean) * rstd, m, b[j]));
-    }
+  const float one = mode == 0 ? 1.f : 0.f;
+  for (int i = lane; i < n4; i += 32) {
+    const float4 v = xr[i], aa = a4[i], bb = b4[i];
+    store4(orow + 4 * i, fmaf((v.x - mean) * rstd, one + aa.x, bb.x),
+           fmaf((v.y - mean) * rstd, one + aa.y, bb.y), fmaf((v.z - mean) * rstd, one + aa.z, bb.z),
+           fmaf((v.w - mean) * rstd, one + aa.w, bb.w));
   }
 }
 
 cudaError_t ln_modulate(const float* x, int M, int d, const float* a, const float* b, int mode,
                         float eps, void* out, int dtype, cudaStream_t s) {
-  if (d > LN_MAXV * 256) return cudaErrorInvalidValue;
-  const int threads = d >= 2048 ? 256 : (d >= 512 ? 128 : 64);
-  if (d > LN_MAXV * threads) return cudaErrorInvalidValue;
-  if (dtype == BF16) k_ln_mod<bf16><<<M, threads, 0, s>>>(x, d, a, b, mode, eps, (bf16*)out);
-  else k_ln_mod<float><<<M, threads, 0, s>>>(x, d, a, b, mode, eps, (float*)out);
+  if (d % 4) return cudaErrorInvalidValue;
+  const int g = (M + 7) / 8;
+  if (dtype == BF16) k_ln_mod<bf16><<<g, 256, 0, s>>>(x, M, d, a, b, mode, eps, (bf16*)out);
+  else k_ln_mod<float><<<g, 256, 0, s>>>(x, M, d, a, b, mode, eps, (float*)out);
   count_launch();
   return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- RMSNorm + RoPE + head split
-// One block per row.  For each present section (q, k, v): load d values, optionally
-// RMSNorm over d with gain, optionally rotate (q, k) pairs, write head-major.
+// One warp per (row, present section).  The row section is read in 8-element
+// chunks (16 bytes for bf16): a first pass for the sum of squares when a gain is
+// given, a second pass that normalizes, rotates (q, k) pairs and writes each chunk
+// to its head-major place.
+__device__ __forceinline__ void load8(const bf16* p, float (&v)[8]) {
+  const uint4 u = *reinterpret_cast<const uint4*>(p);
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    __nv_bfloat162 t = *reinterpret_cast<const __nv_bfloat162*>(&w[i]);
+    v[2 * i] = __low2float(t);
+    v[2 * i + 1] = __high2float(t);
+  }
+}
+__device__ __forceinline__ void load8(const float* p, float (&v)[8]) {
+  const float4 a = reinterpret_cast<const float4*>(p)[0], b = reinterpret_cast<const float4*>(p)[1];
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+__device__ __forceinline__ void store8(bf16* p, const float (&v)[8]) {
+  uint32_t w[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    __nv_bfloat162 t = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+    w[i] = *reinterpret_cast<uint32_t*>(&t);
+  }
+  *reinterpret_cast<uint4*>(p) = make_uint4(w[0], w[1], w[2], w[3]);
+}
+__device__ __forceinline__ void store8(float* p, const float (&v)[8]) {
+  reinterpret_cast<float4*>(p)[0] = make_float4(v[0], v[1], v[2], v[3]);
+  reinterpret_cast<float4*>(p)[1] = make_float4(v[4], v[5], v[6], v[7]);
+}
+
 template <typename T>
-__global__ void __launch_bounds__(256) k_qkv_prep(PrepArgs a) {
-  extern __shared__ float buf[];  // d floats
-  __shared__ float red[32];
-  const int r = blockIdx.x;
-  const int seq = r / a.L, l = r % a.L;
-  const T* src = (const T*)a.src + (int64_t)r * a.ld;
-  const int half = a.hd / 2;
-  const int s6 = a.hd / 6;
-  const int nf = (a.hd - 4 * s6) / 2, nh = s6;  // pairs per axis: frame, height (width = nh)
-  const int pf = l / (a.Hp * a.Wp), ph = (l / a.Wp) % a.Hp, pw = l % a.Wp;
-  for (int sec = 0; sec < 3; ++sec) {
-    if (a.dst[sec] == nullptr) continue;  // uniform across the block
-    const T* sp = src + a.off[sec];
+__global__ void __launch_bounds__(256) k_qkv_prep(PrepArgs a, int nsec, int s0, int s1, int s2) {
+  const int lane = threadIdx.x & 31;
+  const int64_t gw = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int64_t r = gw / nsec;
+  if (r >= a.rows) return;
+  const int k = (int)(gw % nsec);
+  const int sec = k == 0 ? s0 : (k == 1 ? s1 : s2);
+  const int seq = (int)(r / a.L), l = (int)(r % a.L);
+  const T* src = (const T*)a.src + r * a.ld + a.off[sec];
+  const int nc = a.d >> 3;
+  const float* g = a.gain[sec];
+  float rstd = 1.f;
+  if (g != nullptr) {
     float ss = 0.f;
-    for (int j = threadIdx.x; j < a.d; j += blockDim.x) {
-      const float v = ldv(sp, j);
-      buf[j] = v;
-      ss = fmaf(v, v, ss);
+    for (int c = lane; c < nc; c += 32) {
+      float v[8];
+      load8(src + 8 * c, v);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ss = fmaf(v[i], v[i], ss);
     }
-    float rstd = 1.f;
-    if (a.gain[sec] != nullptr) {
-      const float tot = block_sum(ss, red);
-      rstd = 1.f / sqrtf(tot / (float)a.d + a.eps);
-    } else {
-      __syncthreads();
+    rstd = 1.f / sqrtf(warp_sum(ss) / (float)a.d + a.eps);
+  }
+  const bool rot = a.rope && sec < 2;
+  const int s6 = a.hd / 6;
+  const int nf = (a.hd - 4 * s6) / 2, nh = s6;  // rotated pairs per axis: frame, height (= width)
+  const int pf = l / (a.Hp * a.Wp), ph = (l / a.Wp) % a.Hp, pw = l % a.Wp;
+  T* dst = (T*)a.dst[sec];
+  for (int c = lane; c < nc; c += 32) {
+    float v[8];
+    load8(src + 8 * c, v);
+    const int e0 = 8 * c, h = e0 / a.hd, eh = e0 % a.hd;
+    if (g != nullptr) {
+      const float4 g0 = reinterpret_cast<const float4*>(g + e0)[0];
+      const float4 g1 = reinterpret_cast<const float4*>(g + e0)[1];
+      const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+#pragma unroll
+      for (int i = 0; i < 8; ++i) v[i] = v[i] * rstd * gg[i];
     }
-    const float* g = a.gain[sec];
-    T* dst = (T*)a.dst[sec];
-    const bool rot = a.rope && sec < 2;
-    for (int p = threadIdx.x; p < a.d / 2; p += blockDim.x) {
-      const int h = p / half, j = p % half;
-      const int e = 2 * j;
-      float x0 = buf[h * a.hd + e], x1 = buf[h * a.hd + e + 1];
-      if (g) {
-        x0 = x0 * rstd * g[h * a.hd + e];
-        x1 = x1 * rstd * g[h * a.hd + e + 1];
-      }
-      if (rot) {
+    if (rot) {
+#pragma unroll
+      for (int p = 0; p < 4; ++p) {
+        const int j = eh / 2 + p;
         int idx;
         if (j < nf) idx = pf * nf + j;
         else if (j < nf + nh) idx = a.Fp * nf + ph * nh + (j - nf);
         else idx = a.Fp * nf + a.Hp * nh + pw * nh + (j - nf - nh);
         const float2 cs = a.rope_tab[idx];
-        const float y0 = x0 * cs.x - x1 * cs.y;
-        const float y1 = x0 * cs.y + x1 * cs.x;
-        x0 = y0;
-        x1 = y1;
+        const float x0 = v[2 * p], x1 = v[2 * p + 1];
+        v[2 * p] = x0 * cs.x - x1 * cs.y;
+        v[2 * p + 1] = x0 * cs.y + x1 * cs.x;
       }
-      const int64_t o = (((int64_t)seq * a.H + h) * a.L + l) * a.hd + e;
-      stv(dst, o, x0);
-      stv(dst, o + 1, x1);
     }
-    __syncthreads();  // buf reused by the next section
+    store8(dst + (((int64_t)seq * a.H + h) * a.L + l) * a.hd + eh, v);
   }
 }
 
 cudaError_t qkv_prep(const PrepArgs& a, cudaStream_t s) {
-  const size_t sm = (size_t)a.d * sizeof(float);
-  if (sm > 48 * 1024) return cudaErrorInvalidValue;
-  if (a.dtype == BF16) k_qkv_prep<bf16><<<a.rows, 256, sm, s>>>(a);
-  else k_qkv_prep<float><<<a.rows, 256, sm, s>>>(a);
+  int secs[3] = {0, 0, 0}, nsec = 0;
+  for (int i = 0; i < 3; ++i)
+    if (a.dst[i] != nullptr) secs[nsec++] = i;
+  if (nsec == 0 || a.rows <= 0) return cudaSuccess;
+  if (a.d % 8 || a.hd % 8) return cudaErrorInvalidValue;
+  const int64_t warps = (int64_t)a.rows * nsec;
+  const int g = (int)((warps + 7) / 8);
+  if (a.dtype == BF16) k_qkv_prep<bf16><<<g, 256, 0, s>>>(a, nsec, secs[0], secs[1], secs[2]);
+  else k_qkv_prep<float><<<g, 256, 0, s>>>(a, nsec, secs[0], secs[1], secs[2]);
   count_launch();
   return cudaGetLastError();
 }

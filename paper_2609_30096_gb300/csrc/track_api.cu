@@ -484,6 +484,18 @@ static int run_attention(const track_model* m, const void* Q, const void* K, con
   return TRACK_OK;
 }
 
+// LayerNorm-modulate and RMSNorm/RoPE/head-split launches, timed as class 2 with
+// their algorithmic bytes (fp32 row in + activation row out; activation in + out).
+static cudaError_t run_ln(const track_model* m, const float* x, int M, int d, const float* a,
+                          const float* b, int mode, void* out, cudaStream_t s) {
+  ProfScope ps(2, (double)M * d * (4.0 + m->esz), s);
+  return ln_modulate(x, M, d, a, b, mode, m->a.eps, out, m->dtype, s);
+}
+static cudaError_t run_prep(const track_model* m, const PrepArgs& p, int sections, cudaStream_t s) {
+  ProfScope ps(2, (double)p.rows * p.d * sections * 2.0 * m->esz, s);
+  return qkv_prep(p, s);
+}
+
 #define LAUNCH(expr)                                                                  \
   do {                                                                                \
     cudaError_t e_ = (expr);                                                          \
@@ -564,30 +576,30 @@ static int forward(track_model* m, const float* x, int B, int nseq, float t, con
     const float *shift1 = mod, *scale1 = mod + d, *gate1 = mod + 2 * d;
     const float *shift2 = mod + 3 * d, *scale2 = mod + 4 * d, *gate2 = mod + 5 * d;
     // self-attention
-    LAUNCH(ln_modulate(w.xres, M, d, scale1, shift1, 0, a.eps, w.h, m->dtype, s));
+    LAUNCH(run_ln(m, w.xres, M, d, scale1, shift1, 0, w.h, s));
     TRACK_TRY(run_gemm(m, w.h, Ly.Wqkv, M, 3 * d, d, Ly.bqkv, EPI_STORE, nullptr, w.qkv, 3 * d, s));
     ps.src = w.qkv; ps.ld = 3 * d;
     ps.off[0] = 0; ps.off[1] = d; ps.off[2] = 2 * d;
     ps.gain[0] = Ly.qn_g; ps.gain[1] = Ly.kn_g; ps.gain[2] = nullptr;
     ps.dst[0] = w.Qh; ps.dst[1] = w.Kh; ps.dst[2] = w.Vh;
     ps.rope = 1;
-    LAUNCH(qkv_prep(ps, s));
+    LAUNCH(run_prep(m, ps, 3, s));
     TRACK_TRY(run_attention(m, w.Qh, w.Kh, w.Vh, w.attn, nseq, L, L, s));
     TRACK_TRY(run_gemm(m, w.attn, Ly.Wo, M, d, d, Ly.bo, EPI_RESID_GATE, gate1, w.xres, d, s));
     // cross-attention
-    LAUNCH(ln_modulate(w.xres, M, d, Ly.ln3_g, Ly.ln3_b, 1, a.eps, w.h, m->dtype, s));
+    LAUNCH(run_ln(m, w.xres, M, d, Ly.ln3_g, Ly.ln3_b, 1, w.h, s));
     TRACK_TRY(run_gemm(m, w.h, Ly.Wcq, M, d, d, Ly.bcq, EPI_STORE, nullptr, w.qkv, d, s));
     ps.src = w.qkv; ps.ld = d;
     ps.off[0] = 0; ps.off[1] = -1; ps.off[2] = -1;
     ps.gain[0] = Ly.cqn_g; ps.gain[1] = nullptr;
     ps.dst[0] = w.Qh; ps.dst[1] = nullptr; ps.dst[2] = nullptr;
     ps.rope = 0;
-    LAUNCH(qkv_prep(ps, s));
+    LAUNCH(run_prep(m, ps, 1, s));
     const uint8_t* kv = (const uint8_t*)w.kv + (size_t)l * 2 * Mt * d * es;
     TRACK_TRY(run_attention(m, w.Qh, kv, kv + (size_t)Mt * d * es, w.attn, nseq, L, a.text_len, s));
     TRACK_TRY(run_gemm(m, w.attn, Ly.Wco, M, d, d, Ly.bco, EPI_RESID, nullptr, w.xres, d, s));
     // MLP
-    LAUNCH(ln_modulate(w.xres, M, d, scale2, shift2, 0, a.eps, w.h, m->dtype, s));
+    LAUNCH(run_ln(m, w.xres, M, d, scale2, shift2, 0, w.h, s));
     TRACK_TRY(run_gemm(m, w.h, Ly.W1, M, F, d, Ly.b1, EPI_GELU, nullptr, w.ffh, F, s));
     TRACK_TRY(run_gemm(m, w.ffh, Ly.W2, M, d, F, Ly.b2, EPI_RESID_GATE, gate2, w.xres, d, s));
   }
@@ -710,7 +722,7 @@ int track_profile_enable(int enable) {
 int track_profile_read(double* ms, double* flops, int64_t* launches) {
   if (!ms || !flops || !launches) return fail(TRACK_EINVAL, "NULL output");
   std::lock_guard<std::mutex> lk(g_prof_mu);
-  for (int c = 0; c < 2; ++c) {
+  for (int c = 0; c < 3; ++c) {
     ms[c] = 0;
     flops[c] = 0;
     launches[c] = 0;
