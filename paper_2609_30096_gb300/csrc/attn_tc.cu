@@ -2,9 +2,10 @@
 // O = softmax(Q K^T / sqrt(hd)) V per (sequence, head), no mask.
 //
 // One CTA per 128-query tile of one (sequence, head), 192 threads:
-//   warp 0      TMA: the Q tile once, then K and V tiles of 128 keys into a
-//               two-stage ring (3-D tensor maps [S*H, L, hd], 128-byte swizzle,
-//               zero fill past L).
+//   warp 0      TMA: the Q tile once, then K and V tiles of 128 keys, each
+//               through its own two-stage ring (lane 0 K, lane 1 V; 3-D tensor
+//               maps [S*H, L, hd], 128-byte swizzle, zero fill past L).  A K
+//               stage is released as soon as S = Q K^T of its tile completes.
 //   warp 1      allocates TMEM (O: hd columns; S: two 128-column buffers) and
 //               issues, from one thread, S(j+1) = Q K(j+1)^T while the softmax
 //               warps work on S(j), then O += P(j) V(j) once P(j) is ready.
@@ -39,9 +40,9 @@ template <int HD>
 struct AtShape {
   static constexpr uint32_t Q_BYTES = AT_BM * HD * 2;   // HD/64 boxes of [128 rows][128 B]
   static constexpr uint32_t KV_BYTES = AT_BN * HD * 2;  // one K or V tile
-  static constexpr uint32_t P_BYTES = AT_BM * AT_BN * 2;
+  static constexpr uint32_t P_BYTES = AT_BM * AT_BN * 2;  // one P buffer (two in smem)
   static constexpr int STAGES = 2;
-  static constexpr size_t SMEM = 1024 + Q_BYTES + 2 * STAGES * KV_BYTES + P_BYTES + 256;
+  static constexpr size_t SMEM = 1024 + Q_BYTES + 2 * STAGES * KV_BYTES + 2 * P_BYTES + 256;
   static constexpr uint32_t TMEM_COLS = 512;
 };
 
@@ -71,15 +72,17 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   uint8_t* sK = sQ + S::Q_BYTES;
   uint8_t* sV = sK + S::STAGES * S::KV_BYTES;
   uint8_t* sP = sV + S::STAGES * S::KV_BYTES;
-  uint64_t* bars = (uint64_t*)(sP + S::P_BYTES);
+  uint64_t* bars = (uint64_t*)(sP + 2 * S::P_BYTES);
   uint64_t* q_full = bars;
-  uint64_t* kv_full = bars + 1;   // [2]
-  uint64_t* kv_empty = bars + 3;  // [2]
-  uint64_t* s_full = bars + 5;    // [2]
-  uint64_t* p_full = bars + 7;
-  uint64_t* o_done = bars + 8;
-  uint64_t* done = bars + 9;
-  uint32_t* tmem_slot = (uint32_t*)(bars + 10);
+  uint64_t* k_full = bars + 1;    // [2] per K stage
+  uint64_t* k_empty = bars + 3;   // [2] freed once S = Q K^T of the tile has completed
+  uint64_t* v_full = bars + 5;    // [2] per V stage
+  uint64_t* v_empty = bars + 7;   // [2] freed once P V of the tile has completed
+  uint64_t* s_full = bars + 9;    // [2] per S buffer
+  uint64_t* p_full = bars + 11;   // [2] per P buffer
+  uint64_t* o_done = bars + 13;   // [2] P V of a tile using P buffer b has completed
+  uint64_t* done = bars + 15;
+  uint32_t* tmem_slot = (uint32_t*)(bars + 16);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -89,12 +92,14 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   if (threadIdx.x == 0) {
     mbar_init(su32(q_full), 1);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(su32(&kv_full[i]), 1);
-      mbar_init(su32(&kv_empty[i]), 1);
+      mbar_init(su32(&k_full[i]), 1);
+      mbar_init(su32(&k_empty[i]), 1);
+      mbar_init(su32(&v_full[i]), 1);
+      mbar_init(su32(&v_empty[i]), 1);
       mbar_init(su32(&s_full[i]), 1);
+      mbar_init(su32(&p_full[i]), 4);
+      mbar_init(su32(&o_done[i]), 1);
     }
-    mbar_init(su32(p_full), 4);
-    mbar_init(su32(o_done), 1);
     mbar_init(su32(done), 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -106,30 +111,34 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   const uint32_t tmem_base = *tmem_slot;
 
   if (warp == 0) {
-    if (lane == 0) {
-      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmQ) : "memory");
-      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmK) : "memory");
-      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmV) : "memory");
-      mbar_expect_tx(su32(q_full), S::Q_BYTES);
-      for (int b = 0; b < NB; ++b)
-        tma_load_3d(su32(sQ + b * AT_BM * 128), &tmQ, b * 64, q0, bh, su32(q_full));
+    // lane 0 streams Q and the K tiles, lane 1 the V tiles, each through its own ring
+    if (lane < 2) {
+      const bool kside = lane == 0;
+      const CUtensorMap* tm = kside ? &tmK : &tmV;
+      uint8_t* ring = kside ? sK : sV;
+      uint64_t* full = kside ? k_full : v_full;
+      uint64_t* empty = kside ? k_empty : v_empty;
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)tm) : "memory");
+      if (kside) {
+        asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmQ) : "memory");
+        mbar_expect_tx(su32(q_full), S::Q_BYTES);
+        for (int b = 0; b < NB; ++b)
+          tma_load_3d(su32(sQ + b * AT_BM * 128), &tmQ, b * 64, q0, bh, su32(q_full));
+      }
       uint32_t armed[2] = {0, 0};
       for (int kt = 0; kt < nkt; ++kt) {
         const int st = kt & 1;
-        if (!mbar_wait(su32(&kv_empty[st]), ((kt >> 1) & 1) ^ 1, abort_flag, err, 11)) break;
-        mbar_expect_tx(su32(&kv_full[st]), 2 * S::KV_BYTES);
-        for (int b = 0; b < NB; ++b) {
-          tma_load_3d(su32(sK + st * S::KV_BYTES + b * AT_BN * 128), &tmK, b * 64, kt * AT_BN, bh,
-                      su32(&kv_full[st]));
-          tma_load_3d(su32(sV + st * S::KV_BYTES + b * AT_BN * 128), &tmV, b * 64, kt * AT_BN, bh,
-                      su32(&kv_full[st]));
-        }
+        if (!mbar_wait(su32(&empty[st]), ((kt >> 1) & 1) ^ 1, abort_flag, err, 11)) break;
+        mbar_expect_tx(su32(&full[st]), S::KV_BYTES);
+        for (int b = 0; b < NB; ++b)
+          tma_load_3d(su32(ring + st * S::KV_BYTES + b * AT_BN * 128), tm, b * 64, kt * AT_BN, bh,
+                      su32(&full[st]));
         ++armed[st];
       }
       // Every copy this thread issued has landed before the CTA may exit.
-      mbar_drain(su32(q_full), 0, err, 15);
+      if (kside) mbar_drain(su32(q_full), 0, err, 15);
       for (int i = 0; i < 2; ++i)
-        if (armed[i] != 0) mbar_drain(su32(&kv_full[i]), (armed[i] - 1) & 1, err, 15);
+        if (armed[i] != 0) mbar_drain(su32(&full[i]), (armed[i] - 1) & 1, err, 15);
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -138,7 +147,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       const uint32_t qa = su32(sQ), pa = su32(sP);
       auto issue_s = [&](int kt) -> bool {
         const int st = kt & 1;
-        if (!mbar_wait(su32(&kv_full[st]), (kt >> 1) & 1, abort_flag, err, 12)) return false;
+        if (!mbar_wait(su32(&k_full[st]), (kt >> 1) & 1, abort_flag, err, 12)) return false;
         tc_fence_after();
         const uint32_t ka = su32(sK + st * S::KV_BYTES);
         const uint32_t d = tmem_base + TM_S0 + (uint32_t)(st * AT_BN);
@@ -148,6 +157,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                    sdesc_sw128(ka + (kk >> 2) * (AT_BN * 128) + (kk & 3) * 32), idS,
                    kk > 0 ? 1u : 0u);
         mma_commit(su32(&s_full[st]));
+        mma_commit(su32(&k_empty[st]));
         return true;
       };
       bool ok = mbar_wait(su32(q_full), 0, abort_flag, err, 13);
@@ -157,17 +167,19 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       }
       for (int kt = 0; ok && kt < nkt; ++kt) {
         if (kt + 1 < nkt && !issue_s(kt + 1)) break;
-        if (!mbar_wait(su32(p_full), kt & 1, abort_flag, err, 14)) break;
+        const int pb = kt & 1;  // P buffer of this tile (= its V stage)
+        if (!mbar_wait(su32(&v_full[pb]), (kt >> 1) & 1, abort_flag, err, 21)) break;
+        if (!mbar_wait(su32(&p_full[pb]), (kt >> 1) & 1, abort_flag, err, 14)) break;
         tc_fence_after();
-        const int st = kt & 1;
-        const uint32_t va = su32(sV + st * S::KV_BYTES);
+        const uint32_t va = su32(sV + pb * S::KV_BYTES);
+        const uint32_t pbuf = pa + pb * S::P_BYTES;
 #pragma unroll
         for (int kk = 0; kk < AT_BN / 16; ++kk)
-          mma_bf16(tmem_base, sdesc_sw128(pa + (kk >> 2) * (AT_BM * 128) + (kk & 3) * 32),
+          mma_bf16(tmem_base, sdesc_sw128(pbuf + (kk >> 2) * (AT_BM * 128) + (kk & 3) * 32),
                    sdesc_sw128_mn(va + kk * 16 * 128, AT_BN * 128), idO,
                    (kt > 0 || kk > 0) ? 1u : 0u);
-        mma_commit(su32(&kv_empty[st]));
-        mma_commit(su32(o_done));
+        mma_commit(su32(&v_empty[pb]));
+        mma_commit(su32(&o_done[pb]));
       }
       // Every MMA this thread issued has completed before TMEM is freed.
       mma_commit(su32(done));
@@ -188,30 +200,50 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       tc_fence_after();
       const uint32_t tS = tmem_base + lane_off + TM_S0 + (uint32_t)((kt & 1) * AT_BN);
       const int kbase = kt * AT_BN;
-      uint32_t r[32];
-      float mx = -INFINITY;
-#pragma unroll 1
-      for (int c = 0; c < AT_BN / 32; ++c) {
-        tmem_ld32(tS + c * 32, r);
+      const bool full = kbase + AT_BN <= Lk;  // no key of this tile is past Lk
+      uint32_t sv[AT_BN];                     // this row of S, one tile
 #pragma unroll
-        for (int i = 0; i < 32; ++i)
-          if (kbase + c * 32 + i < Lk) mx = fmaxf(mx, __uint_as_float(r[i]));
+      for (int c = 0; c < AT_BN / 32; ++c) tmem_ld32_nowait(tS + c * 32, sv + 32 * c);
+      tmem_ld_wait();
+      if (!full) {
+#pragma unroll
+        for (int i = 0; i < AT_BN; ++i)
+          if (kbase + i >= Lk) sv[i] = __float_as_uint(-INFINITY);
       }
+      // Row maximum as 16 independent partial maxima, then a tree: a single chain
+      // of 128 dependent max operations would dominate the softmax latency.
+      float pm[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) pm[j] = __uint_as_float(sv[j]);
+#pragma unroll
+      for (int i = 16; i < AT_BN; ++i) pm[i & 15] = fmaxf(pm[i & 15], __uint_as_float(sv[i]));
+#pragma unroll
+      for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+        for (int j = 0; j < w; ++j) pm[j] = fmaxf(pm[j], pm[j + w]);
+      const float mx = pm[0];
       const float mt = mx * scale_log2;
+      const int pb = kt & 1;
+      // P buffer pb was last read by P V of tile kt-2.
+      if (kt >= 2 && !warp_wait(su32(&o_done[pb]), ((kt >> 1) & 1) ^ 1, abort_flag, err, 18)) {
+        ok = false;
+        break;
+      }
       if (kt > 0) {
-        // P(kt-1) V(kt-1) must be complete before P is overwritten or O rescaled.
-        if (!warp_wait(su32(o_done), (kt - 1) & 1, abort_flag, err, 18)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
         const bool need = mt > m + 8.f;
         if (__any_sync(0xffffffffu, need)) {
+          // O is rescaled in TMEM: P V of tile kt-1 must have completed.
+          if (!warp_wait(su32(&o_done[pb ^ 1]), ((kt - 1) >> 1) & 1, abort_flag, err, 20)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
           const float alpha = need ? exp2_approx(m - mt) : 1.f;
           if (need) {
             m = mt;
             l *= alpha;
           }
+          uint32_t r[32];
 #pragma unroll 1
           for (int c = 0; c < HD / 32; ++c) {
             tmem_ld32(tO + c * 32, r);
@@ -224,34 +256,32 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       } else {
         m = mt;
       }
-      float rs = 0.f;
-#pragma unroll 1
-      for (int c = 0; c < AT_BN / 32; ++c) {
-        tmem_ld32(tS + c * 32, r);
-        uint32_t pk[16];
+      // P = exp2(S * scale - m); keys past Lk hold -inf and give 0.
+      float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // independent partial sums
+      const float nm = -m;
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const int k0 = kbase + c * 32 + 2 * i;
-          const float p0 = k0 < Lk ? exp2_approx(fmaf(__uint_as_float(r[2 * i]), scale_log2, -m)) : 0.f;
+      for (int cidx = 0; cidx < AT_BN / 8; ++cidx) {  // 16-byte chunks of 8 keys
+        uint32_t pk[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float p0 = exp2_approx(fmaf(__uint_as_float(sv[8 * cidx + 2 * i]), scale_log2, nm));
           const float p1 =
-              k0 + 1 < Lk ? exp2_approx(fmaf(__uint_as_float(r[2 * i + 1]), scale_log2, -m)) : 0.f;
-          rs += p0 + p1;
+              exp2_approx(fmaf(__uint_as_float(sv[8 * cidx + 2 * i + 1]), scale_log2, nm));
+          ps[2 * i] += p0;
+          ps[2 * i + 1] += p1;
           pk[i] = pack_bf16x2(p0, p1);
         }
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int cidx = c * 4 + j;  // 16-byte chunk of the row (8 keys)
-          uint8_t* dst = sP + (cidx >> 3) * (AT_BM * 128) + row * 128 + (((cidx & 7) ^ (row & 7)) << 4);
-          *reinterpret_cast<uint4*>(dst) = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
-        }
+        uint8_t* dst = sP + pb * S::P_BYTES + (cidx >> 3) * (AT_BM * 128) + row * 128 +
+                       (((cidx & 7) ^ (row & 7)) << 4);
+        *reinterpret_cast<uint4*>(dst) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
       }
-      l += rs;
+      l += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
       fence_async_shared();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(su32(p_full));
+      if (lane == 0) mbar_arrive(su32(&p_full[pb]));
     }
-    if (ok && warp_wait(su32(o_done), (nkt - 1) & 1, abort_flag, err, 19)) {
+    if (ok && warp_wait(su32(&o_done[(nkt - 1) & 1]), ((nkt - 1) >> 1) & 1, abort_flag, err, 19)) {
       tc_fence_after();
       const float inv = 1.f / l;
       const int qrow = q0 + row;

@@ -263,14 +263,74 @@ __global__ void __launch_bounds__(256) k_ln_mod(const float* __restrict__ x, int
   }
 }
 
+// Same computation with the row held in registers: VPL float4 per lane, d = 128 * VPL.
+// All loads of the row are issued before the first reduction.
+template <typename T, int VPL>
+__global__ void __launch_bounds__(256) k_ln_mod_r(const float* __restrict__ x, int M,
+                                                  const float* __restrict__ a,
+                                                  const float* __restrict__ b, int mode, float eps,
+                                                  T* __restrict__ out) {
+  constexpr int d = 128 * VPL;
+  const int lane = threadIdx.x & 31;
+  const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (row >= M) return;
+  const float4* xr = reinterpret_cast<const float4*>(x + row * d);
+  float4 v[VPL];
+#pragma unroll
+  for (int i = 0; i < VPL; ++i) v[i] = xr[lane + 32 * i];
+  // four independent partial sums per statistic (short dependency chains)
+  float s4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int i = 0; i < VPL; ++i) {
+    s4[0] += v[i].x; s4[1] += v[i].y; s4[2] += v[i].z; s4[3] += v[i].w;
+  }
+  const float mean = warp_sum((s4[0] + s4[1]) + (s4[2] + s4[3])) / (float)d;
+  float q4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int i = 0; i < VPL; ++i) {
+    float t;
+    t = v[i].x - mean; q4[0] = fmaf(t, t, q4[0]);
+    t = v[i].y - mean; q4[1] = fmaf(t, t, q4[1]);
+    t = v[i].z - mean; q4[2] = fmaf(t, t, q4[2]);
+    t = v[i].w - mean; q4[3] = fmaf(t, t, q4[3]);
+  }
+  const float rstd = 1.f / sqrtf(warp_sum((q4[0] + q4[1]) + (q4[2] + q4[3])) / (float)d + eps);
+  const float4* a4 = reinterpret_cast<const float4*>(a);
+  const float4* b4 = reinterpret_cast<const float4*>(b);
+  T* orow = out + row * d;
+  const float one = mode == 0 ? 1.f : 0.f;
+#pragma unroll
+  for (int i = 0; i < VPL; ++i) {
+    const int j = lane + 32 * i;
+    const float4 aa = a4[j], bb = b4[j];
+    store4(orow + 4 * j, fmaf((v[i].x - mean) * rstd, one + aa.x, bb.x),
+           fmaf((v[i].y - mean) * rstd, one + aa.y, bb.y),
+           fmaf((v[i].z - mean) * rstd, one + aa.z, bb.z),
+           fmaf((v[i].w - mean) * rstd, one + aa.w, bb.w));
+  }
+}
+
+template <typename T>
+static cudaError_t ln_dispatch(const float* x, int M, int d, const float* a, const float* b,
+                               int mode, float eps, T* out, cudaStream_t s) {
+  const int g = (M + 7) / 8;
+  switch (d % 128 == 0 ? d / 128 : 0) {
+#define LN_CASE(V) \
+  case V: k_ln_mod_r<T, V><<<g, 256, 0, s>>>(x, M, a, b, mode, eps, out); break;
+    LN_CASE(1) LN_CASE(2) LN_CASE(4) LN_CASE(6) LN_CASE(8) LN_CASE(12) LN_CASE(16) LN_CASE(24)
+    LN_CASE(32)
+#undef LN_CASE
+    default: k_ln_mod<T><<<g, 256, 0, s>>>(x, M, d, a, b, mode, eps, out);
+  }
+  return cudaGetLastError();
+}
+
 cudaError_t ln_modulate(const float* x, int M, int d, const float* a, const float* b, int mode,
                         float eps, void* out, int dtype, cudaStream_t s) {
   if (d % 4) return cudaErrorInvalidValue;
-  const int g = (M + 7) / 8;
-  if (dtype == BF16) k_ln_mod<bf16><<<g, 256, 0, s>>>(x, M, d, a, b, mode, eps, (bf16*)out);
-  else k_ln_mod<float><<<g, 256, 0, s>>>(x, M, d, a, b, mode, eps, (float*)out);
   count_launch();
-  return cudaGetLastError();
+  if (dtype == BF16) return ln_dispatch<bf16>(x, M, d, a, b, mode, eps, (bf16*)out, s);
+  return ln_dispatch<float>(x, M, d, a, b, mode, eps, (float*)out, s);
 }
 
 // ---------------------------------------------------------------- RMSNorm + RoPE + head split
@@ -363,6 +423,66 @@ __global__ void __launch_bounds__(256) k_qkv_prep(PrepArgs a, int nsec, int s0, 
   }
 }
 
+// bf16 variant with the row section in registers: CPL 8-element chunks per lane,
+// d = 256 * CPL; all loads are issued before the reduction.
+template <int CPL>
+__global__ void __launch_bounds__(256) k_qkv_prep_r(PrepArgs a, int nsec, int s0, int s1, int s2) {
+  constexpr int D = 256 * CPL;
+  const int lane = threadIdx.x & 31;
+  const int64_t gw = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int64_t r = gw / nsec;
+  if (r >= a.rows) return;
+  const int k = (int)(gw % nsec);
+  const int sec = k == 0 ? s0 : (k == 1 ? s1 : s2);
+  const int seq = (int)(r / a.L), l = (int)(r % a.L);
+  const bf16* src = (const bf16*)a.src + r * a.ld + a.off[sec];
+  float v[CPL][8];
+#pragma unroll
+  for (int j = 0; j < CPL; ++j) load8(src + 8 * (lane + 32 * j), v[j]);
+  const float* g = a.gain[sec];
+  float rstd = 1.f;
+  if (g != nullptr) {
+    float s8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int j = 0; j < CPL; ++j)
+#pragma unroll
+      for (int i = 0; i < 8; ++i) s8[i] = fmaf(v[j][i], v[j][i], s8[i]);
+    const float ss = ((s8[0] + s8[1]) + (s8[2] + s8[3])) + ((s8[4] + s8[5]) + (s8[6] + s8[7]));
+    rstd = 1.f / sqrtf(warp_sum(ss) / (float)D + a.eps);
+  }
+  const bool rot = a.rope && sec < 2;
+  const int s6 = a.hd / 6;
+  const int nf = (a.hd - 4 * s6) / 2, nh = s6;
+  const int pf = l / (a.Hp * a.Wp), ph = (l / a.Wp) % a.Hp, pw = l % a.Wp;
+  bf16* dst = (bf16*)a.dst[sec];
+#pragma unroll
+  for (int j = 0; j < CPL; ++j) {
+    const int e0 = 8 * (lane + 32 * j), h = e0 / a.hd, eh = e0 % a.hd;
+    if (g != nullptr) {
+      const float4 g0 = reinterpret_cast<const float4*>(g + e0)[0];
+      const float4 g1 = reinterpret_cast<const float4*>(g + e0)[1];
+      const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+#pragma unroll
+      for (int i = 0; i < 8; ++i) v[j][i] = v[j][i] * rstd * gg[i];
+    }
+    if (rot) {
+#pragma unroll
+      for (int p = 0; p < 4; ++p) {
+        const int jj = eh / 2 + p;
+        int idx;
+        if (jj < nf) idx = pf * nf + jj;
+        else if (jj < nf + nh) idx = a.Fp * nf + ph * nh + (jj - nf);
+        else idx = a.Fp * nf + a.Hp * nh + pw * nh + (jj - nf - nh);
+        const float2 cs = a.rope_tab[idx];
+        const float x0 = v[j][2 * p], x1 = v[j][2 * p + 1];
+        v[j][2 * p] = x0 * cs.x - x1 * cs.y;
+        v[j][2 * p + 1] = x0 * cs.y + x1 * cs.x;
+      }
+    }
+    store8(dst + (((int64_t)seq * a.H + h) * a.L + l) * a.hd + eh, v[j]);
+  }
+}
+
 cudaError_t qkv_prep(const PrepArgs& a, cudaStream_t s) {
   int secs[3] = {0, 0, 0}, nsec = 0;
   for (int i = 0; i < 3; ++i)
@@ -371,8 +491,18 @@ cudaError_t qkv_prep(const PrepArgs& a, cudaStream_t s) {
   if (a.d % 8 || a.hd % 8) return cudaErrorInvalidValue;
   const int64_t warps = (int64_t)a.rows * nsec;
   const int g = (int)((warps + 7) / 8);
-  if (a.dtype == BF16) k_qkv_prep<bf16><<<g, 256, 0, s>>>(a, nsec, secs[0], secs[1], secs[2]);
-  else k_qkv_prep<float><<<g, 256, 0, s>>>(a, nsec, secs[0], secs[1], secs[2]);
+  if (a.dtype == BF16) {
+    switch (a.d % 256 == 0 ? a.d / 256 : 0) {
+#define PREP_CASE(C) \
+  case C: k_qkv_prep_r<C><<<g, 256, 0, s>>>(a, nsec, secs[0], secs[1], secs[2]); break;
+      PREP_CASE(1) PREP_CASE(2) PREP_CASE(3) PREP_CASE(4) PREP_CASE(6) PREP_CASE(8) PREP_CASE(12)
+      PREP_CASE(16)
+#undef PREP_CASE
+      default: k_qkv_prep<bf16><<<g, 256, 0, s>>>(a, nsec, secs[0], secs[1], secs[2]);
+    }
+  } else {
+    k_qkv_prep<float><<<g, 256, 0, s>>>(a, nsec, secs[0], secs[1], secs[2]);
+  }
   count_launch();
   return cudaGetLastError();
 }

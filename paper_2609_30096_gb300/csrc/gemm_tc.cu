@@ -53,7 +53,8 @@ template <int BN, int STAGES>
 struct TcShape {
   static constexpr uint32_t A_BYTES = BM * BK * 2;
   static constexpr uint32_t B_BYTES = BN * BK * 2;
-  static constexpr uint32_t TMEM_COLS = 2 * BN;
+  // two accumulators of BN columns; TMEM is allocated in powers of two columns
+  static constexpr uint32_t TMEM_COLS = 2 * BN <= 256 ? 256 : 512;
   static constexpr uint32_t STG_BYTES = 4 * 2 * 4096;  // two 32x128-byte boxes per epilogue warp
   static constexpr size_t SMEM = 1024 + (size_t)STAGES * (A_BYTES + B_BYTES) + STG_BYTES + 256;
 };
@@ -340,7 +341,23 @@ cudaError_t gemm_bf16_tc(const void* A, const void* W, const GemmArgs& g, cudaSt
   if (g.bias != nullptr && (((uintptr_t)g.bias) & 15)) return cudaErrorMisalignedAddress;
   if (g.epi == EPI_RESID_GATE && (g.gate == nullptr || (((uintptr_t)g.gate) & 15)))
     return cudaErrorInvalidValue;
-  if (g.N >= 512 && g.N % 256 == 0) return launch_tc<256, 4>(A, W, g, s);
+  // Tile width by a makespan model: every CTA of a wave runs concurrently, so a
+  // launch costs about rounds x (BN + per-tile overhead).  The overhead (150
+  // columns' worth) is fitted to measured tile times: a 192-wide tile takes about
+  // 0.85x the time of a 256-wide one.  Ties go to the wider tile.
+  const int m_tiles = (g.M + BM - 1) / BM, sms = num_sms();
+  int best_bn = 256;
+  long best_cost = -1;
+  for (int bn : {256, 192, 128}) {
+    const long tiles = (long)m_tiles * ((g.N + bn - 1) / bn);
+    const long cost = ((tiles + sms - 1) / sms) * (bn + 150);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best_bn = bn;
+    }
+  }
+  if (best_bn == 256) return launch_tc<256, 4>(A, W, g, s);
+  if (best_bn == 192) return launch_tc<192, 4>(A, W, g, s);
   return launch_tc<128, 6>(A, W, g, s);
 }
 
