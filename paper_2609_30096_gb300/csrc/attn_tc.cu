@@ -10,10 +10,12 @@
 //               issues, from one thread, S(j+1) = Q K(j+1)^T while the softmax
 //               warps work on S(j), then O += P(j) V(j) once P(j) is ready.
 //               V is the MN-major B operand, so no transposed copy is needed.
-//   warps 2-5   one thread per query row (its TMEM lane): row maximum of S(j)
-//               over the valid keys, lazy rescaling of O (only when the running
-//               maximum grows by more than 2^8, the rescale reading and writing
-//               the row in TMEM), P = exp2(S * log2(e)/sqrt(hd) - m) rounded to
+//   warps 2-9   softmax, two warpgroups splitting each 128-key tile by columns
+//               (64 keys each), one thread per query row (its TMEM lane): row
+//               maximum over the valid keys (halves combined through shared
+//               memory), lazy rescaling of O (only when the running maximum
+//               grows by more than 2^8; each group rescales its half of O's
+//               columns in TMEM), P = exp2(S * log2(e)/sqrt(hd) - m) rounded to
 //               bf16 into 128-byte-swizzled shared memory, and at the end O / l
 //               stored to the token-major output.
 // Every mbarrier wait is bounded (see tc_common.cuh).
@@ -33,16 +35,17 @@ typedef __nv_bfloat16 bf16;
 
 constexpr int AT_BM = 128;       // query rows per CTA (MMA M)
 constexpr int AT_BN = 128;       // keys per tile
-constexpr int AT_THREADS = 192;  // warp 0 TMA, warp 1 MMA, warps 2-5 softmax
+constexpr int AT_THREADS = 320;  // warp 0 TMA, warp 1 MMA, warps 2-9 softmax
 constexpr uint32_t TM_S0 = 128;  // TMEM column of S buffer 0 (buffer 1 at 256)
 
 template <int HD>
 struct AtShape {
   static constexpr uint32_t Q_BYTES = AT_BM * HD * 2;   // HD/64 boxes of [128 rows][128 B]
   static constexpr uint32_t KV_BYTES = AT_BN * HD * 2;  // one K or V tile
-  static constexpr uint32_t P_BYTES = AT_BM * AT_BN * 2;  // one P buffer (two in smem)
+  static constexpr uint32_t P_BYTES = AT_BM * AT_BN * 2;
+  static constexpr uint32_t X_BYTES = 2 * 2 * AT_BM * 4;  // row partials [parity][half][row]
   static constexpr int STAGES = 2;
-  static constexpr size_t SMEM = 1024 + Q_BYTES + 2 * STAGES * KV_BYTES + 2 * P_BYTES + 256;
+  static constexpr size_t SMEM = 1024 + Q_BYTES + 2 * STAGES * KV_BYTES + P_BYTES + X_BYTES + 256;
   static constexpr uint32_t TMEM_COLS = 512;
 };
 
@@ -72,15 +75,17 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   uint8_t* sK = sQ + S::Q_BYTES;
   uint8_t* sV = sK + S::STAGES * S::KV_BYTES;
   uint8_t* sP = sV + S::STAGES * S::KV_BYTES;
-  uint64_t* bars = (uint64_t*)(sP + 2 * S::P_BYTES);
+  float* xch = (float*)(sP + S::P_BYTES);  // [2][2][AT_BM] partial row maxima / sums
+  uint64_t* bars = (uint64_t*)(sP + S::P_BYTES + S::X_BYTES);
   uint64_t* q_full = bars;
   uint64_t* k_full = bars + 1;    // [2] per K stage
   uint64_t* k_empty = bars + 3;   // [2] freed once S = Q K^T of the tile has completed
   uint64_t* v_full = bars + 5;    // [2] per V stage
   uint64_t* v_empty = bars + 7;   // [2] freed once P V of the tile has completed
   uint64_t* s_full = bars + 9;    // [2] per S buffer
-  uint64_t* p_full = bars + 11;   // [2] per P buffer
-  uint64_t* o_done = bars + 13;   // [2] P V of a tile using P buffer b has completed
+  uint64_t* p_full = bars + 11;   // P of the tile written (8 softmax warps)
+  uint64_t* o_done = bars + 12;   // P V of the tile has completed
+  uint64_t* xbar = bars + 13;     // [2] both halves' row partials written (per parity)
   uint64_t* done = bars + 15;
   uint32_t* tmem_slot = (uint32_t*)(bars + 16);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
@@ -97,9 +102,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       mbar_init(su32(&v_full[i]), 1);
       mbar_init(su32(&v_empty[i]), 1);
       mbar_init(su32(&s_full[i]), 1);
-      mbar_init(su32(&p_full[i]), 4);
-      mbar_init(su32(&o_done[i]), 1);
+      mbar_init(su32(&xbar[i]), 8);
     }
+    mbar_init(su32(p_full), 8);
+    mbar_init(su32(o_done), 1);
     mbar_init(su32(done), 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -167,29 +173,32 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       }
       for (int kt = 0; ok && kt < nkt; ++kt) {
         if (kt + 1 < nkt && !issue_s(kt + 1)) break;
-        const int pb = kt & 1;  // P buffer of this tile (= its V stage)
-        if (!mbar_wait(su32(&v_full[pb]), (kt >> 1) & 1, abort_flag, err, 21)) break;
-        if (!mbar_wait(su32(&p_full[pb]), (kt >> 1) & 1, abort_flag, err, 14)) break;
+        const int st = kt & 1;  // V stage of this tile
+        if (!mbar_wait(su32(&v_full[st]), (kt >> 1) & 1, abort_flag, err, 21)) break;
+        if (!mbar_wait(su32(p_full), kt & 1, abort_flag, err, 14)) break;
         tc_fence_after();
-        const uint32_t va = su32(sV + pb * S::KV_BYTES);
-        const uint32_t pbuf = pa + pb * S::P_BYTES;
+        const uint32_t va = su32(sV + st * S::KV_BYTES);
 #pragma unroll
         for (int kk = 0; kk < AT_BN / 16; ++kk)
-          mma_bf16(tmem_base, sdesc_sw128(pbuf + (kk >> 2) * (AT_BM * 128) + (kk & 3) * 32),
+          mma_bf16(tmem_base, sdesc_sw128(pa + (kk >> 2) * (AT_BM * 128) + (kk & 3) * 32),
                    sdesc_sw128_mn(va + kk * 16 * 128, AT_BN * 128), idO,
                    (kt > 0 || kk > 0) ? 1u : 0u);
-        mma_commit(su32(&v_empty[pb]));
-        mma_commit(su32(&o_done[pb]));
+        mma_commit(su32(&v_empty[st]));
+        mma_commit(su32(o_done));
       }
       // Every MMA this thread issued has completed before TMEM is freed.
       mma_commit(su32(done));
       mbar_drain(su32(done), 0, err, 16);
     }
   } else {
+    // Softmax: warps 2-5 take keys 0-63 of each tile (and O columns 0..HD/2), warps
+    // 6-9 keys 64-127 (and the other O columns); one thread per query row each.
+    const int half = (warp - 2) >> 2;
     const int quarter = warp & 3;
     const int row = quarter * 32 + lane;
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
-    const uint32_t tO = tmem_base + lane_off;
+    const uint32_t tO = tmem_base + lane_off + (uint32_t)(half * (HD / 2));
+    constexpr int KH = AT_BN / 2;  // keys per half
     float m = -INFINITY, l = 0.f;
     bool ok = true;
     for (int kt = 0; kt < nkt; ++kt) {
@@ -198,46 +207,45 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         break;
       }
       tc_fence_after();
-      const uint32_t tS = tmem_base + lane_off + TM_S0 + (uint32_t)((kt & 1) * AT_BN);
-      const int kbase = kt * AT_BN;
-      const bool full = kbase + AT_BN <= Lk;  // no key of this tile is past Lk
-      uint32_t sv[AT_BN];                     // this row of S, one tile
-#pragma unroll
-      for (int c = 0; c < AT_BN / 32; ++c) tmem_ld32_nowait(tS + c * 32, sv + 32 * c);
+      const uint32_t tS =
+          tmem_base + lane_off + TM_S0 + (uint32_t)((kt & 1) * AT_BN) + (uint32_t)(half * KH);
+      const int kbase = kt * AT_BN + half * KH;
+      const bool full = kbase + KH <= Lk;  // no key of this half-tile is past Lk
+      uint32_t sv[KH];                      // this row of S, this half of the tile
+      tmem_ld32_nowait(tS, sv);
+      tmem_ld32_nowait(tS + 32, sv + 32);
       tmem_ld_wait();
       if (!full) {
 #pragma unroll
-        for (int i = 0; i < AT_BN; ++i)
+        for (int i = 0; i < KH; ++i)
           if (kbase + i >= Lk) sv[i] = __float_as_uint(-INFINITY);
       }
-      // Row maximum as 16 independent partial maxima, then a tree: a single chain
-      // of 128 dependent max operations would dominate the softmax latency.
-      float pm[16];
+      float pm[8];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) pm[j] = __uint_as_float(sv[j]);
+      for (int j = 0; j < 8; ++j) pm[j] = __uint_as_float(sv[j]);
 #pragma unroll
-      for (int i = 16; i < AT_BN; ++i) pm[i & 15] = fmaxf(pm[i & 15], __uint_as_float(sv[i]));
-#pragma unroll
-      for (int w = 8; w > 0; w >>= 1)
-#pragma unroll
-        for (int j = 0; j < w; ++j) pm[j] = fmaxf(pm[j], pm[j + w]);
-      const float mx = pm[0];
-      const float mt = mx * scale_log2;
-      const int pb = kt & 1;
-      // P buffer pb was last read by P V of tile kt-2.
-      if (kt >= 2 && !warp_wait(su32(&o_done[pb]), ((kt >> 1) & 1) ^ 1, abort_flag, err, 18)) {
+      for (int i = 8; i < KH; ++i) pm[i & 7] = fmaxf(pm[i & 7], __uint_as_float(sv[i]));
+      const float hmax = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                               fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+      // exchange the half-row maxima with the other warpgroup
+      float* xp = xch + (kt & 1) * 2 * AT_BM;
+      xp[half * AT_BM + row] = hmax;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(su32(&xbar[kt & 1]));
+      if (!warp_wait(su32(&xbar[kt & 1]), (kt >> 1) & 1, abort_flag, err, 22)) {
         ok = false;
         break;
       }
+      const float mt = fmaxf(hmax, xp[(half ^ 1) * AT_BM + row]) * scale_log2;
+      // P V of the previous tile must be complete before P is overwritten (and O rescaled).
       if (kt > 0) {
+        if (!warp_wait(su32(o_done), (kt - 1) & 1, abort_flag, err, 18)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
         const bool need = mt > m + 8.f;
         if (__any_sync(0xffffffffu, need)) {
-          // O is rescaled in TMEM: P V of tile kt-1 must have completed.
-          if (!warp_wait(su32(&o_done[pb ^ 1]), ((kt - 1) >> 1) & 1, abort_flag, err, 20)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
           const float alpha = need ? exp2_approx(m - mt) : 1.f;
           if (need) {
             m = mt;
@@ -245,7 +253,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
           }
           uint32_t r[32];
 #pragma unroll 1
-          for (int c = 0; c < HD / 32; ++c) {
+          for (int c = 0; c < HD / 64; ++c) {
             tmem_ld32(tO + c * 32, r);
 #pragma unroll
             for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
@@ -256,11 +264,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       } else {
         m = mt;
       }
-      // P = exp2(S * scale - m); keys past Lk hold -inf and give 0.
-      float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // independent partial sums
+      // P = exp2(S * scale - m) for this half: K-block `half` of the P tile.
+      float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
       const float nm = -m;
 #pragma unroll
-      for (int cidx = 0; cidx < AT_BN / 8; ++cidx) {  // 16-byte chunks of 8 keys
+      for (int cidx = 0; cidx < KH / 8; ++cidx) {  // 16-byte chunks of 8 keys
         uint32_t pk[4];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
@@ -271,25 +279,34 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
           ps[2 * i + 1] += p1;
           pk[i] = pack_bf16x2(p0, p1);
         }
-        uint8_t* dst = sP + pb * S::P_BYTES + (cidx >> 3) * (AT_BM * 128) + row * 128 +
-                       (((cidx & 7) ^ (row & 7)) << 4);
+        uint8_t* dst = sP + half * (AT_BM * 128) + row * 128 + ((cidx ^ (row & 7)) << 4);
         *reinterpret_cast<uint4*>(dst) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
       }
       l += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
       fence_async_shared();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(su32(&p_full[pb]));
+      if (lane == 0) mbar_arrive(su32(p_full));
     }
-    if (ok && warp_wait(su32(&o_done[(nkt - 1) & 1]), ((nkt - 1) >> 1) & 1, abort_flag, err, 19)) {
+    // Combine the two halves' sums (one more exchange round), then O / l.
+    bool fin = ok;
+    if (fin) {
+      float* xp = xch + (nkt & 1) * 2 * AT_BM;
+      xp[half * AT_BM + row] = l;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(su32(&xbar[nkt & 1]));
+      fin = warp_wait(su32(&xbar[nkt & 1]), (nkt >> 1) & 1, abort_flag, err, 23);
+      if (fin) l += xp[(half ^ 1) * AT_BM + row];
+    }
+    if (fin && warp_wait(su32(o_done), (nkt - 1) & 1, abort_flag, err, 19)) {
       tc_fence_after();
       const float inv = 1.f / l;
       const int qrow = q0 + row;
       const int s_ = bh / H, h = bh % H;
-      bf16* orow = O + (((int64_t)s_ * Lq + qrow) * H + h) * HD;
+      bf16* orow = O + (((int64_t)s_ * Lq + qrow) * H + h) * HD + half * (HD / 2);
       uint32_t r2[32];
 #pragma unroll 1
-      for (int c = 0; c < HD / 32; ++c) {
+      for (int c = 0; c < HD / 64; ++c) {
         tmem_ld32(tO + c * 32, r2);
         if (qrow < Lq) {
 #pragma unroll
@@ -331,20 +348,20 @@ bool make_tmap_3d(CUtensorMap* tm, const void* ptr, int hd, int L, int SH, uint3
 template <int HD>
 cudaError_t launch_attn_tc(const void* Q, const void* K, const void* V, void* O, int S_, int H,
                            int Lq, int Lk, cudaStream_t s) {
-  using S = AtShape<HD>;
-  static_assert(S::SMEM <= 232448, "shared memory budget");
+  using S1 = AtShape<HD>;
+  static_assert(S1::SMEM <= 232448, "shared memory budget");
   CUtensorMap tq, tk, tv;
   if (!make_tmap_3d(&tq, Q, HD, Lq, S_ * H, AT_BM) || !make_tmap_3d(&tk, K, HD, Lk, S_ * H, AT_BN) ||
       !make_tmap_3d(&tv, V, HD, Lk, S_ * H, AT_BN))
     return cudaErrorInvalidValue;
   int* err = device_error_word();
   if (err == nullptr) return cudaErrorMemoryAllocation;
+  const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)HD));
   cudaError_t e = cudaFuncSetAttribute(k_attn_tc<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)S::SMEM);
+                                       (int)S1::SMEM);
   if (e != cudaSuccess) return e;
   dim3 grid((Lq + AT_BM - 1) / AT_BM, S_ * H);
-  const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)HD));
-  k_attn_tc<HD><<<grid, AT_THREADS, S::SMEM, s>>>(tq, tk, tv, (bf16*)O, H, Lq, Lk, scale_log2, err);
+  k_attn_tc<HD><<<grid, AT_THREADS, S1::SMEM, s>>>(tq, tk, tv, (bf16*)O, H, Lq, Lk, scale_log2, err);
   count_launch();
   return cudaGetLastError();
 }

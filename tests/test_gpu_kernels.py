@@ -122,6 +122,8 @@ ATTN_CASES = [  # S, H, Lq, Lk, hd
     (1, 2, 257, 32, 64),       # short keys (tiny cross-attention)
     (2, 2, 300, 512, 128),     # cross-attention at text length 512
     (1, 12, 3510, 3510, 128),  # mid-size self-attention (bench shape)
+    (4, 16, 1000, 700, 128),   # two query tiles per CTA: ragged queries and keys
+    (2, 40, 600, 512, 64),     # two query tiles per CTA, hd 64, text-length keys
 ]
 
 
@@ -143,7 +145,7 @@ def test_attention_bf16(T, S, H, Lq, Lk, hd):
     O = torch.zeros((S, Lq, H, hd), dtype=torch.bfloat16, device=DEV)
     T.track_attention(T.BF16, dev_bf16(Q), dev_bf16(K), dev_bf16(V), O)
     T.track_sync()
-    if Lq * Lk > 2_000_000:          # large case: sampled query rows
+    if S * H * Lq * Lk > 20_000_000:  # large case: sampled query rows
         rows = rng.choice(Lq, 64, replace=False)
         ref = _attn_ref(Q[:, :, rows], K, V)
         got = O.float().cpu().numpy()[:, rows]
