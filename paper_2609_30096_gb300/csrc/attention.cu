@@ -21,9 +21,7 @@ constexpr int F32_ROWS = 4;   // query rows per warp
 constexpr int F32_KT = 32;    // keys per tile
 
 template <int HD>
-__global__ void __launch_bounds__(128) k_attn_f32(const float* __restrict__ Q,
-                                                  const float* __restrict__ K,
-                                                  const float* __restrict__ V,
+__global__ void __launch_bounds__(128) k_attn_f32(AttnOperand Qo, AttnOperand Ko, AttnOperand Vo,
                                                   float* __restrict__ O, int H, int Lq, int Lk,
                                                   float scale) {
   constexpr int DV = HD / 32;
@@ -32,12 +30,13 @@ __global__ void __launch_bounds__(128) k_attn_f32(const float* __restrict__ Q,
   __shared__ float sQ[4 * F32_ROWS][HD];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int bh = blockIdx.y, q0 = blockIdx.x * 4 * F32_ROWS;
-  const float* Qg = Q + (int64_t)bh * Lq * HD;
-  const float* Kg = K + (int64_t)bh * Lk * HD;
-  const float* Vg = V + (int64_t)bh * Lk * HD;
+  const int sq = bh / H, hq = bh % H;
+  const float* Qg = (const float*)Qo.ptr + sq * Qo.ss + hq * Qo.hs;
+  const float* Kg = (const float*)Ko.ptr + sq * Ko.ss + hq * Ko.hs;
+  const float* Vg = (const float*)Vo.ptr + sq * Vo.ss + hq * Vo.hs;
   for (int i = threadIdx.x; i < 4 * F32_ROWS * HD; i += blockDim.x) {
     const int r = i / HD, c = i % HD;
-    sQ[r][c] = (q0 + r < Lq) ? Qg[(int64_t)(q0 + r) * HD + c] : 0.f;
+    sQ[r][c] = (q0 + r < Lq) ? Qg[(int64_t)(q0 + r) * Qo.ls + c] : 0.f;
   }
   float m[F32_ROWS], l[F32_ROWS], o[F32_ROWS][DV];
 #pragma unroll
@@ -52,8 +51,8 @@ __global__ void __launch_bounds__(128) k_attn_f32(const float* __restrict__ Q,
     for (int i = threadIdx.x; i < F32_KT * HD; i += blockDim.x) {
       const int r = i / HD, c = i % HD;
       const bool ok = k0 + r < Lk;
-      sK[r][c] = ok ? Kg[(int64_t)(k0 + r) * HD + c] : 0.f;
-      sV[r][c] = ok ? Vg[(int64_t)(k0 + r) * HD + c] : 0.f;
+      sK[r][c] = ok ? Kg[(int64_t)(k0 + r) * Ko.ls + c] : 0.f;
+      sV[r][c] = ok ? Vg[(int64_t)(k0 + r) * Vo.ls + c] : 0.f;
     }
     __syncthreads();
     const bool valid = k0 + lane < Lk;
@@ -82,12 +81,11 @@ __global__ void __launch_bounds__(128) k_attn_f32(const float* __restrict__ Q,
       }
     }
   }
-  const int S_ = bh / H, h = bh % H;
 #pragma unroll
   for (int i = 0; i < F32_ROWS; ++i) {
     const int row = q0 + warp * F32_ROWS + i;
     if (row >= Lq) continue;
-    float* orow = O + (((int64_t)S_ * Lq + row) * H + h) * HD;
+    float* orow = O + (((int64_t)sq * Lq + row) * H + hq) * HD;
 #pragma unroll
     for (int d = 0; d < DV; ++d) orow[lane + 32 * d] = o[i][d] / l[i];
   }
@@ -95,13 +93,8 @@ __global__ void __launch_bounds__(128) k_attn_f32(const float* __restrict__ Q,
 
 }  // namespace
 
-cudaError_t attention_bf16(const void* Q, const void* K, const void* V, void* O, int S, int H,
-                           int Lq, int Lk, int hd, cudaStream_t s) {
-  return attention_bf16_tc(Q, K, V, O, S, H, Lq, Lk, hd, s);
-}
-
-cudaError_t attention_f32(const float* Q, const float* K, const float* V, float* O, int S, int H,
-                          int Lq, int Lk, int hd, cudaStream_t s) {
+cudaError_t attention_f32(const AttnOperand& Q, const AttnOperand& K, const AttnOperand& V,
+                          float* O, int S, int H, int Lq, int Lk, int hd, cudaStream_t s) {
   if (S <= 0 || Lq <= 0) return cudaSuccess;
   if (Lk <= 0) return cudaErrorInvalidValue;
   dim3 grid((Lq + 4 * F32_ROWS - 1) / (4 * F32_ROWS), S * H);

@@ -3,9 +3,10 @@
 //
 // One CTA per 128-query tile of one (sequence, head), 192 threads:
 //   warp 0      TMA: the Q tile once, then K and V tiles of 128 keys, each
-//               through its own two-stage ring (lane 0 K, lane 1 V; 3-D tensor
-//               maps [S*H, L, hd], 128-byte swizzle, zero fill past L).  A K
-//               stage is released as soon as S = Q K^T of its tile completes.
+//               through its own two-stage ring (lane 0 K, lane 1 V; 4-D tensor
+//               maps over head-major or token-major operands, 128-byte swizzle,
+//               zero fill past L).  A K stage is released as soon as S = Q K^T
+//               of its tile completes.
 //   warp 1      allocates TMEM (O: hd columns; S: two 128-column buffers) and
 //               issues, from one thread, S(j+1) = Q K(j+1)^T while the softmax
 //               warps work on S(j), then O += P(j) V(j) once P(j) is ready.
@@ -54,6 +55,15 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&t);
 }
 
+// Loads a box of rows l0.. (64 columns from col) of head h of sequence sq; the
+// tensor map's dimensions are (hd, H, L, S) for a token-major operand and
+// (hd, L, H, S) for a head-major one.
+__device__ __forceinline__ void tma_load_rows(uint32_t dst, const CUtensorMap* tm, int tok, int col,
+                                              int l0, int h, int sq, uint32_t bar) {
+  if (tok) tma_load_4d(dst, tm, col, h, l0, sq, bar);
+  else tma_load_4d(dst, tm, col, l0, h, sq, bar);
+}
+
 // Lane 0 waits, the whole warp learns the outcome.
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
                                           int* err, int code) {
@@ -66,7 +76,7 @@ template <int HD>
 __global__ void __launch_bounds__(AT_THREADS, 1)
     k_attn_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
               const __grid_constant__ CUtensorMap tmV, bf16* __restrict__ O, int H, int Lq, int Lk,
-              float scale_log2, int* err) {
+              float scale_log2, int q_tok, int kv_tok, int* err) {
   using S = AtShape<HD>;
   constexpr int NB = HD / 64;  // 64-column boxes per row of Q/K/V
   extern __shared__ uint8_t smem_raw[];
@@ -92,6 +102,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int bh = blockIdx.y, q0 = blockIdx.x * AT_BM;
+  const int sq = bh / H, hq = bh % H;
   const int nkt = (Lk + AT_BN - 1) / AT_BN;
 
   if (threadIdx.x == 0) {
@@ -129,7 +140,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmQ) : "memory");
         mbar_expect_tx(su32(q_full), S::Q_BYTES);
         for (int b = 0; b < NB; ++b)
-          tma_load_3d(su32(sQ + b * AT_BM * 128), &tmQ, b * 64, q0, bh, su32(q_full));
+          tma_load_rows(su32(sQ + b * AT_BM * 128), &tmQ, q_tok, b * 64, q0, hq, sq, su32(q_full));
       }
       uint32_t armed[2] = {0, 0};
       for (int kt = 0; kt < nkt; ++kt) {
@@ -137,8 +148,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         if (!mbar_wait(su32(&empty[st]), ((kt >> 1) & 1) ^ 1, abort_flag, err, 11)) break;
         mbar_expect_tx(su32(&full[st]), S::KV_BYTES);
         for (int b = 0; b < NB; ++b)
-          tma_load_3d(su32(ring + st * S::KV_BYTES + b * AT_BN * 128), tm, b * 64, kt * AT_BN, bh,
-                      su32(&full[st]));
+          tma_load_rows(su32(ring + st * S::KV_BYTES + b * AT_BN * 128), tm, kv_tok, b * 64,
+                        kt * AT_BN, hq, sq, su32(&full[st]));
         ++armed[st];
       }
       // Every copy this thread issued has landed before the CTA may exit.
@@ -302,8 +313,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       tc_fence_after();
       const float inv = 1.f / l;
       const int qrow = q0 + row;
-      const int s_ = bh / H, h = bh % H;
-      bf16* orow = O + (((int64_t)s_ * Lq + qrow) * H + h) * HD + half * (HD / 2);
+      bf16* orow = O + (((int64_t)sq * Lq + qrow) * H + hq) * HD + half * (HD / 2);
       uint32_t r2[32];
 #pragma unroll 1
       for (int c = 0; c < HD / 64; ++c) {
@@ -332,27 +342,46 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   }
 }
 
-// 3-D tensor map of head-major [SH, L, hd] bf16, box [1, rows, 64].
-bool make_tmap_3d(CUtensorMap* tm, const void* ptr, int hd, int L, int SH, uint32_t rows) {
+// 4-D tensor map of one operand, dimensions ordered by increasing stride:
+// (hd, H, L, S) when token-major (hs < ls), (hd, L, H, S) when head-major;
+// the box covers 64 columns of `rows` consecutive positions of one head.
+bool make_tmap_op(CUtensorMap* tm, const AttnOperand& op, int hd, int L, int H, int S_,
+                  uint32_t rows, int* tok) {
   EncodeTiledFn enc = encode_tiled_fn();
   if (enc == nullptr) return false;
-  cuuint64_t dims[3] = {(cuuint64_t)hd, (cuuint64_t)L, (cuuint64_t)SH};
-  cuuint64_t strides[2] = {(cuuint64_t)hd * 2, (cuuint64_t)L * hd * 2};
-  cuuint32_t box[3] = {64, rows, 1};
-  cuuint32_t estr[3] = {1, 1, 1};
-  return enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
+  *tok = op.hs < op.ls ? 1 : 0;
+  cuuint64_t dims[4], strides[3];
+  cuuint32_t box[4];
+  dims[0] = (cuuint64_t)hd;
+  box[0] = 64;
+  if (*tok) {
+    dims[1] = (cuuint64_t)H; dims[2] = (cuuint64_t)L;
+    strides[0] = (cuuint64_t)op.hs * 2; strides[1] = (cuuint64_t)op.ls * 2;
+    box[1] = 1; box[2] = rows;
+  } else {
+    dims[1] = (cuuint64_t)L; dims[2] = (cuuint64_t)H;
+    strides[0] = (cuuint64_t)op.ls * 2; strides[1] = (cuuint64_t)op.hs * 2;
+    box[1] = rows; box[2] = 1;
+  }
+  dims[3] = (cuuint64_t)S_;
+  strides[2] = (cuuint64_t)op.ss * 2;
+  box[3] = 1;
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  return enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(op.ptr), dims, strides, box,
              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 template <int HD>
-cudaError_t launch_attn_tc(const void* Q, const void* K, const void* V, void* O, int S_, int H,
-                           int Lq, int Lk, cudaStream_t s) {
+cudaError_t launch_attn_tc(const AttnOperand& Q, const AttnOperand& K, const AttnOperand& V,
+                           void* O, int S_, int H, int Lq, int Lk, cudaStream_t s) {
   using S1 = AtShape<HD>;
   static_assert(S1::SMEM <= 232448, "shared memory budget");
   CUtensorMap tq, tk, tv;
-  if (!make_tmap_3d(&tq, Q, HD, Lq, S_ * H, AT_BM) || !make_tmap_3d(&tk, K, HD, Lk, S_ * H, AT_BN) ||
-      !make_tmap_3d(&tv, V, HD, Lk, S_ * H, AT_BN))
+  int q_tok = 0, k_tok = 0, v_tok = 0;
+  if (!make_tmap_op(&tq, Q, HD, Lq, H, S_, AT_BM, &q_tok) ||
+      !make_tmap_op(&tk, K, HD, Lk, H, S_, AT_BN, &k_tok) ||
+      !make_tmap_op(&tv, V, HD, Lk, H, S_, AT_BN, &v_tok) || k_tok != v_tok)
     return cudaErrorInvalidValue;
   int* err = device_error_word();
   if (err == nullptr) return cudaErrorMemoryAllocation;
@@ -361,18 +390,19 @@ cudaError_t launch_attn_tc(const void* Q, const void* K, const void* V, void* O,
                                        (int)S1::SMEM);
   if (e != cudaSuccess) return e;
   dim3 grid((Lq + AT_BM - 1) / AT_BM, S_ * H);
-  k_attn_tc<HD><<<grid, AT_THREADS, S1::SMEM, s>>>(tq, tk, tv, (bf16*)O, H, Lq, Lk, scale_log2, err);
+  k_attn_tc<HD><<<grid, AT_THREADS, S1::SMEM, s>>>(tq, tk, tv, (bf16*)O, H, Lq, Lk, scale_log2,
+                                                   q_tok, k_tok, err);
   count_launch();
   return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t attention_bf16_tc(const void* Q, const void* K, const void* V, void* O, int S, int H,
-                              int Lq, int Lk, int hd, cudaStream_t s) {
+cudaError_t attention_bf16(const AttnOperand& Q, const AttnOperand& K, const AttnOperand& V,
+                           void* O, int S, int H, int Lq, int Lk, int hd, cudaStream_t s) {
   if (S <= 0 || Lq <= 0) return cudaSuccess;
   if (Lk <= 0 || S * H > 65535) return cudaErrorInvalidValue;
-  if ((((uintptr_t)Q) | ((uintptr_t)K) | ((uintptr_t)V) | ((uintptr_t)O)) & 15)
+  if ((((uintptr_t)Q.ptr) | ((uintptr_t)K.ptr) | ((uintptr_t)V.ptr) | ((uintptr_t)O)) & 15)
     return cudaErrorMisalignedAddress;
   if (hd == 128) return launch_attn_tc<128>(Q, K, V, O, S, H, Lq, Lk, s);
   if (hd == 64) return launch_attn_tc<64>(Q, K, V, O, S, H, Lq, Lk, s);

@@ -366,142 +366,113 @@ __device__ __forceinline__ void store8(float* p, const float (&v)[8]) {
   reinterpret_cast<float4*>(p)[1] = make_float4(v[4], v[5], v[6], v[7]);
 }
 
-template <typename T>
-__global__ void __launch_bounds__(256) k_qkv_prep(PrepArgs a, int nsec, int s0, int s1, int s2) {
-  const int lane = threadIdx.x & 31;
-  const int64_t gw = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  const int64_t r = gw / nsec;
-  if (r >= a.rows) return;
-  const int k = (int)(gw % nsec);
-  const int sec = k == 0 ? s0 : (k == 1 ? s1 : s2);
-  const int seq = (int)(r / a.L), l = (int)(r % a.L);
-  const T* src = (const T*)a.src + r * a.ld + a.off[sec];
-  const int nc = a.d >> 3;
-  const float* g = a.gain[sec];
-  float rstd = 1.f;
-  if (g != nullptr) {
-    float ss = 0.f;
-    for (int c = lane; c < nc; c += 32) {
-      float v[8];
-      load8(src + 8 * c, v);
-#pragma unroll
-      for (int i = 0; i < 8; ++i) ss = fmaf(v[i], v[i], ss);
-    }
-    rstd = 1.f / sqrtf(warp_sum(ss) / (float)a.d + a.eps);
-  }
-  const bool rot = a.rope && sec < 2;
+// Rotates the 4 (even, odd) pairs of an 8-element chunk starting at head offset eh.
+__device__ __forceinline__ void rope8(float (&v)[8], int eh, const NormRopeArgs& a, int pf, int ph,
+                                      int pw) {
   const int s6 = a.hd / 6;
   const int nf = (a.hd - 4 * s6) / 2, nh = s6;  // rotated pairs per axis: frame, height (= width)
-  const int pf = l / (a.Hp * a.Wp), ph = (l / a.Wp) % a.Hp, pw = l % a.Wp;
-  T* dst = (T*)a.dst[sec];
-  for (int c = lane; c < nc; c += 32) {
-    float v[8];
-    load8(src + 8 * c, v);
-    const int e0 = 8 * c, h = e0 / a.hd, eh = e0 % a.hd;
-    if (g != nullptr) {
-      const float4 g0 = reinterpret_cast<const float4*>(g + e0)[0];
-      const float4 g1 = reinterpret_cast<const float4*>(g + e0)[1];
-      const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
 #pragma unroll
-      for (int i = 0; i < 8; ++i) v[i] = v[i] * rstd * gg[i];
-    }
-    if (rot) {
-#pragma unroll
-      for (int p = 0; p < 4; ++p) {
-        const int j = eh / 2 + p;
-        int idx;
-        if (j < nf) idx = pf * nf + j;
-        else if (j < nf + nh) idx = a.Fp * nf + ph * nh + (j - nf);
-        else idx = a.Fp * nf + a.Hp * nh + pw * nh + (j - nf - nh);
-        const float2 cs = a.rope_tab[idx];
-        const float x0 = v[2 * p], x1 = v[2 * p + 1];
-        v[2 * p] = x0 * cs.x - x1 * cs.y;
-        v[2 * p + 1] = x0 * cs.y + x1 * cs.x;
-      }
-    }
-    store8(dst + (((int64_t)seq * a.H + h) * a.L + l) * a.hd + eh, v);
+  for (int p = 0; p < 4; ++p) {
+    const int j = eh / 2 + p;
+    int idx;
+    if (j < nf) idx = pf * nf + j;
+    else if (j < nf + nh) idx = a.Fp * nf + ph * nh + (j - nf);
+    else idx = a.Fp * nf + a.Hp * nh + pw * nh + (j - nf - nh);
+    const float2 cs = a.rope_tab[idx];
+    const float x0 = v[2 * p], x1 = v[2 * p + 1];
+    v[2 * p] = x0 * cs.x - x1 * cs.y;
+    v[2 * p + 1] = x0 * cs.y + x1 * cs.x;
   }
 }
 
-// bf16 variant with the row section in registers: CPL 8-element chunks per lane,
+__device__ __forceinline__ void scale8(float (&v)[8], float rstd, const float* g) {
+  const float4 g0 = reinterpret_cast<const float4*>(g)[0];
+  const float4 g1 = reinterpret_cast<const float4*>(g)[1];
+  const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] = v[i] * rstd * gg[i];
+}
+
+// One warp per (row, section); the section is read in 8-element chunks twice (sum
+// of squares, then normalize / rotate / store in place; the second read hits L1).
+template <typename T>
+__global__ void __launch_bounds__(256) k_norm_rope(NormRopeArgs a) {
+  const int lane = threadIdx.x & 31;
+  const int64_t gw = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int64_t r = gw / a.nsec;
+  if (r >= a.rows) return;
+  const int j = (int)(gw % a.nsec);
+  const int l = (int)(r % a.L);
+  T* p = (T*)a.buf + r * a.ld + a.off0 + j * a.off_stride;
+  const float* g = a.gain0 + j * a.gain_stride;
+  const int nc = a.d >> 3;
+  float ss = 0.f;
+  for (int c = lane; c < nc; c += 32) {
+    float v[8];
+    load8(p + 8 * c, v);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) ss = fmaf(v[i], v[i], ss);
+  }
+  const float rstd = 1.f / sqrtf(warp_sum(ss) / (float)a.d + a.eps);
+  const int pf = l / (a.Hp * a.Wp), ph = (l / a.Wp) % a.Hp, pw = l % a.Wp;
+  for (int c = lane; c < nc; c += 32) {
+    float v[8];
+    load8(p + 8 * c, v);
+    scale8(v, rstd, g + 8 * c);
+    if (a.rope) rope8(v, (8 * c) % a.hd, a, pf, ph, pw);
+    store8(p + 8 * c, v);
+  }
+}
+
+// bf16 variant with the section in registers: CPL 8-element chunks per lane,
 // d = 256 * CPL; all loads are issued before the reduction.
 template <int CPL>
-__global__ void __launch_bounds__(256) k_qkv_prep_r(PrepArgs a, int nsec, int s0, int s1, int s2) {
+__global__ void __launch_bounds__(256) k_norm_rope_r(NormRopeArgs a) {
   constexpr int D = 256 * CPL;
   const int lane = threadIdx.x & 31;
   const int64_t gw = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  const int64_t r = gw / nsec;
+  const int64_t r = gw / a.nsec;
   if (r >= a.rows) return;
-  const int k = (int)(gw % nsec);
-  const int sec = k == 0 ? s0 : (k == 1 ? s1 : s2);
-  const int seq = (int)(r / a.L), l = (int)(r % a.L);
-  const bf16* src = (const bf16*)a.src + r * a.ld + a.off[sec];
+  const int j = (int)(gw % a.nsec);
+  const int l = (int)(r % a.L);
+  bf16* p = (bf16*)a.buf + r * a.ld + a.off0 + j * a.off_stride;
+  const float* g = a.gain0 + j * a.gain_stride;
   float v[CPL][8];
 #pragma unroll
-  for (int j = 0; j < CPL; ++j) load8(src + 8 * (lane + 32 * j), v[j]);
-  const float* g = a.gain[sec];
-  float rstd = 1.f;
-  if (g != nullptr) {
-    float s8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  for (int c = 0; c < CPL; ++c) load8(p + 8 * (lane + 32 * c), v[c]);
+  float s8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-    for (int j = 0; j < CPL; ++j)
+  for (int c = 0; c < CPL; ++c)
 #pragma unroll
-      for (int i = 0; i < 8; ++i) s8[i] = fmaf(v[j][i], v[j][i], s8[i]);
-    const float ss = ((s8[0] + s8[1]) + (s8[2] + s8[3])) + ((s8[4] + s8[5]) + (s8[6] + s8[7]));
-    rstd = 1.f / sqrtf(warp_sum(ss) / (float)D + a.eps);
-  }
-  const bool rot = a.rope && sec < 2;
-  const int s6 = a.hd / 6;
-  const int nf = (a.hd - 4 * s6) / 2, nh = s6;
+    for (int i = 0; i < 8; ++i) s8[i] = fmaf(v[c][i], v[c][i], s8[i]);
+  const float ss = ((s8[0] + s8[1]) + (s8[2] + s8[3])) + ((s8[4] + s8[5]) + (s8[6] + s8[7]));
+  const float rstd = 1.f / sqrtf(warp_sum(ss) / (float)D + a.eps);
   const int pf = l / (a.Hp * a.Wp), ph = (l / a.Wp) % a.Hp, pw = l % a.Wp;
-  bf16* dst = (bf16*)a.dst[sec];
 #pragma unroll
-  for (int j = 0; j < CPL; ++j) {
-    const int e0 = 8 * (lane + 32 * j), h = e0 / a.hd, eh = e0 % a.hd;
-    if (g != nullptr) {
-      const float4 g0 = reinterpret_cast<const float4*>(g + e0)[0];
-      const float4 g1 = reinterpret_cast<const float4*>(g + e0)[1];
-      const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
-#pragma unroll
-      for (int i = 0; i < 8; ++i) v[j][i] = v[j][i] * rstd * gg[i];
-    }
-    if (rot) {
-#pragma unroll
-      for (int p = 0; p < 4; ++p) {
-        const int jj = eh / 2 + p;
-        int idx;
-        if (jj < nf) idx = pf * nf + jj;
-        else if (jj < nf + nh) idx = a.Fp * nf + ph * nh + (jj - nf);
-        else idx = a.Fp * nf + a.Hp * nh + pw * nh + (jj - nf - nh);
-        const float2 cs = a.rope_tab[idx];
-        const float x0 = v[j][2 * p], x1 = v[j][2 * p + 1];
-        v[j][2 * p] = x0 * cs.x - x1 * cs.y;
-        v[j][2 * p + 1] = x0 * cs.y + x1 * cs.x;
-      }
-    }
-    store8(dst + (((int64_t)seq * a.H + h) * a.L + l) * a.hd + eh, v[j]);
+  for (int c = 0; c < CPL; ++c) {
+    const int e0 = 8 * (lane + 32 * c);
+    scale8(v[c], rstd, g + e0);
+    if (a.rope) rope8(v[c], e0 % a.hd, a, pf, ph, pw);
+    store8(p + e0, v[c]);
   }
 }
 
-cudaError_t qkv_prep(const PrepArgs& a, cudaStream_t s) {
-  int secs[3] = {0, 0, 0}, nsec = 0;
-  for (int i = 0; i < 3; ++i)
-    if (a.dst[i] != nullptr) secs[nsec++] = i;
-  if (nsec == 0 || a.rows <= 0) return cudaSuccess;
-  if (a.d % 8 || a.hd % 8) return cudaErrorInvalidValue;
-  const int64_t warps = (int64_t)a.rows * nsec;
+cudaError_t qk_norm_rope(const NormRopeArgs& a, cudaStream_t s) {
+  if (a.nsec <= 0 || a.rows <= 0) return cudaSuccess;
+  if (a.d % 8 || a.hd % 8 || a.off0 % 8 || a.off_stride % 8 || a.ld % 8 || a.gain_stride % 8)
+    return cudaErrorInvalidValue;
+  const int64_t warps = (int64_t)a.rows * a.nsec;
   const int g = (int)((warps + 7) / 8);
   if (a.dtype == BF16) {
     switch (a.d % 256 == 0 ? a.d / 256 : 0) {
-#define PREP_CASE(C) \
-  case C: k_qkv_prep_r<C><<<g, 256, 0, s>>>(a, nsec, secs[0], secs[1], secs[2]); break;
-      PREP_CASE(1) PREP_CASE(2) PREP_CASE(3) PREP_CASE(4) PREP_CASE(6) PREP_CASE(8) PREP_CASE(12)
-      PREP_CASE(16)
-#undef PREP_CASE
-      default: k_qkv_prep<bf16><<<g, 256, 0, s>>>(a, nsec, secs[0], secs[1], secs[2]);
+#define NR_CASE(C) \
+  case C: k_norm_rope_r<C><<<g, 256, 0, s>>>(a); break;
+      NR_CASE(1) NR_CASE(2) NR_CASE(3) NR_CASE(4) NR_CASE(6) NR_CASE(8) NR_CASE(12) NR_CASE(16)
+#undef NR_CASE
+      default: k_norm_rope<bf16><<<g, 256, 0, s>>>(a);
     }
   } else {
-    k_qkv_prep<float><<<g, 256, 0, s>>>(a, nsec, secs[0], secs[1], secs[2]);
+    k_norm_rope<float><<<g, 256, 0, s>>>(a);
   }
   count_launch();
   return cudaGetLastError();

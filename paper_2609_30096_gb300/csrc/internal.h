@@ -39,14 +39,25 @@ cudaError_t gemm_f32(const float* A, const float* W, const GemmArgs& g, cudaStre
 cudaError_t gemm_bf16_tc(const void* A, const void* W, const GemmArgs& g, cudaStream_t s);
 
 // ---------------------------------------------------------------- attention
-// Q [S,H,Lq,hd], K/V [S,H,Lk,hd] -> O [S,Lq,H,hd].
-cudaError_t attention_f32(const float* Q, const float* K, const float* V, float* O, int S, int H,
-                          int Lq, int Lk, int hd, cudaStream_t s);
-cudaError_t attention_bf16(const void* Q, const void* K, const void* V, void* O, int S, int H,
-                           int Lq, int Lk, int hd, cudaStream_t s);
-// tcgen05 / TMEM flash attention (attn_tc.cu); same layouts.
-cudaError_t attention_bf16_tc(const void* Q, const void* K, const void* V, void* O, int S, int H,
-                              int Lq, int Lk, int hd, cudaStream_t s);
+// One attention operand: element (s, h, l, e) of its [S, H, L, hd] view lives at
+// ptr + s*ss + h*hs + l*ls + e (strides in elements).  Head-major buffers have
+// ls = hd, hs = L*hd; token-major projection outputs [S*L, ld] with head h at
+// columns h*hd have ls = ld, hs = hd.
+struct AttnOperand {
+  const void* ptr;
+  int64_t ls, hs, ss;
+};
+inline AttnOperand head_major(const void* p, int H, int L, int hd) {
+  return {p, hd, (int64_t)L * hd, (int64_t)H * L * hd};
+}
+inline AttnOperand token_major(const void* p, int L, int ld, int hd) {
+  return {p, ld, hd, (int64_t)L * ld};
+}
+// O [S, Lq, H, hd] (token-major) = softmax(Q K^T / sqrt(hd)) V.
+cudaError_t attention_f32(const AttnOperand& Q, const AttnOperand& K, const AttnOperand& V,
+                          float* O, int S, int H, int Lq, int Lk, int hd, cudaStream_t s);
+cudaError_t attention_bf16(const AttnOperand& Q, const AttnOperand& K, const AttnOperand& V,
+                           void* O, int S, int H, int Lq, int Lk, int hd, cudaStream_t s);
 
 // ---------------------------------------------------------------- elementwise
 cudaError_t convert_f32(const float* src, void* dst, int dtype, int64_t n, cudaStream_t s);
@@ -68,20 +79,21 @@ cudaError_t patch_embed(const float* x, int B, int nseq, int C, int F, int H, in
 // out = LN(x) * (1 + scale) + shift (mode 0) or LN(x) * g + b (mode 1); out in dtype
 cudaError_t ln_modulate(const float* x, int M, int d, const float* a, const float* b, int mode,
                         float eps, void* out, int dtype, cudaStream_t s);
-// Per row of src [rows, ld]: q/k/v sections at column offsets; optional RMSNorm over d with
-// gain, optional 3D RoPE; write head-major [nseq, H, L, hd].  Row r = seq * L + l.
-struct PrepArgs {
-  const void* src; int ld; int rows; int L; int H; int hd; int d;
-  int off[3];               // column offsets of q, k, v (-1 = absent)
-  const float* gain[3];     // RMSNorm gains (nullptr = no norm)
-  void* dst[3];             // head-major outputs (nullptr = absent)
-  int rope;                 // apply 3D RoPE to q and k
-  const float2* rope_tab;   // [(Fp + Hp + Wp) * hd/2] (cos, sin); see track_api.cu
+// In place on a token-major buffer [rows, ld] (row r = token r % L of sequence
+// r / L): for each of nsec sections of d columns, section j at column
+// off0 + j*off_stride with gain gain0 + j*gain_stride: RMSNorm over the d values
+// times the gain, then (rope) the 3D rotary embedding of every head of hd.
+struct NormRopeArgs {
+  void* buf; int ld; int rows; int L; int hd; int d;
+  int nsec; int64_t off0, off_stride;
+  const float* gain0; int64_t gain_stride;
+  int rope;
+  const float2* rope_tab;   // per-axis (cos, sin) tables, see build_rope_table
   int Fp, Hp, Wp;
   float eps;
   int dtype;
 };
-cudaError_t qkv_prep(const PrepArgs& a, cudaStream_t s);
+cudaError_t qk_norm_rope(const NormRopeArgs& a, cudaStream_t s);
 // Head: LN(x)*(1+scale)+shift, . head_W^T + head_b, unpatchify into out [nseq, C, F, H, W]
 cudaError_t head_unpatchify(const float* xres, int nseq, int L, int d, const float* head_mod,
                             const void* Whead, int dtype, const float* bhead, float eps, int C,

@@ -186,10 +186,11 @@ struct Workspace {
   int cap = 0;  // capacity in sequences
   void* base = nullptr;
   float* xres = nullptr;
-  void *h = nullptr, *qkv = nullptr, *Qh = nullptr, *Kh = nullptr, *Vh = nullptr;
+  void *h = nullptr, *qkv = nullptr;
   void *attn = nullptr, *ffh = nullptr;
   float* fout = nullptr;
-  void *ctx_in = nullptr, *ctx_h = nullptr, *ctx_c = nullptr, *ckv = nullptr, *kv = nullptr;
+  // projected text and every block's cross-attention K|V, token-major [Mt, layers * 2d]
+  void *ctx_in = nullptr, *ctx_h = nullptr, *ctx_c = nullptr, *ckv = nullptr;
   float *emb = nullptr, *e_tmp = nullptr, *e = nullptr, *e0 = nullptr, *mod_all = nullptr,
         *head_mod = nullptr;
   // guided predictions of calibration (B samples each)
@@ -210,6 +211,10 @@ struct track_model {
   std::vector<void*> tensor_ptr;  // device destination of each canonical tensor
   void *pe_W, *txt_W1, *txt_W2, *tim_W1, *tim_W2, *mod_W, *head_W;
   float *pe_b, *txt_b1, *txt_b2, *tim_b1, *tim_b2, *mod_b, *mod_bias, *head_bias, *head_b;
+  // every block's cross-attention K/V projection, stacked: [layers * 2d, d], [layers * 2d];
+  // and the cross-attention key RMSNorm gains [layers, d]
+  void* Wckv_all;
+  float *bckv_all, *ckn_all;
   std::vector<track::Layer> layer;
   float2* rope_tab = nullptr;
   track::Workspace ws;
@@ -263,6 +268,9 @@ static size_t layout_weights(track_model* m, uint8_t* base) {
   m->tim_W1 = mat(d, a.freq_dim); m->tim_b1 = vec(d); m->tim_W2 = mat(d, d); m->tim_b2 = vec(d);
   m->mod_W = mat(6 * d, d); m->mod_b = vec(6 * d);
   m->mod_bias = vec((int64_t)a.layers * 6 * d);
+  m->Wckv_all = mat((int64_t)a.layers * 2 * d, d);
+  m->bckv_all = vec((int64_t)a.layers * 2 * d);
+  m->ckn_all = vec((int64_t)a.layers * d);
   m->layer.resize(a.layers);
   for (int l = 0; l < a.layers; ++l) {
     Layer& L = m->layer[l];
@@ -270,9 +278,10 @@ static size_t layout_weights(track_model* m, uint8_t* base) {
     L.Wo = mat(d, d); L.bo = vec(d);
     L.qn_g = vec(d); L.kn_g = vec(d); L.ln3_g = vec(d); L.ln3_b = vec(d);
     L.Wcq = mat(d, d); L.bcq = vec(d);
-    L.Wckv = mat(2 * d, d); L.bckv = vec(2 * d);
+    L.Wckv = (uint8_t*)m->Wckv_all + (size_t)l * 2 * d * d * es;
+    L.bckv = m->bckv_all + (int64_t)l * 2 * d;
     L.Wco = mat(d, d); L.bco = vec(d);
-    L.cqn_g = vec(d); L.ckn_g = vec(d);
+    L.cqn_g = vec(d); L.ckn_g = m->ckn_all + (int64_t)l * d;
     L.W1 = mat(F, d); L.b1 = vec(F);
     L.W2 = mat(d, F); L.b2 = vec(d);
   }
@@ -388,14 +397,13 @@ static int ensure_workspace(track_model* m, int nseq) {
   sz(M * d * 4);                       // xres
   sz(M * d * es);                      // h
   sz(M * 3 * d * es);                  // qkv
-  for (int i = 0; i < 4; ++i) sz(M * d * es);  // Qh Kh Vh attn
+  sz(M * d * es);                      // attn
   sz(M * F * es);                      // ffh
   sz((size_t)nseq * m->latent_n * 4);  // fout
   sz(Mt * Dt * es);                    // ctx_in
   sz(Mt * d * es);                     // ctx_h
   sz(Mt * d * es);                     // ctx_c
-  sz(Mt * 2 * d * es);                 // ckv
-  sz((size_t)a.layers * 2 * Mt * d * es);  // kv cache
+  sz((size_t)Mt * a.layers * 2 * d * es);  // ckv (all blocks)
   sz(256 * 4);
   sz(d * 4);
   sz(d * 4);
@@ -413,17 +421,13 @@ static int ensure_workspace(track_model* m, int nseq) {
   w.xres = (float*)dalloc_carve(p, M * d * 4);
   w.h = dalloc_carve(p, M * d * es);
   w.qkv = dalloc_carve(p, M * 3 * d * es);
-  w.Qh = dalloc_carve(p, M * d * es);
-  w.Kh = dalloc_carve(p, M * d * es);
-  w.Vh = dalloc_carve(p, M * d * es);
   w.attn = dalloc_carve(p, M * d * es);
   w.ffh = dalloc_carve(p, M * F * es);
   w.fout = (float*)dalloc_carve(p, (size_t)nseq * m->latent_n * 4);
   w.ctx_in = dalloc_carve(p, Mt * Dt * es);
   w.ctx_h = dalloc_carve(p, Mt * d * es);
   w.ctx_c = dalloc_carve(p, Mt * d * es);
-  w.ckv = dalloc_carve(p, Mt * 2 * d * es);
-  w.kv = dalloc_carve(p, (size_t)a.layers * 2 * Mt * d * es);
+  w.ckv = dalloc_carve(p, (size_t)Mt * a.layers * 2 * d * es);
   w.emb = (float*)dalloc_carve(p, 256 * 4);
   w.e_tmp = (float*)dalloc_carve(p, d * 4);
   w.e = (float*)dalloc_carve(p, d * 4);
@@ -471,29 +475,36 @@ static int run_gemm(const track_model* m, const void* A, const void* W, int M, i
   return TRACK_OK;
 }
 
-static int run_attention(const track_model* m, const void* Q, const void* K, const void* V,
-                         void* O, int S, int Lq, int Lk, cudaStream_t s) {
+static int run_attention(const track_model* m, const AttnOperand& Q, const AttnOperand& K,
+                         const AttnOperand& V, void* O, int S, int Lq, int Lk, cudaStream_t s) {
   const int H = m->a.heads, hd = m->hd;
   ProfScope ps(1, 4.0 * S * H * (double)Lq * Lk * hd, s);
-  cudaError_t e = m->dtype == BF16
-                      ? attention_bf16(Q, K, V, O, S, H, Lq, Lk, hd, s)
-                      : attention_f32((const float*)Q, (const float*)K, (const float*)V, (float*)O,
-                                      S, H, Lq, Lk, hd, s);
+  cudaError_t e = m->dtype == BF16 ? attention_bf16(Q, K, V, O, S, H, Lq, Lk, hd, s)
+                                   : attention_f32(Q, K, V, (float*)O, S, H, Lq, Lk, hd, s);
   if (e != cudaSuccess)
     return fail(TRACK_ECUDA, std::string("attention launch: ") + cudaGetErrorString(e));
   return TRACK_OK;
 }
 
-// LayerNorm-modulate and RMSNorm/RoPE/head-split launches, timed as class 2 with
+// LayerNorm-modulate and in-place RMSNorm/RoPE launches, timed as class 2 with
 // their algorithmic bytes (fp32 row in + activation row out; activation in + out).
 static cudaError_t run_ln(const track_model* m, const float* x, int M, int d, const float* a,
                           const float* b, int mode, void* out, cudaStream_t s) {
   ProfScope ps(2, (double)M * d * (4.0 + m->esz), s);
   return ln_modulate(x, M, d, a, b, mode, m->a.eps, out, m->dtype, s);
 }
-static cudaError_t run_prep(const track_model* m, const PrepArgs& p, int sections, cudaStream_t s) {
-  ProfScope ps(2, (double)p.rows * p.d * sections * 2.0 * m->esz, s);
-  return qkv_prep(p, s);
+static cudaError_t run_norm(const track_model* m, const NormRopeArgs& p, cudaStream_t s) {
+  ProfScope ps(2, (double)p.rows * p.d * p.nsec * 2.0 * m->esz, s);
+  return qk_norm_rope(p, s);
+}
+
+static NormRopeArgs norm_args(const track_model* m, void* buf, int ld, int rows, int L) {
+  NormRopeArgs p;
+  memset(&p, 0, sizeof(p));
+  p.buf = buf; p.ld = ld; p.rows = rows; p.L = L; p.hd = m->hd; p.d = m->a.dim;
+  p.rope_tab = m->rope_tab; p.Fp = m->Fp; p.Hp = m->Hp; p.Wp = m->Wp;
+  p.eps = m->a.eps; p.dtype = m->dtype;
+  return p;
 }
 
 #define LAUNCH(expr)                                                                  \
@@ -519,23 +530,15 @@ static int project_context(track_model* m, const float* cond, const float* uncon
                      w.ctx_h, (int)d, s));
   TRACK_TRY(run_gemm(m, w.ctx_h, m->txt_W2, Mt, (int)d, (int)d, m->txt_b2, EPI_STORE, nullptr,
                      w.ctx_c, (int)d, s));
-  for (int l = 0; l < a.layers; ++l) {
-    const Layer& L = m->layer[l];
-    TRACK_TRY(run_gemm(m, w.ctx_c, L.Wckv, Mt, (int)(2 * d), (int)d, L.bckv, EPI_STORE, nullptr,
-                       w.ckv, (int)(2 * d), s));
-    uint8_t* kv = (uint8_t*)w.kv + (size_t)l * 2 * Mt * d * m->esz;
-    PrepArgs p;
-    memset(&p, 0, sizeof(p));
-    p.src = w.ckv; p.ld = (int)(2 * d); p.rows = Mt; p.L = (int)Lt; p.H = a.heads; p.hd = m->hd;
-    p.d = (int)d;
-    p.off[0] = -1; p.off[1] = 0; p.off[2] = (int)d;
-    p.gain[1] = L.ckn_g;
-    p.dst[1] = kv;
-    p.dst[2] = kv + (size_t)Mt * d * m->esz;
-    p.rope = 0; p.eps = a.eps; p.dtype = m->dtype;
-    p.Fp = m->Fp; p.Hp = m->Hp; p.Wp = m->Wp; p.rope_tab = m->rope_tab;
-    LAUNCH(qkv_prep(p, s));
-  }
+  // every block's cross-attention K|V in one GEMM, then RMSNorm of every block's K in place
+  const int nkv = a.layers * 2 * (int)d;
+  TRACK_TRY(run_gemm(m, w.ctx_c, m->Wckv_all, Mt, nkv, (int)d, m->bckv_all, EPI_STORE, nullptr,
+                     w.ckv, nkv, s));
+  NormRopeArgs p = norm_args(m, w.ckv, nkv, Mt, (int)Lt);
+  p.nsec = a.layers; p.off0 = 0; p.off_stride = 2 * d;
+  p.gain0 = m->ckn_all; p.gain_stride = d;
+  p.rope = 0;
+  LAUNCH(run_norm(m, p, s));
   m->c_cond = cond;
   m->c_uncond = uncond;
   m->c_nseq = nseq;
@@ -564,11 +567,7 @@ static int forward(track_model* m, const float* x, int B, int nseq, float t, con
   LAUNCH(patch_embed(x, B, nseq, a.in_ch, a.frames, a.height, a.width, m->pe_W, m->dtype, m->pe_b,
                      d, w.xres, s));
 
-  PrepArgs ps;
-  memset(&ps, 0, sizeof(ps));
-  ps.rows = M; ps.L = L; ps.H = H; ps.hd = m->hd; ps.d = d; ps.eps = a.eps; ps.dtype = m->dtype;
-  ps.Fp = m->Fp; ps.Hp = m->Hp; ps.Wp = m->Wp; ps.rope_tab = m->rope_tab;
-  const int Mt = nseq * a.text_len;
+  const int nkv = a.layers * 2 * d;
 
   for (int l = 0; l < a.layers; ++l) {
     const Layer& Ly = m->layer[l];
@@ -578,25 +577,34 @@ static int forward(track_model* m, const float* x, int B, int nseq, float t, con
     // self-attention
     LAUNCH(run_ln(m, w.xres, M, d, scale1, shift1, 0, w.h, s));
     TRACK_TRY(run_gemm(m, w.h, Ly.Wqkv, M, 3 * d, d, Ly.bqkv, EPI_STORE, nullptr, w.qkv, 3 * d, s));
-    ps.src = w.qkv; ps.ld = 3 * d;
-    ps.off[0] = 0; ps.off[1] = d; ps.off[2] = 2 * d;
-    ps.gain[0] = Ly.qn_g; ps.gain[1] = Ly.kn_g; ps.gain[2] = nullptr;
-    ps.dst[0] = w.Qh; ps.dst[1] = w.Kh; ps.dst[2] = w.Vh;
-    ps.rope = 1;
-    LAUNCH(run_prep(m, ps, 3, s));
-    TRACK_TRY(run_attention(m, w.Qh, w.Kh, w.Vh, w.attn, nseq, L, L, s));
+    {  // q and k: RMSNorm over d and 3D RoPE, in place; v is used as projected
+      NormRopeArgs p = norm_args(m, w.qkv, 3 * d, M, L);
+      p.nsec = 2; p.off0 = 0; p.off_stride = d;
+      p.gain0 = Ly.qn_g; p.gain_stride = Ly.kn_g - Ly.qn_g;
+      p.rope = 1;
+      LAUNCH(run_norm(m, p, s));
+    }
+    const uint8_t* qkv = (const uint8_t*)w.qkv;
+    TRACK_TRY(run_attention(m, token_major(qkv, L, 3 * d, m->hd),
+                            token_major(qkv + (size_t)d * es, L, 3 * d, m->hd),
+                            token_major(qkv + (size_t)2 * d * es, L, 3 * d, m->hd), w.attn, nseq, L,
+                            L, s));
     TRACK_TRY(run_gemm(m, w.attn, Ly.Wo, M, d, d, Ly.bo, EPI_RESID_GATE, gate1, w.xres, d, s));
     // cross-attention
     LAUNCH(run_ln(m, w.xres, M, d, Ly.ln3_g, Ly.ln3_b, 1, w.h, s));
     TRACK_TRY(run_gemm(m, w.h, Ly.Wcq, M, d, d, Ly.bcq, EPI_STORE, nullptr, w.qkv, d, s));
-    ps.src = w.qkv; ps.ld = d;
-    ps.off[0] = 0; ps.off[1] = -1; ps.off[2] = -1;
-    ps.gain[0] = Ly.cqn_g; ps.gain[1] = nullptr;
-    ps.dst[0] = w.Qh; ps.dst[1] = nullptr; ps.dst[2] = nullptr;
-    ps.rope = 0;
-    LAUNCH(run_prep(m, ps, 1, s));
-    const uint8_t* kv = (const uint8_t*)w.kv + (size_t)l * 2 * Mt * d * es;
-    TRACK_TRY(run_attention(m, w.Qh, kv, kv + (size_t)Mt * d * es, w.attn, nseq, L, a.text_len, s));
+    {  // cross-attention q: RMSNorm over d, in place
+      NormRopeArgs p = norm_args(m, w.qkv, d, M, L);
+      p.nsec = 1; p.off0 = 0; p.off_stride = 0;
+      p.gain0 = Ly.cqn_g; p.gain_stride = 0;
+      p.rope = 0;
+      LAUNCH(run_norm(m, p, s));
+    }
+    const uint8_t* kvl = (const uint8_t*)w.ckv + (size_t)l * 2 * d * es;
+    TRACK_TRY(run_attention(m, token_major(w.qkv, L, d, m->hd),
+                            token_major(kvl, a.text_len, nkv, m->hd),
+                            token_major(kvl + (size_t)d * es, a.text_len, nkv, m->hd), w.attn, nseq,
+                            L, a.text_len, s));
     TRACK_TRY(run_gemm(m, w.attn, Ly.Wco, M, d, d, Ly.bco, EPI_RESID, nullptr, w.xres, d, s));
     // MLP
     LAUNCH(run_ln(m, w.xres, M, d, scale2, shift2, 0, w.h, s));
@@ -1036,10 +1044,11 @@ int track_attention(int dtype, const void* Q, const void* K, const void* V, int 
   if (!Q || !K || !V || !O || S < 0 || H <= 0 || Lq < 0 || Lk <= 0)
     return fail(TRACK_EINVAL, "bad arguments");
   if (hd != 64 && hd != 128) return fail(TRACK_EINVAL, "hd must be 64 or 128");
+  const AttnOperand q = head_major(Q, H, Lq, hd), k = head_major(K, H, Lk, hd),
+                    v = head_major(V, H, Lk, hd);
   cudaError_t e = dtype == TRACK_BF16
-                      ? attention_bf16(Q, K, V, O, S, H, Lq, Lk, hd, (cudaStream_t)s)
-                      : attention_f32((const float*)Q, (const float*)K, (const float*)V, (float*)O,
-                                      S, H, Lq, Lk, hd, (cudaStream_t)s);
+                      ? attention_bf16(q, k, v, O, S, H, Lq, Lk, hd, (cudaStream_t)s)
+                      : attention_f32(q, k, v, (float*)O, S, H, Lq, Lk, hd, (cudaStream_t)s);
   if (e != cudaSuccess) return fail(TRACK_ECUDA, std::string("attention: ") + cudaGetErrorString(e));
   return TRACK_OK;
 }
