@@ -346,9 +346,11 @@ cudaError_t gemm_bf16_tc(const void* A, const void* W, const GemmArgs& g, cudaSt
   // columns' worth) is fitted to measured tile times: a 192-wide tile takes about
   // 0.85x the time of a 256-wide one.  Ties go to the wider tile.
   const int m_tiles = (g.M + BM - 1) / BM, sms = num_sms();
+  const bool fp32_out = g.epi == EPI_RESID || g.epi == EPI_RESID_GATE;  // 32-column epilogue chunks
   int best_bn = 256;
   long best_cost = -1;
-  for (int bn : {256, 192, 128}) {
+  for (int bn : {256, 192, 160, 128}) {
+    if (bn == 160 && !fp32_out) continue;  // bf16 epilogue chunks are 64 columns wide
     const long tiles = (long)m_tiles * ((g.N + bn - 1) / bn);
     const long cost = ((tiles + sms - 1) / sms) * (bn + 150);
     if (best_cost < 0 || cost < best_cost) {
@@ -358,6 +360,7 @@ cudaError_t gemm_bf16_tc(const void* A, const void* W, const GemmArgs& g, cudaSt
   }
   if (best_bn == 256) return launch_tc<256, 4>(A, W, g, s);
   if (best_bn == 192) return launch_tc<192, 4>(A, W, g, s);
+  if (best_bn == 160) return launch_tc<160, 5>(A, W, g, s);
   return launch_tc<128, 6>(A, W, g, s);
 }
 
