@@ -82,6 +82,73 @@ def text_flops(arch, batch):
     return batch * (2 * Lt * Dt * d + 2 * Lt * d * d + l * 2 * Lt * d * 2 * d)
 
 
+# ---------------------------------------------------------------- ranks (replicas)
+def rank_env():
+    """(rank, local_rank, world) from the torchrun environment (1 process if absent)."""
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0")),
+            int(os.environ.get("WORLD_SIZE", "1")))
+
+
+def rank_first_sample(rank, batch):
+    """First evaluation sample of a rank: ranks serve disjoint requests (weak scaling)."""
+    return rank * batch
+
+
+def max_over_ranks(ms, world, device=None):
+    """Slowest rank's time (the job's time); a barrier brackets the reduction."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as tdist
+    t = torch.tensor([float(ms)], device=device)
+    tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+    tdist.barrier()
+    return float(t.item())
+
+
+def job_throughput(world, steps_per_trajectory, batch, trajectories, ms):
+    """Routed denoise steps per second of the whole job: every rank ran `trajectories`."""
+    return world * steps_per_trajectory * batch * trajectories / (ms / 1e3)
+
+
+def gpu_uuid(index):
+    """NVML/nvidia-smi identifier of CUDA device `index` ("GPU-<uuid>"), or None."""
+    try:
+        import torch
+        return "GPU-" + str(torch.cuda.get_device_properties(index).uuid)
+    except Exception:  # noqa: BLE001
+        return None
+
+
+class EnergyMeter:
+    """Reads the GPU's total-energy counter (NVML, millijoules since driver load)."""
+
+    def __init__(self, index):
+        import ctypes
+        self.h = None
+        try:
+            self.lib = ctypes.CDLL("libnvidia-ml.so.1")
+            if self.lib.nvmlInit_v2() != 0:
+                return
+            h = ctypes.c_void_p()
+            uuid = gpu_uuid(index)
+            rc = (self.lib.nvmlDeviceGetHandleByUUID(uuid.encode(), ctypes.byref(h)) if uuid
+                  else self.lib.nvmlDeviceGetHandleByIndex_v2(index, ctypes.byref(h)))
+            if rc == 0:
+                self.h = h
+        except OSError:
+            pass
+
+    def read_mj(self):
+        import ctypes
+        if self.h is None:
+            return None
+        v = ctypes.c_ulonglong()
+        if self.lib.nvmlDeviceGetTotalEnergyConsumption(self.h, ctypes.byref(v)) != 0:
+            return None
+        return int(v.value)
+
+
 class ClockSampler:
     """Samples SM clocks and throttle reasons with nvidia-smi while running."""
 
@@ -99,7 +166,8 @@ class ClockSampler:
         os.close(fd)
         try:
             self.proc = subprocess.Popen(
-                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                ["nvidia-smi", "-i", gpu_uuid(self.index) or str(self.index),
+                 f"--query-gpu={self.FIELDS}",
                  "--format=csv,noheader,nounits", "-lms", "100"],
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except Exception:
@@ -188,9 +256,9 @@ def cpu_threads():
 
 # ---------------------------------------------------------------- reference arm
 def run_reference(args):
-    rank = int(os.environ.get("RANK", "0"))
+    rank, _, _ = rank_env()
     if rank != 0:
-        return 0
+        return 0  # the oracle baseline runs once, on rank 0
     wl = synth.WORKLOADS[WORKLOAD]
     sampler = OracleSample(wl)
     for _ in range(args.warmup):
@@ -221,9 +289,7 @@ def run_ours(args):
     import paper_2609_30096_gb300 as T
     from paper_2609_30096_gb300 import _build
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    rank, local, world = rank_env()
     torch.cuda.set_device(local)
     if world > 1:
         tdist.init_process_group("nccl")
@@ -255,7 +321,7 @@ def run_ours(args):
     del xcd, ccd, ucd, r
 
     # --- request inputs: per-rank disjoint evaluation seeds
-    x0, c0, u0 = synth.evaluation_inputs(wl.large, rank * B, B, uses_uncond)
+    x0, c0, u0 = synth.evaluation_inputs(wl.large, rank_first_sample(rank, B), B, uses_uncond)
     xh = torch.from_numpy(x0).pin_memory()
     ch = torch.from_numpy(c0).pin_memory()
     uh = torch.from_numpy(u0).pin_memory() if uses_uncond else None
@@ -298,21 +364,18 @@ def run_ours(args):
         T.track_sync()
         ms = a.elapsed_time(b)
         launches = T.track_launch_count() - n0
-        if world > 1:
-            t = torch.tensor([ms], device=dev)
-            tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
-            if world > 1:
-                tdist.barrier()
-            ms = float(t.item())
-        return ms, launches
+        return max_over_ranks(ms, world, dev), launches
 
     for _ in range(args.warmup):
         step_device(policy)
     torch.cuda.synchronize()
     T.track_profile_read()                         # drop any stale records
 
+    energy = EnergyMeter(local)
     with ClockSampler(local) as clk:
+        e0 = energy.read_mj()
         ms, launches = timed(step_device, policy, args.steps)
+        e1 = energy.read_mj()
     clocks = clk.summary()
     # Same steps again with every GEMM / attention launch bracketed by CUDA events on its
     # stream (the events cost a few percent, so `value` comes from the pass above).
@@ -322,14 +385,40 @@ def run_ours(args):
     all_l = np.zeros(wl.steps, np.uint8)
     for _ in range(max(1, args.warmup // 2)):
         step_device(all_l)
+    e2 = energy.read_mj()
     ms_all_large, _ = timed(step_device, all_l, args.steps)
+    e3 = energy.read_mj()
+    joules = None
+    if None not in (e0, e1, e2, e3):
+        jr, ja = (e1 - e0) / 1e3 / args.steps, (e3 - e2) / 1e3 / args.steps
+        joules = {"routed_j_per_trajectory": jr, "all_large_j_per_trajectory": ja,
+                  "savings": 1.0 - jr / ja if ja > 0 else None,
+                  "source": "NVML total energy counter around the timed passes"}
+
+    # Cost model of Eq. 3 (total ~ sum_i C_pi(i)): latency against the switching budget K,
+    # and the equal-budget policies of the paper's ablation at the workload's K.
+    nsw = max(3, args.steps // 2)
+    sweep = []
+    for kk in range(wl.steps + 1):
+        pol = T.track_policy_topk(q, kk)
+        step_device(pol)
+        t, _ = timed(step_device, pol, nsw)
+        sweep.append({"K": kk, "ms": t / nsw, "policy": "".join("S" if p else "L" for p in pol)})
+    c_l, c_s = sweep[0]["ms"] / wl.steps, sweep[-1]["ms"] / wl.steps
+    cost_err = max(abs(r["ms"] - ((wl.steps - r["K"]) * c_l + r["K"] * c_s)) / r["ms"] for r in sweep)
+    equal_budget = {}
+    for name, pol in (("top_k", policy), ("first_k", T.track_policy_first_k(wl.steps, wl.k)),
+                      ("last_k", T.track_policy_last_k(wl.steps, wl.k)),
+                      ("random_k", T.track_policy_random_k(wl.steps, wl.k, synth.SEED_EVAL))):
+        t, _ = timed(step_device, pol, nsw)
+        equal_budget[name] = {"ms": t / nsw, "policy": "".join("S" if p else "L" for p in pol)}
     for _ in range(max(1, args.warmup // 2)):
         step_e2e(policy)
     ms_e2e, _ = timed(step_e2e, policy, args.steps)
 
     per_step_ms = ms / args.steps
-    value = world * wl.steps * B * args.steps / (ms / 1e3)
-    e2e_value = world * wl.steps * B * args.steps / (ms_e2e / 1e3)
+    value = job_throughput(world, wl.steps, B, args.steps, ms)
+    e2e_value = job_throughput(world, wl.steps, B, args.steps, ms_e2e)
     n_small = int(policy.sum())
     n_large = wl.steps - n_small
     guided = 1 if w == 1.0 else 2
@@ -391,6 +480,10 @@ def run_ours(args):
                                               forward_flops(wl.small, 1) / forward_flops(wl.large, 1)),
             "dit_tflops": tflops, "dit_frac_of_bf16_peak": tflops / peak,
             "calibration_ms": calib_ms, "calibration_seeds": wl.calib_seeds,
+            "energy": joules,
+            "latency_vs_k": sweep,
+            "cost_model": {"C_large_ms": c_l, "C_small_ms": c_s, "max_rel_err": cost_err},
+            "equal_budget_K": wl.k, "equal_budget": equal_budget,
             "score_map": [float(v) for v in q],
             "roofline": roof,
             "cpu_baseline": cpu,

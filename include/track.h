@@ -207,6 +207,17 @@ int track_mean_score(const float* r, int M, int N, float* q_out);
  * NaN or negative.  Host only, bit-exact. */
 int track_policy_topk(const float* score_map, int N, int K, uint8_t* policy_out);
 
+/* Equal-budget baseline policies of the paper's ablation (Sec. 4.5, Table 2):
+ * each routes exactly K of the N steps to the small model (policy_out[k] = 1).
+ * First-K: steps 0..K-1.  Last-K: steps N-K..N-1.  Random-K: a uniformly random
+ * K-subset by a partial Fisher-Yates shuffle of 0..N-1, whose i-th swap partner
+ * is i + (u_i mod (N - i)), u_i the i-th output of the SplitMix64 stream started
+ * at state mix64(seed) (u_i = mix64(state + (i + 1) * 0x9E3779B97F4A7C15)).
+ * EINVAL if N < 1 or K outside [0, N].  Host only, bit-exact. */
+int track_policy_first_k(int N, int K, uint8_t* policy_out);
+int track_policy_last_k(int N, int K, uint8_t* policy_out);
+int track_policy_random_k(int N, int K, uint64_t seed, uint8_t* policy_out);
+
 /* ---- loops (Sec. 3.2.1 calibration, Eq. 3 routed sampling) ---------------- */
 
 /* Reference-trajectory calibration for B samples: for k in 0..n_steps-1,

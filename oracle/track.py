@@ -159,6 +159,34 @@ def last_k_policy(n: int, k: int) -> np.ndarray:
     return pol
 
 
+def random_k_policy(n: int, k: int, seed: int) -> np.ndarray:
+    """Equal-budget baseline Random-K (Sec. 4.5, Table 2): a uniformly random K-subset.
+
+    The random numbers are an input of the method: partial Fisher-Yates shuffle of
+    0..n-1 whose i-th swap partner is i + (u_i mod (n - i)), u_i being output i of
+    a SplitMix64 stream (Steele, Lea and Flood 2014) started at mix64(seed).
+    """
+    if not (0 <= k <= n):
+        raise ValueError("K must satisfy 0 <= K <= N")
+    mask = (1 << 64) - 1
+
+    def mix64(z):
+        z &= mask
+        z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & mask
+        z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & mask
+        return z ^ (z >> 31)
+
+    state = mix64(seed)
+    perm = list(range(n))
+    for i in range(k):
+        u = mix64(state + (i + 1) * 0x9E3779B97F4A7C15)
+        j = i + u % (n - i)
+        perm[i], perm[j] = perm[j], perm[i]
+    pol = np.zeros(n, dtype=np.uint8)
+    pol[perm[:k]] = 1
+    return pol
+
+
 # ---------------------------------------------------------------------------
 # Denoiser evaluation, calibration (Sec. 3.2.1) and routed sampling (Eq. 3)
 # ---------------------------------------------------------------------------

@@ -74,6 +74,9 @@ def lib():
         "track_disagreement_static": (_I, [_P, _P, _I, _L, _F, _P, _P]),
         "track_mean_score": (_I, [_P, _I, _I, _P]),
         "track_policy_topk": (_I, [_P, _I, _I, _P]),
+        "track_policy_first_k": (_I, [_I, _I, _P]),
+        "track_policy_last_k": (_I, [_I, _I, _P]),
+        "track_policy_random_k": (_I, [_I, _I, ctypes.c_uint64, _P]),
         "track_calibrate": (_I, [_P, _P, _P, _I, _P, _P, _F, _P, _I, _F, _P, _P]),
         "track_sample": (_I, [_P, _P, _P, _P, _I, _P, _I, _P, _P, _F, _P]),
         "track_linear": (_I, [_I, _P, _P, _P, _I, _I, _I, _I, _P, _P, _I, _P]),
@@ -302,6 +305,24 @@ def track_policy_topk(score_map, K: int) -> np.ndarray:
     q = np.ascontiguousarray(score_map, dtype=np.float32)
     out = np.zeros(q.shape[0], dtype=np.uint8)
     _check(lib().track_policy_topk(q.ctypes.data, q.shape[0], K, out.ctypes.data))
+    return out
+
+
+def track_policy_first_k(N: int, K: int) -> np.ndarray:
+    out = np.zeros(N, dtype=np.uint8)
+    _check(lib().track_policy_first_k(N, K, out.ctypes.data))
+    return out
+
+
+def track_policy_last_k(N: int, K: int) -> np.ndarray:
+    out = np.zeros(N, dtype=np.uint8)
+    _check(lib().track_policy_last_k(N, K, out.ctypes.data))
+    return out
+
+
+def track_policy_random_k(N: int, K: int, seed: int) -> np.ndarray:
+    out = np.zeros(N, dtype=np.uint8)
+    _check(lib().track_policy_random_k(N, K, seed, out.ctypes.data))
     return out
 
 

@@ -698,6 +698,13 @@ static int disagreement_impl(const float* vL, const float* vS, int B, int64_t n,
 // ====================================================================== C ABI
 using namespace track;
 
+// SplitMix64 output mixing (Steele, Lea and Flood 2014), host side.
+static uint64_t mix64_host(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
 extern "C" {
 
 const char* track_last_error(void) { return g_last_error.c_str(); }
@@ -849,11 +856,6 @@ int track_model_create(const track_arch* arch, const float* const* weights, trac
   return TRACK_OK;
 }
 
-static uint64_t mix64_host(uint64_t z) {
-  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
-  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
-  return z ^ (z >> 31);
-}
 
 int track_model_create_seeded(const track_arch* arch, uint32_t seed, track_model** out) {
   track_model* m = nullptr;
@@ -976,6 +978,33 @@ int track_policy_topk(const float* score_map, int N, int K, uint8_t* policy_out)
                    [&](int a, int b) { return score_map[a] < score_map[b]; });
   for (int i = 0; i < N; ++i) policy_out[i] = 0;
   for (int i = 0; i < K; ++i) policy_out[idx[i]] = 1;
+  return TRACK_OK;
+}
+
+int track_policy_first_k(int N, int K, uint8_t* policy_out) {
+  if (!policy_out || N < 1 || K < 0 || K > N) return fail(TRACK_EINVAL, "bad arguments");
+  for (int i = 0; i < N; ++i) policy_out[i] = i < K ? 1 : 0;
+  return TRACK_OK;
+}
+
+int track_policy_last_k(int N, int K, uint8_t* policy_out) {
+  if (!policy_out || N < 1 || K < 0 || K > N) return fail(TRACK_EINVAL, "bad arguments");
+  for (int i = 0; i < N; ++i) policy_out[i] = i >= N - K ? 1 : 0;
+  return TRACK_OK;
+}
+
+int track_policy_random_k(int N, int K, uint64_t seed, uint8_t* policy_out) {
+  if (!policy_out || N < 1 || K < 0 || K > N) return fail(TRACK_EINVAL, "bad arguments");
+  std::vector<int> perm(N);
+  for (int i = 0; i < N; ++i) perm[i] = i;
+  const uint64_t state = mix64_host(seed);
+  for (int i = 0; i < K; ++i) {
+    const uint64_t u = mix64_host(state + (uint64_t)(i + 1) * 0x9E3779B97F4A7C15ull);
+    const int j = i + (int)(u % (uint64_t)(N - i));
+    std::swap(perm[i], perm[j]);
+  }
+  for (int i = 0; i < N; ++i) policy_out[i] = 0;
+  for (int i = 0; i < K; ++i) policy_out[perm[i]] = 1;
   return TRACK_OK;
 }
 

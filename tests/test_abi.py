@@ -90,3 +90,15 @@ def test_arch_validation(T):
         T.track_weight_count(bad)
     with pytest.raises(T.TrackError):
         T.track_weight_shape(a, 10 ** 6)
+
+
+def test_equal_budget_policies_bit_exact(T):
+    for n in (1, 4, 13, 50):
+        for k in sorted({0, 1, n // 2, n}):
+            assert np.array_equal(T.track_policy_first_k(n, k), otrack.first_k_policy(n, k))
+            assert np.array_equal(T.track_policy_last_k(n, k), otrack.last_k_policy(n, k))
+            for seed in (0, 7, 2 ** 40 + 3):
+                assert np.array_equal(T.track_policy_random_k(n, k, seed),
+                                      otrack.random_k_policy(n, k, seed))
+    with pytest.raises(T.TrackError):
+        T.track_policy_random_k(4, 5, 1)

@@ -250,3 +250,19 @@ def test_mutation_flipped_disagreement_ratio_is_caught():
     pl = np.ones(4)
     assert track.disagreement(pl, np.zeros(4)) == pytest.approx(1.0)
     assert wrong(pl, np.zeros(4)) != pytest.approx(1.0)
+
+
+def test_equal_budget_policies():
+    for n in (1, 4, 7, 50):
+        for k in range(n + 1):
+            f, l = track.first_k_policy(n, k), track.last_k_policy(n, k)
+            assert f.sum() == k and l.sum() == k
+            assert np.all(f[:k] == 1) and np.all(l[n - k:] == 1)
+            r = track.random_k_policy(n, k, seed=123)
+            assert r.sum() == k and set(np.unique(r)) <= {0, 1}
+    # every step is chosen with probability K/N (uniform subsets)
+    n, k = 10, 3
+    counts = np.zeros(n)
+    for seed in range(4000):
+        counts += track.random_k_policy(n, k, seed)
+    assert np.allclose(counts / 4000, k / n, atol=0.03)
