@@ -24,6 +24,8 @@ template <int HD>
 __global__ void __launch_bounds__(128) k_attn_f32(AttnOperand Qo, AttnOperand Ko, AttnOperand Vo,
                                                   float* __restrict__ O, int H, int Lq, int Lk,
                                                   float scale) {
+  pdl_wait();
+  pdl_release();
   constexpr int DV = HD / 32;
   __shared__ float sK[F32_KT][HD + 1];
   __shared__ float sV[F32_KT][HD + 1];
@@ -99,11 +101,10 @@ cudaError_t attention_f32(const AttnOperand& Q, const AttnOperand& K, const Attn
   if (Lk <= 0) return cudaErrorInvalidValue;
   dim3 grid((Lq + 4 * F32_ROWS - 1) / (4 * F32_ROWS), S * H);
   const float scale = (float)(1.0 / sqrt((double)hd));
-  if (hd == 128) k_attn_f32<128><<<grid, 128, 0, s>>>(Q, K, V, O, H, Lq, Lk, scale);
-  else if (hd == 64) k_attn_f32<64><<<grid, 128, 0, s>>>(Q, K, V, O, H, Lq, Lk, scale);
-  else return cudaErrorInvalidValue;
   count_launch();
-  return cudaGetLastError();
+  if (hd == 128) return launch_pdl(k_attn_f32<128>, grid, 128, 0, s, Q, K, V, O, H, Lq, Lk, scale);
+  if (hd == 64) return launch_pdl(k_attn_f32<64>, grid, 128, 0, s, Q, K, V, O, H, Lq, Lk, scale);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace track

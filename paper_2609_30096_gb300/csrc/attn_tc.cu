@@ -126,6 +126,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // The prologue above overlaps the previous kernel; inputs and outputs are touched only now.
+  pdl_wait();
+  pdl_release();
 
   if (warp == 0) {
     // lane 0 streams Q and the K tiles, lane 1 the V tiles, each through its own ring
@@ -390,10 +393,9 @@ cudaError_t launch_attn_tc(const AttnOperand& Q, const AttnOperand& K, const Att
                                        (int)S1::SMEM);
   if (e != cudaSuccess) return e;
   dim3 grid((Lq + AT_BM - 1) / AT_BM, S_ * H);
-  k_attn_tc<HD><<<grid, AT_THREADS, S1::SMEM, s>>>(tq, tk, tv, (bf16*)O, H, Lq, Lk, scale_log2,
-                                                   q_tok, k_tok, err);
   count_launch();
-  return cudaGetLastError();
+  return launch_pdl(k_attn_tc<HD>, grid, AT_THREADS, S1::SMEM, s, tq, tk, tv, (bf16*)O, H, Lq, Lk,
+                    scale_log2, q_tok, k_tok, err);
 }
 
 }  // namespace

@@ -38,6 +38,8 @@ __device__ float block_sum(float v, float* red) {
 // ---------------------------------------------------------------- weights
 template <typename T>
 __global__ void k_convert(const float* __restrict__ src, T* __restrict__ dst, int64_t n) {
+  pdl_wait();
+  pdl_release();
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x)
     stv(dst, i, src[i]);
@@ -46,8 +48,9 @@ __global__ void k_convert(const float* __restrict__ src, T* __restrict__ dst, in
 cudaError_t convert_f32(const float* src, void* dst, int dtype, int64_t n, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int g = grid_for(n, 256);
-  if (dtype == BF16) k_convert<bf16><<<g, 256, 0, s>>>(src, (bf16*)dst, n);
-  else k_convert<float><<<g, 256, 0, s>>>(src, (float*)dst, n);
+  cudaError_t e = dtype == BF16 ? launch_pdl(k_convert<bf16>, g, 256, 0, s, src, (bf16*)dst, n)
+                                : launch_pdl(k_convert<float>, g, 256, 0, s, src, (float*)dst, n);
+  if (e != cudaSuccess) return e;
   count_launch();
   return cudaGetLastError();
 }
@@ -87,6 +90,8 @@ cudaError_t seed_fill(void* dst, int dtype, uint64_t state, int64_t n, float sca
 
 // ---------------------------------------------------------------- timestep embedding
 __global__ void k_sinusoid(float t, float* emb, int dim) {
+  pdl_wait();
+  pdl_release();
   const int half = dim / 2;
   for (int i = threadIdx.x; i < dim; i += blockDim.x) {
     const int j = i < half ? i : i - half;
@@ -96,7 +101,8 @@ __global__ void k_sinusoid(float t, float* emb, int dim) {
 }
 
 cudaError_t sinusoid(float t, float* emb, int freq_dim, cudaStream_t s) {
-  k_sinusoid<<<1, 256, 0, s>>>(t, emb, freq_dim);
+  cudaError_t e = launch_pdl(k_sinusoid, 1, 256, 0, s, t, emb, freq_dim);
+  if (e != cudaSuccess) return e;
   count_launch();
   return cudaGetLastError();
 }
@@ -106,6 +112,8 @@ template <typename T>
 __global__ void k_matvec(const T* __restrict__ W, const float* __restrict__ in,
                          const float* __restrict__ b, float* __restrict__ out, int rows, int cols,
                          int silu_in) {
+  pdl_wait();
+  pdl_release();
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (row >= rows) return;
   float acc = 0.f;
@@ -122,8 +130,10 @@ __global__ void k_matvec(const T* __restrict__ W, const float* __restrict__ in,
 cudaError_t matvec(const void* W, int dtype, const float* in, const float* b, float* out, int rows,
                    int cols, int silu_in, cudaStream_t s) {
   const int g = (rows * 32 + 255) / 256;
-  if (dtype == BF16) k_matvec<bf16><<<g, 256, 0, s>>>((const bf16*)W, in, b, out, rows, cols, silu_in);
-  else k_matvec<float><<<g, 256, 0, s>>>((const float*)W, in, b, out, rows, cols, silu_in);
+  cudaError_t e = dtype == BF16
+      ? launch_pdl(k_matvec<bf16>, g, 256, 0, s, (const bf16*)W, in, b, out, rows, cols, silu_in)
+      : launch_pdl(k_matvec<float>, g, 256, 0, s, (const float*)W, in, b, out, rows, cols, silu_in);
+  if (e != cudaSuccess) return e;
   count_launch();
   return cudaGetLastError();
 }
@@ -132,6 +142,8 @@ __global__ void k_modulation(const float* __restrict__ e0, const float* __restri
                              int layers, const float* __restrict__ e,
                              const float* __restrict__ head_bias, int d, float* __restrict__ mod_all,
                              float* __restrict__ head_mod) {
+  pdl_wait();
+  pdl_release();
   const int64_t n1 = (int64_t)layers * 6 * d;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n1 + 2 * d;
        i += (int64_t)gridDim.x * blockDim.x) {
@@ -147,8 +159,9 @@ cudaError_t modulation(const float* e0, const float* mod_bias, int layers, const
                        const float* head_bias, int d, float* mod_all, float* head_mod,
                        cudaStream_t s) {
   const int64_t n = (int64_t)layers * 6 * d + 2 * d;
-  k_modulation<<<grid_for(n, 256), 256, 0, s>>>(e0, mod_bias, layers, e, head_bias, d, mod_all,
-                                                head_mod);
+  cudaError_t err = launch_pdl(k_modulation, grid_for(n, 256), 256, 0, s, e0, mod_bias, layers, e,
+                               head_bias, d, mod_all, head_mod);
+  if (err != cudaSuccess) return err;
   count_launch();
   return cudaGetLastError();
 }
@@ -163,6 +176,8 @@ __global__ void __launch_bounds__(256) k_patch_embed(const float* __restrict__ x
                                                      const T* __restrict__ Wpe,
                                                      const float* __restrict__ bpe, int d,
                                                      float* __restrict__ xres) {
+  pdl_wait();
+  pdl_release();
   __shared__ float patch[PE_TOK][64];
   const int Hp = H / 2, Wp = W / 2, L = F * Hp * Wp;
   const int r0 = blockIdx.x * PE_TOK;
@@ -200,12 +215,12 @@ cudaError_t patch_embed(const float* x, int B, int nseq, int C, int F, int H, in
                         int dtype, const float* bpe, int d, float* xres, cudaStream_t s) {
   const int rows = nseq * F * (H / 2) * (W / 2);
   const int g = (rows + PE_TOK - 1) / PE_TOK;
-  if (dtype == BF16)
-    k_patch_embed<bf16><<<g, 256, 0, s>>>(x, B, rows, C, F, H, W, (const bf16*)Wpe, bpe, d, xres);
-  else
-    k_patch_embed<float><<<g, 256, 0, s>>>(x, B, rows, C, F, H, W, (const float*)Wpe, bpe, d, xres);
   count_launch();
-  return cudaGetLastError();
+  if (dtype == BF16)
+    return launch_pdl(k_patch_embed<bf16>, g, 256, 0, s, x, B, rows, C, F, H, W, (const bf16*)Wpe,
+                      bpe, d, xres);
+  return launch_pdl(k_patch_embed<float>, g, 256, 0, s, x, B, rows, C, F, H, W, (const float*)Wpe,
+                    bpe, d, xres);
 }
 
 // ---------------------------------------------------------------- LayerNorm + modulation
@@ -230,6 +245,8 @@ __global__ void __launch_bounds__(256) k_ln_mod(const float* __restrict__ x, int
                                                 const float* __restrict__ a,
                                                 const float* __restrict__ b, int mode, float eps,
                                                 T* __restrict__ out) {
+  pdl_wait();
+  pdl_release();
   const int lane = threadIdx.x & 31;
   const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (row >= M) return;
@@ -270,6 +287,8 @@ __global__ void __launch_bounds__(256) k_ln_mod_r(const float* __restrict__ x, i
                                                   const float* __restrict__ a,
                                                   const float* __restrict__ b, int mode, float eps,
                                                   T* __restrict__ out) {
+  pdl_wait();
+  pdl_release();
   constexpr int d = 128 * VPL;
   const int lane = threadIdx.x & 31;
   const int64_t row = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -316,11 +335,11 @@ static cudaError_t ln_dispatch(const float* x, int M, int d, const float* a, con
   const int g = (M + 7) / 8;
   switch (d % 128 == 0 ? d / 128 : 0) {
 #define LN_CASE(V) \
-  case V: k_ln_mod_r<T, V><<<g, 256, 0, s>>>(x, M, a, b, mode, eps, out); break;
+  case V: return launch_pdl(k_ln_mod_r<T, V>, g, 256, 0, s, x, M, a, b, mode, eps, out);
     LN_CASE(1) LN_CASE(2) LN_CASE(4) LN_CASE(6) LN_CASE(8) LN_CASE(12) LN_CASE(16) LN_CASE(24)
     LN_CASE(32)
 #undef LN_CASE
-    default: k_ln_mod<T><<<g, 256, 0, s>>>(x, M, d, a, b, mode, eps, out);
+    default: return launch_pdl(k_ln_mod<T>, g, 256, 0, s, x, M, d, a, b, mode, eps, out);
   }
   return cudaGetLastError();
 }
@@ -397,6 +416,8 @@ __device__ __forceinline__ void scale8(float (&v)[8], float rstd, const float* g
 // of squares, then normalize / rotate / store in place; the second read hits L1).
 template <typename T>
 __global__ void __launch_bounds__(256) k_norm_rope(NormRopeArgs a) {
+  pdl_wait();
+  pdl_release();
   const int lane = threadIdx.x & 31;
   const int64_t gw = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int64_t r = gw / a.nsec;
@@ -428,6 +449,8 @@ __global__ void __launch_bounds__(256) k_norm_rope(NormRopeArgs a) {
 // d = 256 * CPL; all loads are issued before the reduction.
 template <int CPL>
 __global__ void __launch_bounds__(256) k_norm_rope_r(NormRopeArgs a) {
+  pdl_wait();
+  pdl_release();
   constexpr int D = 256 * CPL;
   const int lane = threadIdx.x & 31;
   const int64_t gw = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -463,19 +486,20 @@ cudaError_t qk_norm_rope(const NormRopeArgs& a, cudaStream_t s) {
     return cudaErrorInvalidValue;
   const int64_t warps = (int64_t)a.rows * a.nsec;
   const int g = (int)((warps + 7) / 8);
+  cudaError_t e = cudaSuccess;
   if (a.dtype == BF16) {
     switch (a.d % 256 == 0 ? a.d / 256 : 0) {
 #define NR_CASE(C) \
-  case C: k_norm_rope_r<C><<<g, 256, 0, s>>>(a); break;
+  case C: e = launch_pdl(k_norm_rope_r<C>, g, 256, 0, s, a); break;
       NR_CASE(1) NR_CASE(2) NR_CASE(3) NR_CASE(4) NR_CASE(6) NR_CASE(8) NR_CASE(12) NR_CASE(16)
 #undef NR_CASE
-      default: k_norm_rope<bf16><<<g, 256, 0, s>>>(a);
+      default: e = launch_pdl(k_norm_rope<bf16>, g, 256, 0, s, a);
     }
   } else {
-    k_norm_rope<float><<<g, 256, 0, s>>>(a);
+    e = launch_pdl(k_norm_rope<float>, g, 256, 0, s, a);
   }
   count_launch();
-  return cudaGetLastError();
+  return e;
 }
 
 // ---------------------------------------------------------------- head + unpatchify
@@ -485,6 +509,8 @@ __global__ void __launch_bounds__(256) k_head(const float* __restrict__ xres, in
                                               const T* __restrict__ Wh,
                                               const float* __restrict__ bh, float eps, int C, int F,
                                               int H, int W, float* __restrict__ out) {
+  pdl_wait();
+  pdl_release();
   extern __shared__ float h[];  // d floats
   __shared__ float red[32];
   const int r = blockIdx.x;
@@ -527,14 +553,12 @@ cudaError_t head_unpatchify(const float* xres, int nseq, int L, int d, const flo
   const size_t sm = (size_t)d * sizeof(float);
   if (sm > 48 * 1024) return cudaErrorInvalidValue;
   const int rows = nseq * L;
-  if (dtype == BF16)
-    k_head<bf16><<<rows, 256, sm, s>>>(xres, L, d, head_mod, (const bf16*)Whead, bhead, eps, C, F, H,
-                                       W, out);
-  else
-    k_head<float><<<rows, 256, sm, s>>>(xres, L, d, head_mod, (const float*)Whead, bhead, eps, C, F,
-                                        H, W, out);
   count_launch();
-  return cudaGetLastError();
+  if (dtype == BF16)
+    return launch_pdl(k_head<bf16>, rows, 256, sm, s, xres, L, d, head_mod, (const bf16*)Whead,
+                      bhead, eps, C, F, H, W, out);
+  return launch_pdl(k_head<float>, rows, 256, sm, s, xres, L, d, head_mod, (const float*)Whead,
+                    bhead, eps, C, F, H, W, out);
 }
 
 // ---------------------------------------------------------------- guidance and Euler update
@@ -553,6 +577,8 @@ __device__ __forceinline__ float euler_val(float x, float p, float dsig) {
 __global__ void k_guide(float* __restrict__ x, const float* __restrict__ fc,
                         const float* __restrict__ fu, float* __restrict__ out, int64_t n, float w,
                         float dsig, int mode) {
+  pdl_wait();
+  pdl_release();
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   const int64_t n4 = n / 4;
   const bool vec = ((((uintptr_t)x) | ((uintptr_t)fc) | ((uintptr_t)fu) | ((uintptr_t)out)) & 15) == 0;
@@ -588,7 +614,9 @@ __global__ void k_guide(float* __restrict__ x, const float* __restrict__ fc,
 static cudaError_t launch_guide(float* x, const float* fc, const float* fu, float* out, int64_t n,
                                 float w, float dsig, int mode, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
-  k_guide<<<grid_for((n + 3) / 4, 256), 256, 0, s>>>(x, fc, fu, out, n, w, dsig, mode);
+  cudaError_t e = launch_pdl(k_guide, grid_for((n + 3) / 4, 256), 256, 0, s, x, fc, fu, out, n, w,
+                             dsig, mode);
+  if (e != cudaSuccess) return e;
   count_launch();
   return cudaGetLastError();
 }
@@ -615,6 +643,8 @@ constexpr int DIS_THREADS = 256;
 __global__ void __launch_bounds__(DIS_THREADS) k_dis_partial(const float* __restrict__ vL,
                                                              const float* __restrict__ vS,
                                                              int64_t n, float* __restrict__ part) {
+  pdl_wait();
+  pdl_release();
   __shared__ float red[32];
   const int b = blockIdx.y, nblk = gridDim.x;
   const float* l = vL + (int64_t)b * n;
@@ -651,6 +681,8 @@ __global__ void __launch_bounds__(DIS_THREADS) k_dis_partial(const float* __rest
 
 __global__ void __launch_bounds__(256) k_dis_final(const float* __restrict__ part, int nblk,
                                                    float eps, float* __restrict__ accum) {
+  pdl_wait();
+  pdl_release();
   __shared__ double rd[256], rl[256];
   const int b = blockIdx.x;
   double sd = 0.0, sl = 0.0;
@@ -685,8 +717,10 @@ int disagreement_blocks(int64_t n_per_sample) {
 cudaError_t disagreement(const float* vL, const float* vS, int B, int64_t n, float eps,
                          float* accum, float* scratch, int nblk, cudaStream_t s) {
   if (B <= 0) return cudaSuccess;
-  k_dis_partial<<<dim3(nblk, B), DIS_THREADS, 0, s>>>(vL, vS, n, scratch);
-  k_dis_final<<<B, 256, 0, s>>>(scratch, nblk, eps, accum);
+  cudaError_t e = launch_pdl(k_dis_partial, dim3(nblk, B), DIS_THREADS, 0, s, vL, vS, n, scratch);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(k_dis_final, B, 256, 0, s, scratch, nblk, eps, accum);
+  if (e != cudaSuccess) return e;
   count_launch(2);
   return cudaGetLastError();
 }

@@ -16,6 +16,8 @@ __device__ __forceinline__ float gelu_tanh(float u) {
 
 __global__ void __launch_bounds__(256) k_gemm_f32(const float* __restrict__ A,
                                                   const float* __restrict__ W, GemmArgs g) {
+  pdl_wait();
+  pdl_release();
   __shared__ float As[TK][TM + 4];
   __shared__ float Ws[TK][TN + 4];
   const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
@@ -69,9 +71,8 @@ cudaError_t gemm_f32(const float* A, const float* W, const GemmArgs& g, cudaStre
   if (g.M <= 0 || g.N <= 0) return cudaSuccess;
   dim3 grid((g.N + TN - 1) / TN, (g.M + TM - 1) / TM);
   if (grid.y > 65535) return cudaErrorInvalidConfiguration;
-  k_gemm_f32<<<grid, 256, 0, s>>>(A, W, g);
   count_launch();
-  return cudaGetLastError();
+  return launch_pdl(k_gemm_f32, grid, 256, 0, s, A, W, g);
 }
 
 }  // namespace track

@@ -101,6 +101,9 @@ __global__ void __launch_bounds__(192, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // The prologue above overlaps the previous kernel; inputs and outputs are touched only now.
+  pdl_wait();
+  pdl_release();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -314,9 +317,8 @@ cudaError_t launch_tc(const void* A, const void* W, const GemmArgs& g, cudaStrea
   if (e != cudaSuccess) return e;
   const int tiles = ((g.M + BM - 1) / BM) * ((g.N + BN - 1) / BN);
   const int grid = tiles < num_sms() ? tiles : num_sms();
-  k_gemm_tc<BN, STAGES><<<grid, 192, S::SMEM, s>>>(ta, tb, tc, g);
   count_launch();
-  return cudaGetLastError();
+  return launch_pdl(k_gemm_tc<BN, STAGES>, grid, 192, S::SMEM, s, ta, tb, tc, g);
 }
 
 }  // namespace
