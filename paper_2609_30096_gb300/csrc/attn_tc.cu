@@ -2,23 +2,29 @@
 // O = softmax(Q K^T / sqrt(hd)) V per (sequence, head), no mask.
 //
 // One CTA per 128-query tile of one (sequence, head), 192 threads:
-//   warp 0      TMA: the Q tile once, then K and V tiles of 128 keys, each
-//               through its own two-stage ring (lane 0 K, lane 1 V; 4-D tensor
-//               maps over head-major or token-major operands, 128-byte swizzle,
-//               zero fill past L).  A K stage is released as soon as S = Q K^T
-//               of its tile completes.
+//   warp 0      TMA: the Q tile once, then K and V tiles of 128 keys, K through
+//               a three-stage ring (lane 0) and V through a two-stage ring
+//               (lane 1); 4-D tensor maps over head-major or token-major
+//               operands, 128-byte swizzle, zero fill past L.  A K stage is
+//               released as soon as S = Q K^T of its tile completes.
 //   warp 1      allocates TMEM (O: hd columns; S: two 128-column buffers) and
 //               issues, from one thread, S(j+1) = Q K(j+1)^T while the softmax
-//               warps work on S(j), then O += P(j) V(j) once P(j) is ready.
-//               V is the MN-major B operand, so no transposed copy is needed.
+//               warps work on S(j), then O += P(j) V(j) once P(j) is ready.  P
+//               is read from TMEM (the A operand of the MMA), V is the MN-major
+//               B operand from shared memory, so no transposed copy is needed.
 //   warps 2-9   softmax, two warpgroups splitting each 128-key tile by columns
 //               (64 keys each), one thread per query row (its TMEM lane): row
 //               maximum over the valid keys (halves combined through shared
 //               memory), lazy rescaling of O (only when the running maximum
 //               grows by more than 2^8; each group rescales its half of O's
-//               columns in TMEM), P = exp2(S * log2(e)/sqrt(hd) - m) rounded to
-//               bf16 into 128-byte-swizzled shared memory, and at the end O / l
-//               stored to the token-major output.
+//               columns in TMEM, after P V of the previous tile completes),
+//               P = exp2(S * log2(e)/sqrt(hd) - m) rounded to bf16 pairs and
+//               written over the first 32 of the group's 64 S columns, and at
+//               the end O / l stored to the token-major output.  Because P
+//               lives in the S buffer it came from, the softmax of tile j+1
+//               never waits for P V of tile j unless it must rescale O.
+// Tensor-core operations issued by one thread execute in issue order, so
+// S(j+2), issued after O += P(j) V(j), overwrites P(j) only after it was read.
 // Every mbarrier wait is bounded (see tc_common.cuh).
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -43,10 +49,10 @@ template <int HD>
 struct AtShape {
   static constexpr uint32_t Q_BYTES = AT_BM * HD * 2;   // HD/64 boxes of [128 rows][128 B]
   static constexpr uint32_t KV_BYTES = AT_BN * HD * 2;  // one K or V tile
-  static constexpr uint32_t P_BYTES = AT_BM * AT_BN * 2;
   static constexpr uint32_t X_BYTES = 2 * 2 * AT_BM * 4;  // row partials [parity][half][row]
-  static constexpr int STAGES = 2;
-  static constexpr size_t SMEM = 1024 + Q_BYTES + 2 * STAGES * KV_BYTES + P_BYTES + X_BYTES + 256;
+  static constexpr int KST = 3;  // K ring stages
+  static constexpr int VST = 2;  // V ring stages
+  static constexpr size_t SMEM = 1024 + Q_BYTES + (KST + VST) * KV_BYTES + X_BYTES + 256;
   static constexpr uint32_t TMEM_COLS = 512;
 };
 
@@ -83,21 +89,20 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* sQ = smem;
   uint8_t* sK = sQ + S::Q_BYTES;
-  uint8_t* sV = sK + S::STAGES * S::KV_BYTES;
-  uint8_t* sP = sV + S::STAGES * S::KV_BYTES;
-  float* xch = (float*)(sP + S::P_BYTES);  // [2][2][AT_BM] partial row maxima / sums
-  uint64_t* bars = (uint64_t*)(sP + S::P_BYTES + S::X_BYTES);
+  uint8_t* sV = sK + S::KST * S::KV_BYTES;
+  float* xch = (float*)(sV + S::VST * S::KV_BYTES);  // [2][2][AT_BM] partial row maxima / sums
+  uint64_t* bars = (uint64_t*)((uint8_t*)xch + S::X_BYTES);
   uint64_t* q_full = bars;
-  uint64_t* k_full = bars + 1;    // [2] per K stage
-  uint64_t* k_empty = bars + 3;   // [2] freed once S = Q K^T of the tile has completed
-  uint64_t* v_full = bars + 5;    // [2] per V stage
-  uint64_t* v_empty = bars + 7;   // [2] freed once P V of the tile has completed
-  uint64_t* s_full = bars + 9;    // [2] per S buffer
-  uint64_t* p_full = bars + 11;   // P of the tile written (8 softmax warps)
-  uint64_t* o_done = bars + 12;   // P V of the tile has completed
-  uint64_t* xbar = bars + 13;     // [2] both halves' row partials written (per parity)
-  uint64_t* done = bars + 15;
-  uint32_t* tmem_slot = (uint32_t*)(bars + 16);
+  uint64_t* k_full = bars + 1;    // [3] per K stage
+  uint64_t* k_empty = bars + 4;   // [3] freed once S = Q K^T of the tile has completed
+  uint64_t* v_full = bars + 7;    // [2] per V stage
+  uint64_t* v_empty = bars + 9;   // [2] freed once P V of the tile has completed
+  uint64_t* s_full = bars + 11;   // [2] per S buffer
+  uint64_t* p_full = bars + 13;   // [2] P of the tile written into its S buffer (8 softmax warps)
+  uint64_t* o_done = bars + 15;   // P V of the tile has completed
+  uint64_t* xbar = bars + 16;     // [2] both halves' row partials written (per parity)
+  uint64_t* done = bars + 18;     // every MMA of the CTA has completed
+  uint32_t* tmem_slot = (uint32_t*)(bars + 19);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -107,15 +112,17 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(su32(q_full), 1);
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < S::KST; ++i) {
       mbar_init(su32(&k_full[i]), 1);
       mbar_init(su32(&k_empty[i]), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
       mbar_init(su32(&v_full[i]), 1);
       mbar_init(su32(&v_empty[i]), 1);
       mbar_init(su32(&s_full[i]), 1);
+      mbar_init(su32(&p_full[i]), 8);
       mbar_init(su32(&xbar[i]), 8);
     }
-    mbar_init(su32(p_full), 8);
     mbar_init(su32(o_done), 1);
     mbar_init(su32(done), 1);
     *abort_flag = 0;
@@ -145,10 +152,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         for (int b = 0; b < NB; ++b)
           tma_load_rows(su32(sQ + b * AT_BM * 128), &tmQ, q_tok, b * 64, q0, hq, sq, su32(q_full));
       }
-      uint32_t armed[2] = {0, 0};
+      const int nst = kside ? S::KST : S::VST;
+      uint32_t armed[S::KST] = {};
       for (int kt = 0; kt < nkt; ++kt) {
-        const int st = kt & 1;
-        if (!mbar_wait(su32(&empty[st]), ((kt >> 1) & 1) ^ 1, abort_flag, err, 11)) break;
+        const int st = kt % nst;
+        if (!mbar_wait(su32(&empty[st]), ((kt / nst) & 1) ^ 1, abort_flag, err, 11)) break;
         mbar_expect_tx(su32(&full[st]), S::KV_BYTES);
         for (int b = 0; b < NB; ++b)
           tma_load_rows(su32(ring + st * S::KV_BYTES + b * AT_BN * 128), tm, kv_tok, b * 64,
@@ -157,26 +165,26 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       }
       // Every copy this thread issued has landed before the CTA may exit.
       if (kside) mbar_drain(su32(q_full), 0, err, 15);
-      for (int i = 0; i < 2; ++i)
+      for (int i = 0; i < nst; ++i)
         if (armed[i] != 0) mbar_drain(su32(&full[i]), (armed[i] - 1) & 1, err, 15);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idS = idesc_bf16(AT_BM, AT_BN);
       constexpr uint32_t idO = idesc_bf16_bmn(AT_BM, HD);
-      const uint32_t qa = su32(sQ), pa = su32(sP);
+      const uint32_t qa = su32(sQ);
       auto issue_s = [&](int kt) -> bool {
-        const int st = kt & 1;
-        if (!mbar_wait(su32(&k_full[st]), (kt >> 1) & 1, abort_flag, err, 12)) return false;
+        const int st = kt % S::KST;
+        if (!mbar_wait(su32(&k_full[st]), (kt / S::KST) & 1, abort_flag, err, 12)) return false;
         tc_fence_after();
         const uint32_t ka = su32(sK + st * S::KV_BYTES);
-        const uint32_t d = tmem_base + TM_S0 + (uint32_t)(st * AT_BN);
+        const uint32_t d = tmem_base + TM_S0 + (uint32_t)((kt & 1) * AT_BN);
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk)
           mma_bf16(d, sdesc_sw128(qa + (kk >> 2) * (AT_BM * 128) + (kk & 3) * 32),
                    sdesc_sw128(ka + (kk >> 2) * (AT_BN * 128) + (kk & 3) * 32), idS,
                    kk > 0 ? 1u : 0u);
-        mma_commit(su32(&s_full[st]));
+        mma_commit(su32(&s_full[kt & 1]));
         mma_commit(su32(&k_empty[st]));
         return true;
       };
@@ -187,16 +195,18 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       }
       for (int kt = 0; ok && kt < nkt; ++kt) {
         if (kt + 1 < nkt && !issue_s(kt + 1)) break;
-        const int st = kt & 1;  // V stage of this tile
+        const int st = kt & 1;  // V stage and S/P buffer of this tile
         if (!mbar_wait(su32(&v_full[st]), (kt >> 1) & 1, abort_flag, err, 21)) break;
-        if (!mbar_wait(su32(p_full), kt & 1, abort_flag, err, 14)) break;
+        if (!mbar_wait(su32(&p_full[st]), (kt >> 1) & 1, abort_flag, err, 14)) break;
         tc_fence_after();
         const uint32_t va = su32(sV + st * S::KV_BYTES);
+        // P keys 16kk..16kk+15: half kk/4 of the tile, columns 8(kk%4).. of that half's S
+        const uint32_t pt = tmem_base + TM_S0 + (uint32_t)(st * AT_BN);
 #pragma unroll
         for (int kk = 0; kk < AT_BN / 16; ++kk)
-          mma_bf16(tmem_base, sdesc_sw128(pa + (kk >> 2) * (AT_BM * 128) + (kk & 3) * 32),
-                   sdesc_sw128_mn(va + kk * 16 * 128, AT_BN * 128), idO,
-                   (kt > 0 || kk > 0) ? 1u : 0u);
+          mma_bf16_ts(tmem_base, pt + (uint32_t)((kk >> 2) * (AT_BN / 2) + (kk & 3) * 8),
+                      sdesc_sw128_mn(va + kk * 16 * 128, AT_BN * 128), idO,
+                      (kt > 0 || kk > 0) ? 1u : 0u);
         mma_commit(su32(&v_empty[st]));
         mma_commit(su32(o_done));
       }
@@ -251,15 +261,17 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         break;
       }
       const float mt = fmaxf(hmax, xp[(half ^ 1) * AT_BM + row]) * scale_log2;
-      // P V of the previous tile must be complete before P is overwritten (and O rescaled).
       if (kt > 0) {
-        if (!warp_wait(su32(o_done), (kt - 1) & 1, abort_flag, err, 18)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
         const bool need = mt > m + 8.f;
         if (__any_sync(0xffffffffu, need)) {
+          // P V of the previous tile must be complete before O is rescaled.  At
+          // least P V of tile kt-2 has completed (S(kt) was issued after it),
+          // and P V of tile kt needs this warp's P, so the parity names tile kt-1.
+          if (!warp_wait(su32(o_done), (kt - 1) & 1, abort_flag, err, 18)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
           const float alpha = need ? exp2_approx(m - mt) : 1.f;
           if (need) {
             m = mt;
@@ -278,29 +290,25 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       } else {
         m = mt;
       }
-      // P = exp2(S * scale - m) for this half: K-block `half` of the P tile.
+      // P = exp2(S * scale - m) for this half, two keys per TMEM column (the
+      // lower key in the low 16 bits), over this half's first 32 S columns.
       float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
       const float nm = -m;
+      uint32_t pk[KH / 2];
 #pragma unroll
-      for (int cidx = 0; cidx < KH / 8; ++cidx) {  // 16-byte chunks of 8 keys
-        uint32_t pk[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const float p0 = exp2_approx(fmaf(__uint_as_float(sv[8 * cidx + 2 * i]), scale_log2, nm));
-          const float p1 =
-              exp2_approx(fmaf(__uint_as_float(sv[8 * cidx + 2 * i + 1]), scale_log2, nm));
-          ps[2 * i] += p0;
-          ps[2 * i + 1] += p1;
-          pk[i] = pack_bf16x2(p0, p1);
-        }
-        uint8_t* dst = sP + half * (AT_BM * 128) + row * 128 + ((cidx ^ (row & 7)) << 4);
-        *reinterpret_cast<uint4*>(dst) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      for (int i = 0; i < KH / 2; ++i) {
+        const float p0 = exp2_approx(fmaf(__uint_as_float(sv[2 * i]), scale_log2, nm));
+        const float p1 = exp2_approx(fmaf(__uint_as_float(sv[2 * i + 1]), scale_log2, nm));
+        ps[(2 * i) & 7] += p0;
+        ps[(2 * i + 1) & 7] += p1;
+        pk[i] = pack_bf16x2(p0, p1);
       }
+      tmem_st32(tS, pk);
       l += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
-      fence_async_shared();
+      tmem_st_wait();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(su32(p_full));
+      if (lane == 0) mbar_arrive(su32(&p_full[kt & 1]));
     }
     // Combine the two halves' sums (one more exchange round), then O / l.
     bool fin = ok;
@@ -312,7 +320,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       fin = warp_wait(su32(&xbar[nkt & 1]), (nkt >> 1) & 1, abort_flag, err, 23);
       if (fin) l += xp[(half ^ 1) * AT_BM + row];
     }
-    if (fin && warp_wait(su32(o_done), (nkt - 1) & 1, abort_flag, err, 19)) {
+    if (fin && warp_wait(su32(done), 0, abort_flag, err, 19)) {
       tc_fence_after();
       const float inv = 1.f / l;
       const int qrow = q0 + row;
