@@ -294,6 +294,7 @@ def run_ours(args):
     if world > 1:
         tdist.init_process_group("nccl")
     _build.build()
+    T.track_gemm_schedule(GEMM_SCHEDULES[args.gemm_schedule])
 
     wl = synth.WORKLOADS[WORKLOAD]
     B = wl.batch
@@ -501,6 +502,9 @@ def run_ours(args):
 
 
 # ---------------------------------------------------------------- single kernels
+GEMM_SCHEDULES = {"auto": 0, "dp": 1, "sk": 2}   # track_gemm_schedule modes
+
+
 def run_kernel(args):
     """Times one kernel class alone at the workload's shapes (large model, `--batch`
     sequences): the GEMMs of one block, or self- and cross-attention."""
@@ -511,6 +515,7 @@ def run_kernel(args):
 
     _build.build()
     torch.cuda.set_device(0)
+    T.track_gemm_schedule(GEMM_SCHEDULES[args.gemm_schedule])
     wl = synth.WORKLOADS[WORKLOAD]
     a = wl.large
     M = args.batch * a.tokens
@@ -520,6 +525,7 @@ def run_kernel(args):
     cases = []
     if args.kernel == "gemm":
         for name, N, K, epi in (("qkv", 3 * d, d, T.EPI_STORE), ("out_proj", d, d, T.EPI_RESID_GATE),
+                                ("cross_q", d, d, T.EPI_STORE),
                                 ("ffn_up", F, d, T.EPI_GELU), ("ffn_down", d, F, T.EPI_RESID_GATE)):
             X, W = rnd(M, K), rnd(N, K)
             b = torch.zeros(N, device="cuda")
@@ -591,6 +597,8 @@ def main():
     ap.add_argument("--kernel", choices=["gemm", "attention", "hbm"], default=None,
                     help="time one kernel class alone at the workload's shapes")
     ap.add_argument("--batch", type=int, default=1, help="sequences for --kernel")
+    ap.add_argument("--gemm-schedule", choices=["auto", "dp", "sk"], default="auto",
+                    help="bf16 GEMM schedule: makespan model, data-parallel or stream-K")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)     # at least three untimed warm-up steps
     if args.impl == "reference":

@@ -246,6 +246,26 @@ int track_sample(track_model* large, track_model* small, const uint8_t* policy,
 int track_linear(int dtype, const void* X, const void* W, const float* bias, int M, int N,
                  int K, int epilogue, const float* gate, void* out, int ldo, track_stream s);
 
+/* Schedule of the TRACK_BF16 GEMM (process-wide, every device and stream).
+ * TRACK_GEMM_AUTO (the default) picks per launch, by a makespan model, between
+ * data-parallel (each CTA computes whole output tiles) and stream-K (the
+ * tiles' 64-wide k-blocks are shared out evenly over one CTA per SM; a tile
+ * split across CTAs is summed by the last of them in k order).
+ * TRACK_GEMM_DATA_PARALLEL always uses whole tiles; TRACK_GEMM_STREAM_K uses
+ * stream-K wherever the shape allows it (every CTA gets at least one k-block
+ * and no tile spans more than 4 CTAs), else decides as AUTO.  OR-ing in
+ * TRACK_GEMM_MULTICAST runs the CTAs in clusters of two that compute vertically
+ * adjacent row tiles and share each W tile through TMA multicast (half the W
+ * bytes per SM), when the GEMM has more than 128 rows.  Every schedule is
+ * deterministic (same inputs, same launch: same bits); two schedules differ in
+ * fp32 rounding only (data-parallel gives the same bits with or without
+ * multicast).  EINVAL for any other mode. */
+#define TRACK_GEMM_AUTO 0
+#define TRACK_GEMM_DATA_PARALLEL 1
+#define TRACK_GEMM_STREAM_K 2
+#define TRACK_GEMM_MULTICAST 4
+int track_gemm_schedule(int mode);
+
 /* O = softmax(Q K^T / sqrt(hd)) V per (sequence, head), no mask.  Q: [S, H, Lq,
  * hd], K, V: [S, H, Lk, hd], O: [S, Lq, H, hd], all in dtype (bf16 or fp32);
  * hd in {64, 128}. */

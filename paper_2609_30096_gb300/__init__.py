@@ -20,6 +20,8 @@ from ._build import LIB as _LIB_PATH
 TRACK_OK, TRACK_EINVAL, TRACK_ENOMEM, TRACK_ECUDA, TRACK_EUNSUPPORTED, TRACK_ETIMEOUT = range(6)
 FP32, BF16 = 0, 1
 EPI_STORE, EPI_GELU, EPI_RESID_GATE, EPI_RESID = range(4)
+GEMM_AUTO, GEMM_DATA_PARALLEL, GEMM_STREAM_K = range(3)
+GEMM_MULTICAST = 4  # OR-ed into a schedule: two-CTA clusters sharing W tiles
 
 
 class TrackError(RuntimeError):
@@ -56,6 +58,7 @@ def lib():
         "track_sync": (_I, [_P]),
         "track_launch_count": (_L, []),
         "track_profile_enable": (_I, [_I]),
+        "track_gemm_schedule": (_I, [_I]),
         "track_profile_read": (_I, [_P, _P, _P]),
         "track_weight_count": (_I, [_P]),
         "track_weight_shape": (_I, [_P, _I, _P, _P]),
@@ -137,6 +140,12 @@ def track_sync(stream=None):
 
 def track_launch_count() -> int:
     return lib().track_launch_count()
+
+
+def track_gemm_schedule(mode: int):
+    """GEMM_AUTO, GEMM_DATA_PARALLEL or GEMM_STREAM_K (optionally | GEMM_MULTICAST)
+    for every later bf16 GEMM."""
+    _check(lib().track_gemm_schedule(int(mode)))
 
 
 def track_profile_enable(enable: bool):

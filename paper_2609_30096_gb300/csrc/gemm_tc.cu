@@ -1,6 +1,22 @@
 // bf16 GEMM on the sm_103a tensor cores: out = A[M,K] . W[N,K]^T (+ epilogue).
 //
-// Persistent, warp-specialised kernel, one CTA per SM:
+// Persistent, warp-specialised kernel, one CTA per SM.  When there are at
+// least two row tiles the CTAs run in clusters of two: the pair computes a
+// 256-row work tile (one 128-row tile each) and shares the W tile through TMA
+// multicast, each CTA fetching half of it for both, which cuts the operand
+// bytes an SM pulls from L2 per k-block by a third at BN = 256.  A worker (a
+// CTA, or a cluster) follows one of two schedules:
+//   data-parallel  worker w takes work tiles w, w + workers, ... (whole K loop);
+//   stream-K       the work tiles' k-blocks form one sequence of U units and
+//                  worker w takes the contiguous share [w U / G, (w+1) U / G),
+//                  so every worker does the same number of k-blocks whatever
+//                  the tile count.  A tile split across workers is finished by
+//                  whichever ends its part last: the others write their fp32
+//                  partial sums to a workspace slot and count in on a
+//                  per-(tile, warp) counter; the last one adds the parts in k
+//                  order (a fixed order, so the result does not depend on
+//                  timing), applies the epilogue and resets the counter for
+//                  the next launch.
 //   warp 0      TMA producer: 128x64 A tile and BNx64 W tile per stage into a
 //               STAGES-deep shared-memory ring (128-byte swizzle, zero fill past
 //               the matrix edges), completion counted on an mbarrier.
@@ -18,7 +34,10 @@
 #include <cuda_bf16.h>
 #include <math.h>
 
+#include <atomic>
+#include <map>
 #include <mutex>
+#include <utility>
 
 #include "internal.h"
 #include "tc_common.cuh"
@@ -31,8 +50,12 @@ using namespace tc;
 typedef __nv_bfloat16 bf16;
 constexpr int BM = 128, BK = 64;
 
+// GELU, tanh form: 0.5 u (1 + tanh z) with z = sqrt(2/pi) (u + 0.044715 u^3),
+// evaluated as u / (1 + e^(-2z)) (the same function; no cancellation for
+// negative u) with the fast exp and divide intrinsics (about 1e-6 relative).
 __device__ __forceinline__ float gelu_tanh(float u) {
-  return 0.5f * u * (1.f + tanhf(0.7978845608028654f * fmaf(0.044715f * u, u * u, u)));
+  const float z = 0.7978845608028654f * fmaf(0.044715f * u, u * u, u);
+  return __fdividef(u, 1.f + __expf(-2.f * z));
 }
 
 // Writes this thread's 128-byte row `row` (8 chunks of 16 bytes) into a staging
@@ -49,6 +72,66 @@ __device__ __forceinline__ uint32_t pack2(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&t);
 }
 
+// Stream-K state: counters [4 * CTA tiles] (zero between launches) and 2 * grid
+// partial-sum slots of 128 x BN floats.  cnt == nullptr selects data-parallel.
+struct SkArgs {
+  int* cnt;
+  float* ws;
+  int64_t units;  // work tiles * k-blocks
+};
+
+// Worker (cluster) whose share [w U / G, (w+1) U / G) holds unit u.
+__device__ __forceinline__ int sk_worker_of(int64_t u, int64_t U, int G) {
+  return (int)(((u + 1) * G + U - 1) / U) - 1;
+}
+
+// Segment sequence of worker w of G: (work tile, first k-block, end k-block).
+struct SegIter {
+  int64_t u, u1;
+  int tile, stride, num_tiles, nk;
+  bool sk;
+  __device__ SegIter(bool sk_, int64_t U, int num_tiles_, int nk_, int w, int G) {
+    sk = sk_;
+    num_tiles = num_tiles_;
+    nk = nk_;
+    u = (int64_t)w * U / G;
+    u1 = (int64_t)(w + 1) * U / G;
+    tile = w;
+    stride = G;
+  }
+  // True once the segment just returned is the worker's last.
+  __device__ bool done() const { return sk ? u >= u1 : tile >= num_tiles; }
+  __device__ bool next(int& t, int& k0, int& k1) {
+    if (sk) {
+      if (u >= u1) return false;
+      t = (int)(u / nk);
+      k0 = (int)(u - (int64_t)t * nk);
+      const int64_t left = u1 - u;
+      k1 = left < (int64_t)(nk - k0) ? k0 + (int)left : nk;
+      u += k1 - k0;
+      return true;
+    }
+    if (tile >= num_tiles) return false;
+    t = tile;
+    k0 = 0;
+    k1 = nk;
+    tile += stride;
+    return true;
+  }
+};
+
+__device__ __forceinline__ int ld_acquire(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+constexpr int SK_MAX_PARTS = 4;     // the host only picks stream-K when no tile spans more workers
+// Makespan-model cost of the stream-K fix-up (publishing a partial tile, the
+// counter round trips and the final combine: about 8 us), in the model's units
+// of one 64-deep k-block of a 256-wide tile = 406 (about 0.33 us).
+constexpr double SK_FIXUP = 10000.0;
+
 template <int BN, int STAGES>
 struct TcShape {
   static constexpr uint32_t A_BYTES = BM * BK * 2;
@@ -59,10 +142,17 @@ struct TcShape {
   static constexpr size_t SMEM = 1024 + (size_t)STAGES * (A_BYTES + B_BYTES) + STG_BYTES + 256;
 };
 
-template <int BN, int STAGES>
+// CL = CTAs per cluster (1 or 2).  With CL = 2 the two CTAs of a cluster take
+// vertically adjacent 128-row tiles of the same BN columns (a "work tile" of
+// 256 rows): each loads its own A tile and one half of the shared W tile, which
+// TMA multicasts into both CTAs, so each SM pulls 128x64 + (BN/2)x64 elements
+// per k-block instead of 128x64 + BNx64.  A stage is refilled only after the
+// MMAs of both CTAs have read it (its empty barrier counts one multicast
+// commit from each).
+template <int BN, int STAGES, int CL>
 __global__ void __launch_bounds__(192, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-              const __grid_constant__ CUtensorMap tmC, const GemmArgs g) {
+              const __grid_constant__ CUtensorMap tmC, const GemmArgs g, const SkArgs sk) {
   using S = TcShape<BN, STAGES>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -79,14 +169,18 @@ __global__ void __launch_bounds__(192, 1)
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int rank = CL == 1 ? 0 : (int)cluster_ctarank();
+  const int worker = blockIdx.x / CL, workers = gridDim.x / CL;
   const int m_tiles = (g.M + BM - 1) / BM, n_tiles = (g.N + BN - 1) / BN;
-  const int num_tiles = m_tiles * n_tiles;
+  const int m_units = (m_tiles + CL - 1) / CL;  // work tiles per column of tiles
+  const int num_tiles = m_units * n_tiles;
   const int nk = g.K / BK;
+  const bool use_sk = sk.cnt != nullptr;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < STAGES; ++i) {
       mbar_init(su32(&full[i]), 1);
-      mbar_init(su32(&empty[i]), 1);
+      mbar_init(su32(&empty[i]), CL);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(su32(&accf[i]), 1);
@@ -99,6 +193,7 @@ __global__ void __launch_bounds__(192, 1)
   if (warp == 1) tmem_alloc(su32(tmem_slot), S::TMEM_COLS);
   tc_fence_before();
   __syncthreads();
+  if (CL > 1) cluster_sync();  // the peer's barriers exist before any multicast reaches them
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   // The prologue above overlaps the previous kernel; inputs and outputs are touched only now.
@@ -114,10 +209,12 @@ __global__ void __launch_bounds__(192, 1)
       uint32_t armed[STAGES];
 #pragma unroll
       for (int i = 0; i < STAGES; ++i) armed[i] = 0;
-      for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
-        const int mt = tile % m_tiles, nt = tile / m_tiles;
+      SegIter it(use_sk, sk.units, num_tiles, nk, worker, workers);
+      int tile, kb0, kb1;
+      while (it.next(tile, kb0, kb1)) {
+        const int mt = (tile % m_units) * CL + rank, nt = tile / m_units;
         bool ok = true;
-        for (int kb = 0; kb < nk; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(su32(&empty[stage]), phase ^ 1, abort_flag, g.err, 1)) {
             ok = false;
             break;
@@ -125,7 +222,13 @@ __global__ void __launch_bounds__(192, 1)
           const uint32_t fb = su32(&full[stage]);
           mbar_expect_tx(fb, S::A_BYTES + S::B_BYTES);
           tma_load_2d(su32(sA + stage * S::A_BYTES), &tmA, kb * BK, mt * BM, fb);
-          tma_load_2d(su32(sB + stage * S::B_BYTES), &tmB, kb * BK, nt * BN, fb);
+          if (CL == 1) {
+            tma_load_2d(su32(sB + stage * S::B_BYTES), &tmB, kb * BK, nt * BN, fb);
+          } else {
+            constexpr int HB = BN / CL;  // W rows this CTA fetches for the cluster
+            tma_load_2d_mc(su32(sB + stage * S::B_BYTES + rank * HB * 128), &tmB, kb * BK,
+                           nt * BN + rank * HB, fb, (uint16_t)((1u << CL) - 1));
+          }
           ++armed[stage];
           if (++stage == STAGES) {
             stage = 0;
@@ -134,22 +237,28 @@ __global__ void __launch_bounds__(192, 1)
         }
         if (!ok) break;
       }
-      // Every copy this thread issued has landed before the CTA may exit.
+      // Every copy into this CTA has landed, and (in a cluster) both CTAs' MMAs
+      // have released every stage, before the CTA may exit.
 #pragma unroll
-      for (int i = 0; i < STAGES; ++i)
-        if (armed[i] != 0) mbar_drain(su32(&full[i]), (armed[i] - 1) & 1, g.err, 5);
+      for (int i = 0; i < STAGES; ++i) {
+        if (armed[i] == 0) continue;
+        mbar_drain(su32(&full[i]), (armed[i] - 1) & 1, g.err, 5);
+        if (CL > 1) mbar_drain(su32(&empty[i]), (armed[i] - 1) & 1, g.err, 8);
+      }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(BM, BN);
       int stage = 0, acc = 0;
       uint32_t phase = 0, acc_phase = 0;
-      for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+      SegIter it(use_sk, sk.units, num_tiles, nk, worker, workers);
+      int tile, kb0, kb1;
+      while (it.next(tile, kb0, kb1)) {
         if (!mbar_wait(su32(&acce[acc]), acc_phase ^ 1, abort_flag, g.err, 2)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
         bool ok = true;
-        for (int kb = 0; kb < nk; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(su32(&full[stage]), phase, abort_flag, g.err, 3)) {
             ok = false;
             break;
@@ -160,8 +269,9 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
             mma_bf16(d_tmem, sdesc_sw128(a0 + k * 32), sdesc_sw128(b0 + k * 32), idesc,
-                     (kb | k) != 0 ? 1u : 0u);
-          mma_commit(su32(&empty[stage]));
+                     (kb > kb0 || k != 0) ? 1u : 0u);
+          if (CL == 1) mma_commit(su32(&empty[stage]));
+          else mma_commit_mc(su32(&empty[stage]), (uint16_t)((1u << CL) - 1));
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1;
@@ -182,11 +292,25 @@ __global__ void __launch_bounds__(192, 1)
     const int quarter = warp & 3;  // TMEM lanes 32*quarter .. 32*quarter+31
     uint8_t* stg = stg_all + (warp - 2) * 2 * 4096;
     const bool bf16_out = g.epi == EPI_STORE || g.epi == EPI_GELU;
-    const int cw = bf16_out ? 64 : 32;  // columns per staged box (128-byte rows)
     int sb = 0, acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
-      const int mt = tile % m_tiles, nt = tile / m_tiles;
+    const int64_t U = sk.units;
+    constexpr int SLOT = BM * BN;  // floats per partial-sum slot
+    SegIter it(use_sk, U, num_tiles, nk, worker, workers);
+    int tile, kb0, kb1;
+    while (it.next(tile, kb0, kb1)) {
+      const int mt = (tile % m_units) * CL + rank, nt = tile / m_units;
+      const bool final_seg = it.done();
+      // Bias and gate of this tile's columns are pulled into L1 while the MMAs run
+      // (lane l: columns 8l..8l+7); the column loop below reads them with
+      // warp-uniform loads, which L1 broadcasts.
+      {
+        const int cb = nt * BN + 8 * lane;
+        if (8 * lane < BN && cb < g.N) {
+          if (g.bias != nullptr) asm volatile("prefetch.global.L1 [%0];" ::"l"(g.bias + cb));
+          if (g.epi == EPI_RESID_GATE) asm volatile("prefetch.global.L1 [%0];" ::"l"(g.gate + cb));
+        }
+      }
       int ok = 1;
       if (lane == 0) ok = mbar_wait(su32(&accf[acc]), acc_phase, abort_flag, g.err, 4) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);  // the whole warp takes the same branch
@@ -194,59 +318,129 @@ __global__ void __launch_bounds__(192, 1)
       tc_fence_after();
       const int row_base = mt * BM + quarter * 32;
       const uint32_t tbase = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * BN);
-#pragma unroll 1
-      for (int c = 0; c < BN; c += cw) {
-        const int col0 = nt * BN + c;
-        if (row_base >= g.M || col0 >= g.N) continue;  // uniform across the warp
-        uint4 chunk[8];
-        if (bf16_out) {
-          uint32_t r0[32], r1[32];
-          tmem_ld32(tbase + (uint32_t)c, r0);
-          tmem_ld32(tbase + (uint32_t)(c + 32), r1);
-          const float4* b4 = reinterpret_cast<const float4*>(g.bias + col0);
-          const bool gelu = g.epi == EPI_GELU;
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            float v[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              const int i = 8 * j + e;
-              v[e] = __uint_as_float(i < 32 ? r0[i] : r1[i - 32]);
-            }
-            if (g.bias != nullptr && (j < 4 || col0 + 64 <= g.N)) {  // columns >= N are clipped
-              const float4 ba = b4[2 * j], bb = b4[2 * j + 1];
-              v[0] += ba.x; v[1] += ba.y; v[2] += ba.z; v[3] += ba.w;
-              v[4] += bb.x; v[5] += bb.y; v[6] += bb.z; v[7] += bb.w;
-            }
-            if (gelu) {
-#pragma unroll
-              for (int e = 0; e < 8; ++e) v[e] = gelu_tanh(v[e]);
-            }
-            chunk[j] = make_uint4(pack2(v[0], v[1]), pack2(v[2], v[3]), pack2(v[4], v[5]),
-                                  pack2(v[6], v[7]));
+      // Stream-K parts of this work tile: workers w_first .. w_first + nparts - 1 in k order.
+      int nparts = 1, part = 0, w_first = 0;
+      bool finish = true, staged = false;
+      // Partial-sum slot of part i (this CTA's rank): 2w for worker w's first
+      // segment, 2w+1 for its last.
+      auto slot_of = [&](int i) -> float4* {
+        const int wi = w_first + i;
+        const int first_tile = (int)(((int64_t)wi * U / workers) / nk);
+        const int s = 2 * wi + (first_tile == tile ? 0 : 1);
+        return reinterpret_cast<float4*>(sk.ws + (size_t)(s * CL + rank) * SLOT);
+      };
+      const int rowq = quarter * 32 + lane;  // this thread's row within the tile
+      if (kb0 != 0 || kb1 != nk) {
+        const int64_t tu = (int64_t)tile * nk;
+        w_first = sk_worker_of(tu, U, workers);
+        nparts = sk_worker_of(tu + nk - 1, U, workers) - w_first + 1;
+        part = worker - w_first;
+        if (nparts > SK_MAX_PARTS) {  // excluded by the host's choice of schedule
+          if (lane == 0) {
+            *abort_flag = 1;
+            atomicExch(g.err, 7);
           }
-        } else {
-          uint32_t r0[32];
-          tmem_ld32(tbase + (uint32_t)c, r0);
-          const float4* b4 = reinterpret_cast<const float4*>(g.bias + col0);
-          const float4* g4 = reinterpret_cast<const float4*>(g.gate + col0);
-          const bool gated = g.epi == EPI_RESID_GATE;
+          break;
+        }
+        int* cnt = sk.cnt + 4 * (tile * CL + rank) + quarter;
+        int last = 0;
+        if (lane == 0) last = ld_acquire(cnt) == nparts - 1 ? 1 : 0;
+        last = __shfl_sync(0xffffffffu, last, 0);
+        if (!last) {
+          // Publish this part: rows of this warp, 32-column chunks, chunk-major so
+          // that each store instruction of the warp covers 512 contiguous bytes.
+          float4* mine = slot_of(part);
+          if (row_base < g.M) {
+#pragma unroll 1
+            for (int c = 0; c < BN; c += 32) {
+              if (nt * BN + c >= g.N) break;
+              uint32_t r[32];
+              tmem_ld32(tbase + (uint32_t)c, r);
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            float4 v = make_float4(__uint_as_float(r0[4 * j]), __uint_as_float(r0[4 * j + 1]),
-                                   __uint_as_float(r0[4 * j + 2]), __uint_as_float(r0[4 * j + 3]));
-            if (g.bias != nullptr) {
-              const float4 b = b4[j];
-              v.x += b.x; v.y += b.y; v.z += b.z; v.w += b.w;
+              for (int j = 0; j < 8; ++j)
+                mine[((c >> 5) * 8 + j) * BM + rowq] =
+                    make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                                __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
             }
-            if (gated) {
-              const float4 gg = g4[j];
-              v.x *= gg.x; v.y *= gg.y; v.z *= gg.z; v.w *= gg.w;
+          }
+          __threadfence();
+          __syncwarp();
+          if (lane == 0) last = atomicAdd(cnt, 1) == nparts - 1 ? 1 : 0;
+          last = __shfl_sync(0xffffffffu, last, 0);
+        }
+        finish = last != 0;
+        if (finish) {
+          __threadfence();  // the other parts' stores are visible to this warp's loads
+          if (lane == 0) *cnt = 0;  // every part has counted in: reset for the next launch
+          // After the worker's last segment the operand stages are idle (every load
+          // was consumed by an MMA that has completed), so the one other part is
+          // copied into this warp's 32 KB of them in a single asynchronous batch.
+          if (final_seg && nparts == 2 && row_base < g.M) {
+            const float4* src = slot_of(1 - part) + rowq;
+            const uint32_t dst = su32(smem) + (uint32_t)(warp - 2) * 32768u + lane * 16u;
+            fence_async_shared();  // after the tensor core's reads of these stages
+#pragma unroll 1
+            for (int c = 0; c < BN; c += 32) {
+              if (nt * BN + c >= g.N) break;
+#pragma unroll
+              for (int j = 0; j < 8; ++j)
+                cp_async16(dst + (uint32_t)(((c >> 5) * 8 + j) * 512), src + ((c >> 5) * 8 + j) * BM);
             }
-            chunk[j] = make_uint4(__float_as_uint(v.x), __float_as_uint(v.y),
-                                  __float_as_uint(v.z), __float_as_uint(v.w));
+            cp_async_wait_all();
+            staged = true;
           }
         }
+      }
+      // Adds the other parts' columns c..c+31 of this thread's row to its own (in r),
+      // in k order: p_0 + p_1 + ... with this CTA's part at index `part` (fp32
+      // addition is commutative, so t + own and own + t are the same bits).  A
+      // part's eight loads are issued together: one memory latency per part.
+      auto combine32 = [&](int c, uint32_t (&r)[32]) {
+        float4 t[8];
+#pragma unroll 1
+        for (int i = 0; i < nparts; ++i) {
+          if (i == part) {
+            if (i > 0) {
+#pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                r[4 * j] = __float_as_uint(t[j].x + __uint_as_float(r[4 * j]));
+                r[4 * j + 1] = __float_as_uint(t[j].y + __uint_as_float(r[4 * j + 1]));
+                r[4 * j + 2] = __float_as_uint(t[j].z + __uint_as_float(r[4 * j + 2]));
+                r[4 * j + 3] = __float_as_uint(t[j].w + __uint_as_float(r[4 * j + 3]));
+              }
+            }
+            continue;
+          }
+          float4 x[8];
+          if (staged) {
+            const float4* src = reinterpret_cast<const float4*>(smem + (warp - 2) * 32768) +
+                                (c >> 5) * 8 * 32 + lane;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) x[j] = src[j * 32];
+          } else {
+            const float4* src = slot_of(i) + (c >> 5) * 8 * BM + rowq;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) x[j] = __ldcg(src + j * BM);
+          }
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            if (i < part) {  // running sum of the parts before this CTA's
+              if (i == 0) {
+                t[j] = x[j];
+              } else {
+                t[j].x += x[j].x; t[j].y += x[j].y; t[j].z += x[j].z; t[j].w += x[j].w;
+              }
+            } else {  // parts after this CTA's: add onto the running total in r
+              r[4 * j] = __float_as_uint(__uint_as_float(r[4 * j]) + x[j].x);
+              r[4 * j + 1] = __float_as_uint(__uint_as_float(r[4 * j + 1]) + x[j].y);
+              r[4 * j + 2] = __float_as_uint(__uint_as_float(r[4 * j + 2]) + x[j].z);
+              r[4 * j + 3] = __float_as_uint(__uint_as_float(r[4 * j + 3]) + x[j].w);
+            }
+          }
+        }
+      };
+      // Stages 32 rows x 128 bytes (this warp's box) and sends it with TMA.
+      auto send_box = [&](const uint4 (&chunk)[8], int col) {
         // The box written two stores ago must have been read out by its TMA.
         if (lane == 0) bulk_wait_read_1();
         __syncwarp();
@@ -255,11 +449,95 @@ __global__ void __launch_bounds__(192, 1)
         fence_async_shared();
         __syncwarp();
         if (lane == 0) {
-          if (bf16_out) tma_store_2d(&tmC, col0, row_base, su32(box));
-          else tma_reduce_add_2d(&tmC, col0, row_base, su32(box));
+          if (bf16_out) tma_store_2d(&tmC, col, row_base, su32(box));
+          else tma_reduce_add_2d(&tmC, col, row_base, su32(box));
           bulk_commit();
         }
         sb ^= 1;
+      };
+      // A split tile: add the other parts into this CTA's accumulator in TMEM first,
+      // so the epilogue below is the same for every tile.
+      if (finish && nparts > 1 && row_base < g.M) {
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          if (nt * BN + c >= g.N) break;
+          uint32_t r[32];
+          tmem_ld32(tbase + (uint32_t)c, r);
+          combine32(c, r);
+          tmem_st32(tbase + (uint32_t)c, r);
+        }
+        tmem_st_wait();
+      }
+      // 64 columns per step: both 32-column TMEM loads in flight under one wait.
+#pragma unroll 1
+      for (int c = 0; finish && c < BN; c += 64) {
+        const int col0 = nt * BN + c;
+        if (row_base >= g.M || col0 >= g.N) continue;  // uniform across the warp
+        const bool two = c + 32 < BN && col0 + 32 < g.N;  // second 32-column half present
+        // This step's bias (bf16 output) or bias and gate of the first half (fp32
+        // output), requested before the TMEM loads so the two latencies overlap.
+        float4 pb[8], pg[8];
+        if (g.bias != nullptr) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            pb[j] = __ldg(reinterpret_cast<const float4*>(g.bias + col0) + (bf16_out ? 2 * j : j));
+        }
+        if (!bf16_out && g.epi == EPI_RESID_GATE) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) pg[j] = __ldg(reinterpret_cast<const float4*>(g.gate + col0) + j);
+        }
+        uint32_t r0[32], r1[32];
+        tmem_ld32_nowait(tbase + (uint32_t)c, r0);
+        if (two) tmem_ld32_nowait(tbase + (uint32_t)(c + 32), r1);
+        tmem_ld_wait();
+        uint4 chunk[8];
+        if (bf16_out) {
+          const bool gelu = g.epi == EPI_GELU;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {  // columns c + 8j .. c + 8j + 7 (bias in lane c/8 + j)
+            float v[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) v[e] = __uint_as_float(j < 4 ? r0[8 * j + e] : r1[8 * j + e - 32]);
+            if (g.bias != nullptr) {
+              const float4 b0 = pb[j];  // columns c + 8j .. c + 8j + 3 (first four of eight)
+              const float4 b1 = __ldg(reinterpret_cast<const float4*>(g.bias + col0 + 8 * j + 4));
+              v[0] += b0.x; v[1] += b0.y; v[2] += b0.z; v[3] += b0.w;
+              v[4] += b1.x; v[5] += b1.y; v[6] += b1.z; v[7] += b1.w;
+            }
+            if (gelu) {
+#pragma unroll
+              for (int e = 0; e < 8; ++e) v[e] = gelu_tanh(v[e]);
+            }
+            chunk[j] = make_uint4(pack2(v[0], v[1]), pack2(v[2], v[3]), pack2(v[4], v[5]),
+                                  pack2(v[6], v[7]));
+          }
+          send_box(chunk, col0);  // columns >= N are clipped by the tensor map
+        } else {
+          const bool gated = g.epi == EPI_RESID_GATE;
+#pragma unroll
+          for (int hh = 0; hh < 2; ++hh) {
+            if (hh == 1 && !two) break;
+            const uint32_t* r = hh == 0 ? r0 : r1;
+            const int cc = c + 32 * hh;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              float4 v = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                                     __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+              const int cg = nt * BN + cc + 4 * j;  // columns cg .. cg + 3
+              if (g.bias != nullptr) {
+                const float4 b = hh == 0 ? pb[j] : __ldg(reinterpret_cast<const float4*>(g.bias + cg));
+                v.x += b.x; v.y += b.y; v.z += b.z; v.w += b.w;
+              }
+              if (gated) {
+                const float4 gg = hh == 0 ? pg[j] : __ldg(reinterpret_cast<const float4*>(g.gate + cg));
+                v.x *= gg.x; v.y *= gg.y; v.z *= gg.z; v.w *= gg.w;
+              }
+              chunk[j] = make_uint4(__float_as_uint(v.x), __float_as_uint(v.y),
+                                    __float_as_uint(v.z), __float_as_uint(v.w));
+            }
+            send_box(chunk, nt * BN + cc);
+          }
+        }
       }
       tc_fence_before();
       __syncwarp();
@@ -280,6 +558,8 @@ __global__ void __launch_bounds__(192, 1)
     __syncwarp();
     tmem_dealloc(tmem_base, S::TMEM_COLS);
   }
+  // Neither CTA of a cluster exits while the other may still signal its barriers.
+  if (CL > 1) cluster_sync();
 }
 
 // 2-D tensor map of a row-major [rows, cols] matrix with leading dimension ld
@@ -297,28 +577,162 @@ bool make_tmap(CUtensorMap* tm, CUtensorMapDataType dt, size_t esize, const void
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, int STAGES>
-cudaError_t launch_tc(const void* A, const void* W, const GemmArgs& g, cudaStream_t s) {
+// Stream-K counters and partial-sum slots, one set per (device, stream): GEMMs
+// on one stream run one after another, so they can share them.
+struct SkScratch {
+  int* cnt = nullptr;
+  size_t ncnt = 0;
+  float* ws = nullptr;
+  size_t nws = 0;
+};
+std::mutex g_sk_mu;
+std::map<std::pair<int, cudaStream_t>, SkScratch> g_sk;
+
+// Returns false (and leaves *out empty) if the buffers cannot be had.
+bool sk_scratch(cudaStream_t s, size_t ncnt, size_t nws, SkArgs* out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  std::lock_guard<std::mutex> lk(g_sk_mu);
+  SkScratch& sc = g_sk[std::make_pair(dev, s)];
+  if (sc.ncnt < ncnt || sc.nws < nws) {
+    if (cudaStreamSynchronize(s) != cudaSuccess) return false;
+    cudaFree(sc.cnt);
+    cudaFree(sc.ws);
+    sc = SkScratch();
+    const size_t nc = ncnt > 4096 ? ncnt : 4096, nw = nws;
+    if (cudaMalloc(&sc.cnt, nc * sizeof(int)) != cudaSuccess ||
+        cudaMalloc(&sc.ws, nw * sizeof(float)) != cudaSuccess ||
+        cudaMemsetAsync(sc.cnt, 0, nc * sizeof(int), s) != cudaSuccess) {
+      cudaGetLastError();
+      cudaFree(sc.cnt);
+      cudaFree(sc.ws);
+      sc = SkScratch();
+      return false;
+    }
+    sc.ncnt = nc;
+    sc.nws = nw;
+  }
+  out->cnt = sc.cnt;
+  out->ws = sc.ws;
+  return true;
+}
+
+// Concurrently resident workers (CTAs, or clusters of CL CTAs) of one kernel
+// instantiation on the current device, looked up once.
+template <int BN, int STAGES, int CL>
+int max_workers() {
+  static std::mutex mu;
+  static std::map<int, int> cache;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  std::lock_guard<std::mutex> lk(mu);
+  auto it = cache.find(dev);
+  if (it != cache.end()) return it->second;
+  int n = num_sms() / CL;
+  if (CL > 1 &&
+      cudaFuncSetAttribute(k_gemm_tc<BN, STAGES, CL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)TcShape<BN, STAGES>::SMEM) == cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(num_sms());
+    cfg.blockDim = dim3(192);
+    cfg.dynamicSmemBytes = TcShape<BN, STAGES>::SMEM;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CL;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int c = 0;
+    if (cudaOccupancyMaxActiveClusters(&c, k_gemm_tc<BN, STAGES, CL>, &cfg) == cudaSuccess && c > 0)
+      n = c;
+    cudaGetLastError();
+  }
+  cache[dev] = n;
+  return n;
+}
+
+template <int BN, int STAGES, int CL>
+cudaError_t launch_tc(const void* A, const void* W, const GemmArgs& g, bool stream_k,
+                      cudaStream_t s) {
   using S = TcShape<BN, STAGES>;
   static_assert(S::SMEM <= 232448, "shared memory budget");
   CUtensorMap ta, tb, tc;
   const CUtensorMapDataType BF = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
   if (!make_tmap(&ta, BF, 2, A, (uint64_t)g.M, (uint64_t)g.K, (uint64_t)g.K, BM, BK))
     return cudaErrorInvalidValue;
-  if (!make_tmap(&tb, BF, 2, W, (uint64_t)g.N, (uint64_t)g.K, (uint64_t)g.K, BN, BK))
+  if (!make_tmap(&tb, BF, 2, W, (uint64_t)g.N, (uint64_t)g.K, (uint64_t)g.K, BN / CL, BK))
     return cudaErrorInvalidValue;
   const bool bf16_out = g.epi == EPI_STORE || g.epi == EPI_GELU;
   if (bf16_out ? !make_tmap(&tc, BF, 2, g.out, (uint64_t)g.M, (uint64_t)g.N, (uint64_t)g.ldo, 32, 64)
                : !make_tmap(&tc, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, g.out, (uint64_t)g.M,
                             (uint64_t)g.N, (uint64_t)g.ldo, 32, 32))
     return cudaErrorInvalidValue;
-  cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN, STAGES>,
+  cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN, STAGES, CL>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)S::SMEM);
   if (e != cudaSuccess) return e;
-  const int tiles = ((g.M + BM - 1) / BM) * ((g.N + BN - 1) / BN);
-  const int grid = tiles < num_sms() ? tiles : num_sms();
+  const int m_units = ((g.M + BM - 1) / BM + CL - 1) / CL;
+  const int tiles = m_units * ((g.N + BN - 1) / BN);
+  const int wmax = max_workers<BN, STAGES, CL>();
+  int workers = tiles < wmax ? tiles : wmax;
+  SkArgs sk = {nullptr, nullptr, 0};
+  if (stream_k) {
+    sk.units = (int64_t)tiles * (g.K / BK);
+    if (sk_scratch(s, (size_t)4 * tiles * CL, (size_t)2 * wmax * CL * BM * BN, &sk))
+      workers = wmax;
+    else
+      sk = {nullptr, nullptr, 0};
+  }
   count_launch();
-  return launch_pdl(k_gemm_tc<BN, STAGES>, grid, 192, S::SMEM, s, ta, tb, tc, g);
+  if (CL == 1)
+    return launch_pdl(k_gemm_tc<BN, STAGES, CL>, workers, 192, S::SMEM, s, ta, tb, tc, g, sk);
+  return launch_pdl_cluster(k_gemm_tc<BN, STAGES, CL>, workers * CL, 192, S::SMEM, s, CL, ta, tb,
+                            tc, g, sk);
+}
+
+template <int CL>
+cudaError_t gemm_dispatch(const void* A, const void* W, const GemmArgs& g, int sched,
+                          cudaStream_t s) {
+  // Schedule and tile width by a makespan model: every worker of a wave runs
+  // concurrently, so a data-parallel launch costs about rounds x k-blocks x
+  // (BN + 150), the 150 columns' worth of per-k-block overhead fitted to
+  // measured tile times (a 192-wide tile takes about 0.85x the time of a
+  // 256-wide one).  Ties go to the wider tile.  Stream-K with 256-wide tiles
+  // costs the average number of work tiles per worker (fractional) times the
+  // same figure, plus SK_FIXUP; it is taken only when no tile spans more than
+  // SK_MAX_PARTS workers.
+  const int m_units = ((g.M + BM - 1) / BM + CL - 1) / CL;
+  const bool fp32_out = g.epi == EPI_RESID || g.epi == EPI_RESID_GATE;  // 32-column epilogue chunks
+  const long nk = g.K / BK;
+  int best_bn = 256;
+  long best_cost = -1;
+  for (int bn : {256, 192, 160, 128}) {
+    if (bn == 160 && !fp32_out) continue;  // bf16 epilogue chunks are 64 columns wide
+    const int wk = bn == 256   ? max_workers<256, 4, CL>()
+                   : bn == 192 ? max_workers<192, 4, CL>()
+                   : bn == 160 ? max_workers<160, 5, CL>()
+                               : max_workers<128, 6, CL>();
+    const long tiles = (long)m_units * ((g.N + bn - 1) / bn);
+    const long cost = ((tiles + wk - 1) / wk) * nk * (bn + 150);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best_bn = bn;
+    }
+  }
+  if (sched != 1) {
+    const int wk = max_workers<256, 4, CL>();
+    const long tiles = (long)m_units * ((g.N + 255) / 256);
+    const long units = tiles * nk, per_worker = units / wk;
+    const bool spans_ok =
+        per_worker > 0 && 1 + (nk - 1 + per_worker - 1) / per_worker <= SK_MAX_PARTS;
+    const double sk_cost = (double)tiles / wk * nk * (256 + 150) + SK_FIXUP;
+    if (spans_ok && (sched == 2 || (tiles > wk / 2 && sk_cost < (double)best_cost)))
+      return launch_tc<256, 4, CL>(A, W, g, true, s);
+  }
+  if (best_bn == 256) return launch_tc<256, 4, CL>(A, W, g, false, s);
+  if (best_bn == 192) return launch_tc<192, 4, CL>(A, W, g, false, s);
+  if (best_bn == 160) return launch_tc<160, 5, CL>(A, W, g, false, s);
+  return launch_tc<128, 6, CL>(A, W, g, false, s);
 }
 
 }  // namespace
@@ -336,6 +750,12 @@ EncodeTiledFn encode_tiled_fn() {
   return fn;
 }
 
+namespace {
+std::atomic<int> g_schedule{0};
+}
+
+void set_gemm_schedule(int mode) { g_schedule.store(mode); }
+
 cudaError_t gemm_bf16_tc(const void* A, const void* W, const GemmArgs& g, cudaStream_t s) {
   if (g.M <= 0 || g.N <= 0) return cudaSuccess;
   if (g.K <= 0 || g.K % BK != 0 || g.N % 32 != 0 || g.ldo % 8 != 0) return cudaErrorInvalidValue;
@@ -343,27 +763,10 @@ cudaError_t gemm_bf16_tc(const void* A, const void* W, const GemmArgs& g, cudaSt
   if (g.bias != nullptr && (((uintptr_t)g.bias) & 15)) return cudaErrorMisalignedAddress;
   if (g.epi == EPI_RESID_GATE && (g.gate == nullptr || (((uintptr_t)g.gate) & 15)))
     return cudaErrorInvalidValue;
-  // Tile width by a makespan model: every CTA of a wave runs concurrently, so a
-  // launch costs about rounds x (BN + per-tile overhead).  The overhead (150
-  // columns' worth) is fitted to measured tile times: a 192-wide tile takes about
-  // 0.85x the time of a 256-wide one.  Ties go to the wider tile.
-  const int m_tiles = (g.M + BM - 1) / BM, sms = num_sms();
-  const bool fp32_out = g.epi == EPI_RESID || g.epi == EPI_RESID_GATE;  // 32-column epilogue chunks
-  int best_bn = 256;
-  long best_cost = -1;
-  for (int bn : {256, 192, 160, 128}) {
-    if (bn == 160 && !fp32_out) continue;  // bf16 epilogue chunks are 64 columns wide
-    const long tiles = (long)m_tiles * ((g.N + bn - 1) / bn);
-    const long cost = ((tiles + sms - 1) / sms) * (bn + 150);
-    if (best_cost < 0 || cost < best_cost) {
-      best_cost = cost;
-      best_bn = bn;
-    }
-  }
-  if (best_bn == 256) return launch_tc<256, 4>(A, W, g, s);
-  if (best_bn == 192) return launch_tc<192, 4>(A, W, g, s);
-  if (best_bn == 160) return launch_tc<160, 5>(A, W, g, s);
-  return launch_tc<128, 6>(A, W, g, s);
+  // Clusters of two CTAs (shared W tile) on request, when there are two row tiles to pair.
+  const int mode = g_schedule.load();
+  if ((mode & 4) != 0 && g.M > BM) return gemm_dispatch<2>(A, W, g, mode & 3, s);
+  return gemm_dispatch<1>(A, W, g, mode & 3, s);
 }
 
 }  // namespace track

@@ -729,6 +729,14 @@ int track_sync(track_stream s) {
   return TRACK_OK;
 }
 
+int track_gemm_schedule(int mode) {
+  if ((mode & ~TRACK_GEMM_MULTICAST) < TRACK_GEMM_AUTO ||
+      (mode & ~TRACK_GEMM_MULTICAST) > TRACK_GEMM_STREAM_K)
+    return fail(TRACK_EINVAL, "unknown GEMM schedule");
+  set_gemm_schedule(mode);
+  return TRACK_OK;
+}
+
 int track_profile_enable(int enable) {
   g_prof_on.store(enable != 0);
   return TRACK_OK;

@@ -102,3 +102,13 @@ def test_equal_budget_policies_bit_exact(T):
                                       otrack.random_k_policy(n, k, seed))
     with pytest.raises(T.TrackError):
         T.track_policy_random_k(4, 5, 1)
+
+
+def test_gemm_schedule_modes(T):
+    for mode in (T.GEMM_DATA_PARALLEL, T.GEMM_STREAM_K, T.GEMM_AUTO | T.GEMM_MULTICAST,
+                 T.GEMM_STREAM_K | T.GEMM_MULTICAST, T.GEMM_AUTO):
+        T.track_gemm_schedule(mode)
+    for bad in (-1, 3, 7, 8):
+        with pytest.raises(T.TrackError) as e:
+            T.track_gemm_schedule(bad)
+        assert e.value.code == T.TRACK_EINVAL

@@ -82,6 +82,81 @@ def test_linear_bf16_tcgen05(T, M, N, K, epi):
         assert rel_l2(delta, want) < 2e-5
 
 
+# Stream-K forced where the shape allows it: a ragged 32-column last tile and
+# ragged rows (three CTAs per tile), the output projection at 3510 tokens (two),
+# wide N, and K = 4096 over 52 tiles, where a tile spans four CTAs.
+SK_SHAPES = [
+    (2000, 1568, 1536),
+    (3510, 1536, 1536),
+    (600, 8960, 1536),
+    (1664, 1024, 4096),
+]
+
+
+@pytest.fixture(params=["sk", "sk+multicast", "dp+multicast"])
+def schedule(T, request):
+    T.track_gemm_schedule({"sk": T.GEMM_STREAM_K,
+                           "sk+multicast": T.GEMM_STREAM_K | T.GEMM_MULTICAST,
+                           "dp+multicast": T.GEMM_DATA_PARALLEL | T.GEMM_MULTICAST}[request.param])
+    yield request.param
+    T.track_gemm_schedule(T.GEMM_AUTO)
+
+
+@pytest.mark.parametrize("M,N,K", SK_SHAPES)
+@pytest.mark.parametrize("epi", [0, 1, 2, 3])
+def test_linear_bf16_schedules(T, schedule, M, N, K, epi):
+    rng = np.random.default_rng(M * 5 + N + K * 3 + epi)
+    X = dit.round_bf16(rng.normal(size=(M, K)).astype(np.float32))
+    W = dit.round_bf16((rng.normal(size=(N, K)) / np.sqrt(K)).astype(np.float32))
+    b = rng.normal(size=N).astype(np.float32) * 0.1
+    gate = rng.normal(size=N).astype(np.float32)
+    ref = dit.linear(X, W, b)
+    if epi == T.EPI_GELU:
+        ref = dit.gelu_tanh(ref)
+    Xd, Wd, bd = dev_bf16(X), dev_bf16(W), dev_f32(b)
+    gd = dev_f32(gate) if epi == T.EPI_RESID_GATE else None
+    outs = []
+    for _ in range(2):  # twice: same bits (fixed summation order, counters reset)
+        if epi in (T.EPI_STORE, T.EPI_GELU):
+            out = torch.zeros((M, N), dtype=torch.bfloat16, device=DEV)
+        else:
+            r0 = rng.normal(size=(M, N)).astype(np.float32) if not outs else r0
+            out = dev_f32(r0)
+        T.track_linear(T.BF16, Xd, Wd, bd, epi, out, gate=gd)
+        T.track_sync()
+        outs.append(out.float().cpu().numpy())
+    assert np.array_equal(outs[0], outs[1])
+    if epi in (T.EPI_STORE, T.EPI_GELU):
+        got = outs[0]
+        assert rel_l2(got, ref) < 4e-3
+        assert np.all(np.abs(got - ref) <= 8e-3 * np.abs(ref) + 2e-3 * np.sqrt(np.mean(ref ** 2)))
+    else:
+        delta = outs[0].astype(np.float64) - r0
+        want = ref * gate if epi == T.EPI_RESID_GATE else ref
+        assert rel_l2(delta, want) < 2e-5
+
+
+def test_linear_bf16_schedules_agree(T):
+    # Stream-K differs from data-parallel only in the order of fp32 partial sums;
+    # multicast under data-parallel changes no bit.
+    rng = np.random.default_rng(11)
+    M, N, K = 3510, 1536, 8960
+    X = dev_bf16(rng.normal(size=(M, K)).astype(np.float32))
+    W = dev_bf16((rng.normal(size=(N, K)) / np.sqrt(K)).astype(np.float32))
+    res = []
+    for mode in (T.GEMM_DATA_PARALLEL, T.GEMM_STREAM_K, T.GEMM_DATA_PARALLEL | T.GEMM_MULTICAST):
+        T.track_gemm_schedule(mode)
+        out = torch.zeros((M, N), dtype=torch.float32, device=DEV)
+        T.track_linear(T.BF16, X, W, None, T.EPI_RESID, out)
+        T.track_sync()
+        res.append(out.cpu().numpy().astype(np.float64))
+    T.track_gemm_schedule(T.GEMM_AUTO)
+    assert np.array_equal(res[2], res[0])
+    # Two fp32 sums of K terms in different association differ by about
+    # sqrt(K) * 2^-24 relative (6e-6 at K = 8960); the bound allows 3x that.
+    assert rel_l2(res[1], res[0]) < 2e-5
+
+
 @pytest.mark.parametrize("M,N,K", [(1, 32, 64), (100, 96, 80), (513, 700, 256)])
 @pytest.mark.parametrize("epi", [0, 1, 2, 3])
 def test_linear_fp32(T, M, N, K, epi):
@@ -122,8 +197,8 @@ ATTN_CASES = [  # S, H, Lq, Lk, hd
     (1, 2, 257, 32, 64),       # short keys (tiny cross-attention)
     (2, 2, 300, 512, 128),     # cross-attention at text length 512
     (1, 12, 3510, 3510, 128),  # mid-size self-attention (bench shape)
-    (4, 16, 1000, 700, 128),   # two query tiles per CTA: ragged queries and keys
-    (2, 40, 600, 512, 64),     # two query tiles per CTA, hd 64, text-length keys
+    (4, 16, 1000, 700, 128),   # ragged queries and keys, last key tile under half full
+    (2, 40, 600, 512, 64),     # hd 64, text-length keys
 ]
 
 
@@ -162,6 +237,23 @@ def test_attention_fp32(T, S, H, Lq, Lk, hd):
     T.track_attention(T.FP32, dev_f32(Q), dev_f32(K), dev_f32(V), O)
     T.track_sync()
     assert rel_l2(O.cpu().numpy(), _attn_ref(Q, K, V)) < 2e-6
+
+
+@pytest.mark.parametrize("hd", [64, 128])
+def test_attention_growing_logits(T, hd):
+    # Key norms grow along the sequence and queries are scaled up, so each half
+    # of every key tile raises the running row maximum by far more than the
+    # lazy-rescaling threshold many times over: every O rescale path runs.
+    rng = np.random.default_rng(hd + 7)
+    S, H, Lq, Lk = 1, 3, 200, 900
+    ramp = (1.0 + 4.0 * np.arange(Lk) / Lk)[None, None, :, None]
+    Q = dit.round_bf16((4.0 * rng.normal(size=(S, H, Lq, hd))).astype(np.float32))
+    K = dit.round_bf16((ramp * rng.normal(size=(S, H, Lk, hd))).astype(np.float32))
+    V = dit.round_bf16(rng.normal(size=(S, H, Lk, hd)).astype(np.float32))
+    O = torch.zeros((S, Lq, H, hd), dtype=torch.bfloat16, device=DEV)
+    T.track_attention(T.BF16, dev_bf16(Q), dev_bf16(K), dev_bf16(V), O)
+    T.track_sync()
+    assert rel_l2(O.float().cpu().numpy(), _attn_ref(Q, K, V)) < 1e-2
 
 
 def test_attention_single_key_returns_value_row(T):
