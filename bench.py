@@ -439,7 +439,7 @@ def run_ours(args):
     traffic, traffic_src = measured_traffic("k_gemm_tc" if dominant == "gemm" else "k_attn_tc",
                                             dflops / dn if dn else 0.0)
     roof = {"bound": "tensor", "kernel": "bf16 GEMM (tcgen05)" if dominant == "gemm"
-            else "flash attention (bf16 mma.sync)",
+            else "flash attention (tcgen05)",
             "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
             "frac": achieved / peak if achieved else None, "traffic": traffic,
             "traffic_unit": "bytes per launch", "traffic_source": traffic_src,
