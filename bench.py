@@ -295,6 +295,7 @@ def run_ours(args):
         tdist.init_process_group("nccl")
     _build.build()
     T.track_gemm_schedule(GEMM_SCHEDULES[args.gemm_schedule])
+    T.track_attention_schedule(GEMM_SCHEDULES[args.attn_schedule])
 
     wl = synth.WORKLOADS[WORKLOAD]
     B = wl.batch
@@ -502,7 +503,7 @@ def run_ours(args):
 
 
 # ---------------------------------------------------------------- single kernels
-GEMM_SCHEDULES = {"auto": 0, "dp": 1, "sk": 2}   # track_gemm_schedule modes
+GEMM_SCHEDULES = {"auto": 0, "dp": 1, "sk": 2}   # track_gemm/attention_schedule modes
 
 
 def run_kernel(args):
@@ -516,6 +517,7 @@ def run_kernel(args):
     _build.build()
     torch.cuda.set_device(0)
     T.track_gemm_schedule(GEMM_SCHEDULES[args.gemm_schedule])
+    T.track_attention_schedule(GEMM_SCHEDULES[args.attn_schedule])
     wl = synth.WORKLOADS[WORKLOAD]
     a = wl.large
     M = args.batch * a.tokens
@@ -599,6 +601,8 @@ def main():
     ap.add_argument("--batch", type=int, default=1, help="sequences for --kernel")
     ap.add_argument("--gemm-schedule", choices=["auto", "dp", "sk"], default="auto",
                     help="bf16 GEMM schedule: makespan model, data-parallel or stream-K")
+    ap.add_argument("--attn-schedule", choices=["auto", "dp", "sk"], default="auto",
+                    help="bf16 attention schedule: makespan model, data-parallel or stream-K")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)     # at least three untimed warm-up steps
     if args.impl == "reference":

@@ -266,6 +266,18 @@ int track_linear(int dtype, const void* X, const void* W, const float* bias, int
 #define TRACK_GEMM_MULTICAST 4
 int track_gemm_schedule(int mode);
 
+/* Schedule of the TRACK_BF16 attention kernel (process-wide), with the mode
+ * values of track_gemm_schedule (no multicast).  The kernel is persistent, at
+ * most one CTA per SM.  TRACK_GEMM_DATA_PARALLEL gives each CTA whole
+ * 128-query tiles of one (sequence, head); TRACK_GEMM_STREAM_K shares the
+ * tiles' 128-key blocks out evenly over one CTA per SM.  It is used wherever
+ * no query tile would span more than 4 CTAs.  A split query tile is finished
+ * by the last of its CTAs, which combines the parts' row maxima, row sums and
+ * unnormalized outputs in key order.  TRACK_GEMM_AUTO (the default) picks per
+ * launch by a makespan model.  Each schedule is deterministic; the two differ
+ * in fp32 rounding only.  EINVAL for any other mode. */
+int track_attention_schedule(int mode);
+
 /* O = softmax(Q K^T / sqrt(hd)) V per (sequence, head), no mask.  Q: [S, H, Lq,
  * hd], K, V: [S, H, Lk, hd], O: [S, Lq, H, hd], all in dtype (bf16 or fp32);
  * hd in {64, 128}. */

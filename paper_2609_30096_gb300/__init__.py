@@ -59,6 +59,7 @@ def lib():
         "track_launch_count": (_L, []),
         "track_profile_enable": (_I, [_I]),
         "track_gemm_schedule": (_I, [_I]),
+        "track_attention_schedule": (_I, [_I]),
         "track_profile_read": (_I, [_P, _P, _P]),
         "track_weight_count": (_I, [_P]),
         "track_weight_shape": (_I, [_P, _I, _P, _P]),
@@ -146,6 +147,11 @@ def track_gemm_schedule(mode: int):
     """GEMM_AUTO, GEMM_DATA_PARALLEL or GEMM_STREAM_K (optionally | GEMM_MULTICAST)
     for every later bf16 GEMM."""
     _check(lib().track_gemm_schedule(int(mode)))
+
+
+def track_attention_schedule(mode: int):
+    """GEMM_AUTO, GEMM_DATA_PARALLEL or GEMM_STREAM_K for every later bf16 attention."""
+    _check(lib().track_attention_schedule(int(mode)))
 
 
 def track_profile_enable(enable: bool):

@@ -1,34 +1,50 @@
 // Flash attention on the sm_103a tensor cores (bf16 in, fp32 accumulate):
 // O = softmax(Q K^T / sqrt(hd)) V per (sequence, head), no mask.
 //
-// One CTA per 128-query tile of one (sequence, head), 192 threads:
-//   warp 0      TMA: the Q tile once, then K and V tiles of 128 keys, K through
-//               a three-stage ring (lane 0) and V through a two-stage ring
-//               (lane 1); 4-D tensor maps over head-major or token-major
-//               operands, 128-byte swizzle, zero fill past L.  A K stage is
-//               released as soon as S = Q K^T of its tile completes.
-//   warp 1      allocates TMEM (O: hd columns; S: two 128-column buffers) and
-//               issues, from one thread, S(j+1) = Q K(j+1)^T while the softmax
-//               warps work on S(j), then O += P(j) V(j) once P(j) is ready.  P
-//               is read from TMEM (the A operand of the MMA), V is the MN-major
-//               B operand from shared memory, so no transposed copy is needed.
-//   warps 2-9   softmax, two warpgroups splitting each 128-key tile by columns
-//               (64 keys each), one thread per query row (its TMEM lane): row
+// Work: an item is one 128-query tile of one (sequence, head); its KT key tiles
+// of 128 keys are its units.  The kernel is persistent (at most one CTA per SM)
+// and follows one of two schedules:
+//   data-parallel  CTA w takes items w, w + G, ... with all their key tiles;
+//   stream-K       the items' key tiles form one sequence of U units and CTA w
+//                  takes the contiguous share [w U / G, (w+1) U / G), so every
+//                  SM processes the same number of key tiles whatever the item
+//                  count.  A query tile split across CTAs is finished by
+//                  whichever part ends last: the others publish their running
+//                  row maximum m, row sum l and unnormalized O (fp32) to a
+//                  workspace slot and count in on a per-(item, warp) counter;
+//                  the last one combines the parts in key order,
+//                  O = sum_p 2^(m_p - M) O_p / sum_p 2^(m_p - M) l_p with
+//                  M = max_p m_p (a fixed order: the bits do not depend on
+//                  timing), writes the output and resets the counter.
+// A CTA walks its segments (item, first key tile, end key tile) with 320
+// threads:
+//   warp 0      TMA: lane 0 the Q tile of each segment (two buffers) and the K
+//               tiles (three-stage ring), lane 1 the V tiles (two-stage ring);
+//               4-D tensor maps over head-major or token-major operands,
+//               128-byte swizzle, zero fill past L.
+//   warp 1      allocates TMEM (two O accumulators of hd columns, two
+//               128-column S buffers) and issues, from one thread,
+//               S(j+1) = Q K(j+1)^T (possibly the next segment's first tile)
+//               while the softmax warps work on S(j), then O += P(j) V(j)
+//               into the segment's O buffer.  P is read from TMEM (the A
+//               operand), V is the MN-major B operand from shared memory.
+//   warps 2-9   softmax, two warpgroups splitting each key tile by columns (64
+//               keys each), one thread per query row (its TMEM lane): row
 //               maximum over the valid keys (halves combined through shared
 //               memory), lazy rescaling of O (only when the running maximum
-//               grows by more than 2^8; each group rescales its half of O's
-//               columns in TMEM, after P V of the previous tile completes),
-//               P = exp2(S * log2(e)/sqrt(hd) - m) rounded to bf16 pairs and
-//               written over the first 32 of the group's 64 S columns, and at
-//               the end O / l stored to the token-major output.  Because P
-//               lives in the S buffer it came from, the softmax of tile j+1
-//               never waits for P V of tile j unless it must rescale O.
+//               grows by more than 2^8), P = exp2(S log2(e)/sqrt(hd) - m)
+//               rounded to bf16 pairs and written over the first 32 of the
+//               group's 64 S columns, and at the end of a segment the output
+//               (or the stream-K publish / combine).  O is double-buffered, so
+//               the next segment's MMAs run while a segment's output is read.
 // Tensor-core operations issued by one thread execute in issue order, so
 // S(j+2), issued after O += P(j) V(j), overwrites P(j) only after it was read.
 // Every mbarrier wait is bounded (see tc_common.cuh).
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <math.h>
+
+#include <atomic>
 
 #include "internal.h"
 #include "tc_common.cuh"
@@ -40,20 +56,34 @@ namespace {
 using namespace tc;
 typedef __nv_bfloat16 bf16;
 
-constexpr int AT_BM = 128;       // query rows per CTA (MMA M)
-constexpr int AT_BN = 128;       // keys per tile
-constexpr int AT_THREADS = 320;  // warp 0 TMA, warp 1 MMA, warps 2-9 softmax
-constexpr uint32_t TM_S0 = 128;  // TMEM column of S buffer 0 (buffer 1 at 256)
+constexpr int AT_BM = 128;        // query rows per item (MMA M)
+constexpr int AT_BN = 128;        // keys per tile
+constexpr int AT_KH = AT_BN / 2;  // keys per softmax group
+constexpr int AT_THREADS = 320;   // warp 0 TMA, warp 1 MMA, warps 2-9 softmax
+constexpr int AT_MAX_PARTS = 4;   // the host only picks stream-K when no item spans more CTAs
 
 template <int HD>
 struct AtShape {
   static constexpr uint32_t Q_BYTES = AT_BM * HD * 2;   // HD/64 boxes of [128 rows][128 B]
   static constexpr uint32_t KV_BYTES = AT_BN * HD * 2;  // one K or V tile
   static constexpr uint32_t X_BYTES = 2 * 2 * AT_BM * 4;  // row partials [parity][half][row]
-  static constexpr int KST = 3;  // K ring stages
-  static constexpr int VST = 2;  // V ring stages
-  static constexpr size_t SMEM = 1024 + Q_BYTES + (KST + VST) * KV_BYTES + X_BYTES + 256;
+  static constexpr int KST = 3;  // K ring stages (V: 2)
+  // The dynamic shared window starts 1024-byte aligned (after the reserved
+  // 1 KB); the kernel checks that before its first copy.
+  static constexpr size_t SMEM = 2 * Q_BYTES + (KST + 2) * (size_t)KV_BYTES + X_BYTES + 256;
+  // TMEM columns: O buffer b at b*HD, S buffer b at TM_S0 + 128 b
+  static constexpr uint32_t TM_S0 = 2 * HD;
   static constexpr uint32_t TMEM_COLS = 512;
+  static_assert(TM_S0 + 2 * AT_BN <= TMEM_COLS, "TMEM budget");
+  // Stream-K slot: per softmax warp, its 32 rows x HD/2 columns of O (float4
+  // index (w * HD/8 + j) * 32 + lane), then per warp m[32] and l[32].
+  static constexpr int SLOT = AT_BM * HD + 8 * 2 * 32;
+};
+
+struct AtSk {
+  int* cnt;       // [8 * items] counters, zero between launches (nullptr: data-parallel)
+  float* ws;      // [2 * G] slots
+  int64_t units;  // items * key tiles
 };
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
@@ -78,49 +108,201 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
   return __shfl_sync(0xffffffffu, ok, 0) != 0;
 }
 
+// Output of a segment's query tile, by one softmax warp (its 32 rows, columns
+// half*HD/2 ..): O / l for a whole item; for a stream-K part, publish (m, l, O)
+// or, as the last part, combine all parts in key order.  tO addresses this
+// warp's lanes and columns of the segment's O buffer.  False if the item
+// spans more CTAs than the kernel supports (excluded by the host).
+template <int HD>
+__device__ __noinline__ bool segment_output(uint32_t tO, float m, float lt, int item, int kt0,
+                                            int kt1, int KT, int QT, int H, int Lq, int64_t U,
+                                            bf16* __restrict__ O, int half, int row, int lane,
+                                            int wi, const AtSk& sk, int* err,
+                                            volatile int* abort_flag) {
+  using S = AtShape<HD>;
+  // Writes 32 output columns (row-normalized by inv) of this thread's row.
+  auto store32 = [&](bf16* dst, const float (&v)[32], float inv) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      uint4 u;
+      u.x = pack_bf16x2(v[8 * j] * inv, v[8 * j + 1] * inv);
+      u.y = pack_bf16x2(v[8 * j + 2] * inv, v[8 * j + 3] * inv);
+      u.z = pack_bf16x2(v[8 * j + 4] * inv, v[8 * j + 5] * inv);
+      u.w = pack_bf16x2(v[8 * j + 6] * inv, v[8 * j + 7] * inv);
+      *reinterpret_cast<uint4*>(dst + 8 * j) = u;
+    }
+  };
+  const int bh = item / QT, sq = bh / H, hq = bh % H;
+  const int qrow = (item % QT) * AT_BM + row;
+  bf16* orow = O + (((int64_t)sq * Lq + qrow) * H + hq) * HD + half * (HD / 2);
+  if (kt0 == 0 && kt1 == KT) {
+    // The whole item: O / l.
+    const float inv = 1.f / lt;
+#pragma unroll 1
+    for (int cc = 0; cc < HD / 64; ++cc) {
+      uint32_t r[32];
+      tmem_ld32(tO + cc * 32, r);
+      float v[32];
+#pragma unroll
+      for (int t = 0; t < 32; ++t) v[t] = __uint_as_float(r[t]);
+      if (qrow < Lq) store32(orow + cc * 32, v, inv);
+    }
+  } else {
+    // Stream-K part of an item split across CTAs.
+    const int64_t iu = (int64_t)item * KT;
+    const int w_first = sk_worker_of(iu, U, gridDim.x);
+    const int nparts = sk_worker_of(iu + KT - 1, U, gridDim.x) - w_first + 1;
+    const int part = (int)blockIdx.x - w_first;
+    if (nparts > AT_MAX_PARTS) {  // excluded by the host's choice of schedule
+      if (lane == 0) {
+        *abort_flag = 1;
+        atomicExch(err, 24);
+      }
+      return false;
+    }
+    // Slot of part i: 2w for worker w's first segment, 2w+1 for its last.
+    auto slot_of = [&](int i) -> float* {
+      const int wk = w_first + i;
+      const int first_item = (int)(((int64_t)wk * U / gridDim.x) / KT);
+      return sk.ws + (size_t)(2 * wk + (first_item == item ? 0 : 1)) * S::SLOT;
+    };
+    int* cnt = sk.cnt + 8 * item + wi;
+    int last = 0;
+    if (lane == 0) last = ld_acquire(cnt) == nparts - 1 ? 1 : 0;
+    last = __shfl_sync(0xffffffffu, last, 0);
+    if (!last) {
+      // Publish m, l and this warp's 32 rows x HD/2 columns of O.
+      float* mine = slot_of(part);
+      float4* o4 = reinterpret_cast<float4*>(mine) + (size_t)wi * (HD / 8) * 32 + lane;
+#pragma unroll 1
+      for (int cc = 0; cc < HD / 64; ++cc) {
+        uint32_t r[32];
+        tmem_ld32(tO + cc * 32, r);
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          o4[(cc * 8 + j) * 32] =
+              make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                          __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+      }
+      float* ml = mine + AT_BM * HD + wi * 64;
+      ml[lane] = m;
+      ml[32 + lane] = lt;
+      __threadfence();
+      __syncwarp();
+      if (lane == 0) last = atomicAdd(cnt, 1) == nparts - 1 ? 1 : 0;
+      last = __shfl_sync(0xffffffffu, last, 0);
+    }
+    if (last) {
+      __threadfence();  // the other parts' stores are visible to this warp's loads
+      if (lane == 0) *cnt = 0;  // every part has counted in: reset for the next launch
+      // Weights 2^(m_p - M) and the combined row sum, parts in key order.
+      float wp[AT_MAX_PARTS], lp[AT_MAX_PARTS];
+      float M = m;
+#pragma unroll
+      for (int i = 0; i < AT_MAX_PARTS; ++i) {
+        wp[i] = -INFINITY;
+        lp[i] = 0.f;
+        if (i < nparts) {
+          if (i == part) {
+            wp[i] = m;
+            lp[i] = lt;
+          } else {
+            const float* ml = slot_of(i) + AT_BM * HD + wi * 64;
+            wp[i] = __ldcg(ml + lane);
+            lp[i] = __ldcg(ml + 32 + lane);
+          }
+          M = fmaxf(M, wp[i]);
+        }
+      }
+      float den = 0.f;
+#pragma unroll
+      for (int i = 0; i < AT_MAX_PARTS; ++i) {
+        wp[i] = i < nparts ? exp2_approx(wp[i] - M) : 0.f;
+        den = fmaf(wp[i], lp[i], den);
+      }
+      const float inv = 1.f / den;
+#pragma unroll 1
+      for (int cc = 0; cc < HD / 64; ++cc) {
+        uint32_t r[32];
+        tmem_ld32(tO + cc * 32, r);
+        float acc[32];
+#pragma unroll
+        for (int t = 0; t < 32; ++t) acc[t] = 0.f;
+#pragma unroll
+        for (int i = 0; i < AT_MAX_PARTS; ++i) {
+          if (i >= nparts) break;
+          float x[32];
+          if (i == part) {
+#pragma unroll
+            for (int t = 0; t < 32; ++t) x[t] = __uint_as_float(r[t]);
+          } else {
+            const float4* src = reinterpret_cast<const float4*>(slot_of(i)) +
+                                (size_t)wi * (HD / 8) * 32 + lane;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const float4 q = __ldcg(src + (cc * 8 + j) * 32);
+              x[4 * j] = q.x; x[4 * j + 1] = q.y; x[4 * j + 2] = q.z; x[4 * j + 3] = q.w;
+            }
+          }
+#pragma unroll
+          for (int t = 0; t < 32; ++t) acc[t] = fmaf(wp[i], x[t], acc[t]);
+        }
+        if (qrow < Lq) store32(orow + cc * 32, acc, inv);
+      }
+    }
+  }
+  return true;
+}
+
 template <int HD>
 __global__ void __launch_bounds__(AT_THREADS, 1)
     k_attn_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
               const __grid_constant__ CUtensorMap tmV, bf16* __restrict__ O, int H, int Lq, int Lk,
-              float scale_log2, int q_tok, int kv_tok, int* err) {
+              float scale_log2, int q_tok, int kv_tok, int* err, int items, const AtSk sk) {
   using S = AtShape<HD>;
   constexpr int NB = HD / 64;  // 64-column boxes per row of Q/K/V
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* sQ = smem;
-  uint8_t* sK = sQ + S::Q_BYTES;
-  uint8_t* sV = sK + S::KST * S::KV_BYTES;
-  float* xch = (float*)(sV + S::VST * S::KV_BYTES);  // [2][2][AT_BM] partial row maxima / sums
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = smem_raw;
+  uint8_t* sQ = smem;                         // [2] Q buffers
+  uint8_t* sK = sQ + 2 * S::Q_BYTES;          // [3] K stages
+  uint8_t* sV = sK + S::KST * S::KV_BYTES;    // [2] V stages
+  float* xch = (float*)(sV + 2 * S::KV_BYTES);  // [2][2][AT_BM] row partials
   uint64_t* bars = (uint64_t*)((uint8_t*)xch + S::X_BYTES);
-  uint64_t* q_full = bars;
-  uint64_t* k_full = bars + 1;    // [3] per K stage
-  uint64_t* k_empty = bars + 4;   // [3] freed once S = Q K^T of the tile has completed
-  uint64_t* v_full = bars + 7;    // [2] per V stage
-  uint64_t* v_empty = bars + 9;   // [2] freed once P V of the tile has completed
-  uint64_t* s_full = bars + 11;   // [2] per S buffer
-  uint64_t* p_full = bars + 13;   // [2] P of the tile written into its S buffer (8 softmax warps)
-  uint64_t* o_done = bars + 15;   // P V of the tile has completed
-  uint64_t* xbar = bars + 16;     // [2] both halves' row partials written (per parity)
-  uint64_t* done = bars + 18;     // every MMA of the CTA has completed
-  uint32_t* tmem_slot = (uint32_t*)(bars + 19);
+  uint64_t* q_full = bars;        // [2] per Q buffer
+  uint64_t* q_empty = bars + 2;   // [2] freed once the segment's last S MMA completed
+  uint64_t* k_full = bars + 4;    // [3] per K stage
+  uint64_t* k_empty = bars + 7;   // [3] freed once S = Q K^T of the tile has completed
+  uint64_t* v_full = bars + 10;   // [2] per V stage
+  uint64_t* v_empty = bars + 12;  // [2] freed once P V of the tile has completed
+  uint64_t* s_full = bars + 14;   // [2] per S buffer
+  uint64_t* p_full = bars + 16;   // [2] P of the tile written into its S buffer (8 softmax warps)
+  uint64_t* o_done = bars + 18;   // P V of the tile has completed
+  uint64_t* o_full = bars + 19;   // [2] every P V of the segment in this O buffer has completed
+  uint64_t* o_empty = bars + 21;  // [2] the segment's output was read out of this O buffer (8 warps)
+  uint64_t* xbar = bars + 23;     // [2] all 8 softmax warps' row partials written (per parity)
+  uint64_t* done = bars + 25;     // every MMA of the CTA has completed
+  uint32_t* tmem_slot = (uint32_t*)(bars + 26);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int bh = blockIdx.y, q0 = blockIdx.x * AT_BM;
-  const int sq = bh / H, hq = bh % H;
-  const int nkt = (Lk + AT_BN - 1) / AT_BN;
+  const int QT = (Lq + AT_BM - 1) / AT_BM, KT = (Lk + AT_BN - 1) / AT_BN;
+  const bool use_sk = sk.cnt != nullptr;
+  const int64_t U = use_sk ? sk.units : (int64_t)items * KT;
 
   if (threadIdx.x == 0) {
-    mbar_init(su32(q_full), 1);
     for (int i = 0; i < S::KST; ++i) {
       mbar_init(su32(&k_full[i]), 1);
       mbar_init(su32(&k_empty[i]), 1);
     }
     for (int i = 0; i < 2; ++i) {
+      mbar_init(su32(&q_full[i]), 1);
+      mbar_init(su32(&q_empty[i]), 1);
       mbar_init(su32(&v_full[i]), 1);
       mbar_init(su32(&v_empty[i]), 1);
       mbar_init(su32(&s_full[i]), 1);
       mbar_init(su32(&p_full[i]), 8);
+      mbar_init(su32(&o_full[i]), 1);
+      mbar_init(su32(&o_empty[i]), 8);
       mbar_init(su32(&xbar[i]), 8);
     }
     mbar_init(su32(o_done), 1);
@@ -136,9 +318,15 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   // The prologue above overlaps the previous kernel; inputs and outputs are touched only now.
   pdl_wait();
   pdl_release();
+  if ((su32(smem) & 1023u) != 0) {  // the 128-byte-swizzled tiles need 1024-byte alignment
+    if (threadIdx.x == 0) atomicExch(err, 25);
+    __syncthreads();
+    if (warp == 1) tmem_dealloc(tmem_base, S::TMEM_COLS);
+    return;
+  }
 
   if (warp == 0) {
-    // lane 0 streams Q and the K tiles, lane 1 the V tiles, each through its own ring
+    // lane 0 streams the Q tiles and the K tiles, lane 1 the V tiles
     if (lane < 2) {
       const bool kside = lane == 0;
       const CUtensorMap* tm = kside ? &tmK : &tmV;
@@ -146,201 +334,244 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       uint64_t* full = kside ? k_full : v_full;
       uint64_t* empty = kside ? k_empty : v_empty;
       asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)tm) : "memory");
-      if (kside) {
-        asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmQ) : "memory");
-        mbar_expect_tx(su32(q_full), S::Q_BYTES);
-        for (int b = 0; b < NB; ++b)
-          tma_load_rows(su32(sQ + b * AT_BM * 128), &tmQ, q_tok, b * 64, q0, hq, sq, su32(q_full));
-      }
-      const int nst = kside ? S::KST : S::VST;
-      uint32_t armed[S::KST] = {};
-      for (int kt = 0; kt < nkt; ++kt) {
-        const int st = kt % nst;
-        if (!mbar_wait(su32(&empty[st]), ((kt / nst) & 1) ^ 1, abort_flag, err, 11)) break;
-        mbar_expect_tx(su32(&full[st]), S::KV_BYTES);
-        for (int b = 0; b < NB; ++b)
-          tma_load_rows(su32(ring + st * S::KV_BYTES + b * AT_BN * 128), tm, kv_tok, b * 64,
-                        kt * AT_BN, hq, sq, su32(&full[st]));
-        ++armed[st];
+      if (kside) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmQ) : "memory");
+      const int nst = kside ? S::KST : 2;
+      uint32_t armed[S::KST] = {}, q_armed[2] = {0, 0};
+      SegIter it(use_sk, U, items, KT, blockIdx.x, gridDim.x);
+      int item, kt0, kt1;
+      int g = 0, si = 0;
+      bool ok = true;
+      while (ok && it.next(item, kt0, kt1)) {
+        const int bh = item / QT, sq = bh / H, hq = bh % H;
+        if (kside) {
+          const int qb = si & 1;
+          if (!mbar_wait(su32(&q_empty[qb]), ((si >> 1) & 1) ^ 1, abort_flag, err, 10)) break;
+          mbar_expect_tx(su32(&q_full[qb]), S::Q_BYTES);
+          const int q0 = (item % QT) * AT_BM;
+          for (int b = 0; b < NB; ++b)
+            tma_load_rows(su32(sQ + qb * S::Q_BYTES + b * AT_BM * 128), &tmQ, q_tok, b * 64, q0, hq,
+                          sq, su32(&q_full[qb]));
+          ++q_armed[qb];
+        }
+        for (int kt = kt0; kt < kt1; ++kt, ++g) {
+          const int st = g % nst;
+          if (!mbar_wait(su32(&empty[st]), ((g / nst) & 1) ^ 1, abort_flag, err, 11)) {
+            ok = false;
+            break;
+          }
+          mbar_expect_tx(su32(&full[st]), S::KV_BYTES);
+          for (int b = 0; b < NB; ++b)
+            tma_load_rows(su32(ring + st * S::KV_BYTES + b * AT_BN * 128), tm, kv_tok, b * 64,
+                          kt * AT_BN, hq, sq, su32(&full[st]));
+          ++armed[st];
+        }
+        ++si;
       }
       // Every copy this thread issued has landed before the CTA may exit.
-      if (kside) mbar_drain(su32(q_full), 0, err, 15);
       for (int i = 0; i < nst; ++i)
         if (armed[i] != 0) mbar_drain(su32(&full[i]), (armed[i] - 1) & 1, err, 15);
+      for (int i = 0; i < 2; ++i)
+        if (q_armed[i] != 0) mbar_drain(su32(&q_full[i]), (q_armed[i] - 1) & 1, err, 15);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idS = idesc_bf16(AT_BM, AT_BN);
       constexpr uint32_t idO = idesc_bf16_bmn(AT_BM, HD);
-      const uint32_t qa = su32(sQ);
-      auto issue_s = [&](int kt) -> bool {
-        const int st = kt % S::KST;
-        if (!mbar_wait(su32(&k_full[st]), (kt / S::KST) & 1, abort_flag, err, 12)) return false;
+      // S(g) = Q K(g)^T for key tile g of segment si (q buffer si & 1).
+      auto issue_s = [&](int g, int si, bool first, bool last) -> bool {
+        const int qb = si & 1;
+        if (first && !mbar_wait(su32(&q_full[qb]), (si >> 1) & 1, abort_flag, err, 13))
+          return false;
+        const int st = g % S::KST;
+        if (!mbar_wait(su32(&k_full[st]), (g / S::KST) & 1, abort_flag, err, 12)) return false;
         tc_fence_after();
-        const uint32_t ka = su32(sK + st * S::KV_BYTES);
-        const uint32_t d = tmem_base + TM_S0 + (uint32_t)((kt & 1) * AT_BN);
+        const uint32_t qa = su32(sQ + qb * S::Q_BYTES), ka = su32(sK + st * S::KV_BYTES);
+        const uint32_t d = tmem_base + S::TM_S0 + (uint32_t)((g & 1) * AT_BN);
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk)
           mma_bf16(d, sdesc_sw128(qa + (kk >> 2) * (AT_BM * 128) + (kk & 3) * 32),
                    sdesc_sw128(ka + (kk >> 2) * (AT_BN * 128) + (kk & 3) * 32), idS,
                    kk > 0 ? 1u : 0u);
-        mma_commit(su32(&s_full[kt & 1]));
+        mma_commit(su32(&s_full[g & 1]));
         mma_commit(su32(&k_empty[st]));
+        if (last) mma_commit(su32(&q_empty[qb]));
         return true;
       };
-      bool ok = mbar_wait(su32(q_full), 0, abort_flag, err, 13);
-      if (ok) {
-        tc_fence_after();
-        ok = issue_s(0);
-      }
-      for (int kt = 0; ok && kt < nkt; ++kt) {
-        if (kt + 1 < nkt && !issue_s(kt + 1)) break;
-        const int st = kt & 1;  // V stage and S/P buffer of this tile
-        if (!mbar_wait(su32(&v_full[st]), (kt >> 1) & 1, abort_flag, err, 21)) break;
-        if (!mbar_wait(su32(&p_full[st]), (kt >> 1) & 1, abort_flag, err, 14)) break;
+      // O(si & 1) += P(g) V(g) for key tile g of segment si.
+      auto issue_pv = [&](int g, int si, bool first, bool last) -> bool {
+        const int ob = si & 1, st = g & 1;
+        if (first && !mbar_wait(su32(&o_empty[ob]), ((si >> 1) & 1) ^ 1, abort_flag, err, 20))
+          return false;
+        if (!mbar_wait(su32(&v_full[st]), (g >> 1) & 1, abort_flag, err, 21)) return false;
+        if (!mbar_wait(su32(&p_full[g & 1]), (g >> 1) & 1, abort_flag, err, 14)) return false;
         tc_fence_after();
         const uint32_t va = su32(sV + st * S::KV_BYTES);
         // P keys 16kk..16kk+15: half kk/4 of the tile, columns 8(kk%4).. of that half's S
-        const uint32_t pt = tmem_base + TM_S0 + (uint32_t)(st * AT_BN);
+        const uint32_t pt = tmem_base + S::TM_S0 + (uint32_t)((g & 1) * AT_BN);
 #pragma unroll
         for (int kk = 0; kk < AT_BN / 16; ++kk)
-          mma_bf16_ts(tmem_base, pt + (uint32_t)((kk >> 2) * (AT_BN / 2) + (kk & 3) * 8),
+          mma_bf16_ts(tmem_base + (uint32_t)(ob * HD),
+                      pt + (uint32_t)((kk >> 2) * (AT_BN / 2) + (kk & 3) * 8),
                       sdesc_sw128_mn(va + kk * 16 * 128, AT_BN * 128), idO,
-                      (kt > 0 || kk > 0) ? 1u : 0u);
+                      (!first || kk > 0) ? 1u : 0u);
         mma_commit(su32(&v_empty[st]));
         mma_commit(su32(o_done));
+        if (last) mma_commit(su32(&o_full[ob]));
+        return true;
+      };
+      // Segments walked with one of lookahead: S of the next key tile (possibly
+      // the next segment's first) is issued before P V of the current one.
+      SegIter it(use_sk, U, items, KT, blockIdx.x, gridDim.x);
+      int cur_item, c0, c1, nxt_item, n0 = 0, n1 = 0;
+      bool have = it.next(cur_item, c0, c1);
+      bool have_next = have && it.next(nxt_item, n0, n1);
+      int g = 0, si = 0;
+      bool ok = !have || issue_s(0, 0, true, c0 + 1 == c1);
+      while (ok && have) {
+        for (int kt = c0; kt < c1; ++kt, ++g) {
+          if (kt + 1 < c1) {
+            if (!issue_s(g + 1, si, false, kt + 2 == c1)) { ok = false; break; }
+          } else if (have_next) {
+            if (!issue_s(g + 1, si + 1, true, n0 + 1 == n1)) { ok = false; break; }
+          }
+          if (!issue_pv(g, si, kt == c0, kt + 1 == c1)) { ok = false; break; }
+        }
+        have = have_next;
+        c0 = n0;
+        c1 = n1;
+        ++si;
+        if (have) have_next = it.next(nxt_item, n0, n1);
       }
+      (void)cur_item;
       // Every MMA this thread issued has completed before TMEM is freed.
       mma_commit(su32(done));
       mbar_drain(su32(done), 0, err, 16);
     }
   } else {
-    // Softmax: warps 2-5 take keys 0-63 of each tile (and O columns 0..HD/2), warps
-    // 6-9 keys 64-127 (and the other O columns); one thread per query row each.
+    // Softmax: warps 2-5 take keys 0-63 of each tile (and output columns
+    // 0..HD/2), warps 6-9 keys 64-127 (and the other columns); one thread per
+    // query row each.
     const int half = (warp - 2) >> 2;
     const int quarter = warp & 3;
     const int row = quarter * 32 + lane;
+    const int wi = warp - 2;  // this warp's index among the softmax warps
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
-    const uint32_t tO = tmem_base + lane_off + (uint32_t)(half * (HD / 2));
-    constexpr int KH = AT_BN / 2;  // keys per half
-    float m = -INFINITY, l = 0.f;
+    SegIter it(use_sk, U, items, KT, blockIdx.x, gridDim.x);
+    int item, kt0, kt1;
+    // key tiles, segments and exchange rounds (row maxima per tile, row sums
+    // per segment) so far
+    int g = 0, si = 0, e = 0;
     bool ok = true;
-    for (int kt = 0; kt < nkt; ++kt) {
-      if (!warp_wait(su32(&s_full[kt & 1]), (kt >> 1) & 1, abort_flag, err, 17)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      const uint32_t tS =
-          tmem_base + lane_off + TM_S0 + (uint32_t)((kt & 1) * AT_BN) + (uint32_t)(half * KH);
-      const int kbase = kt * AT_BN + half * KH;
-      const bool full = kbase + KH <= Lk;  // no key of this half-tile is past Lk
-      uint32_t sv[KH];                      // this row of S, this half of the tile
-      tmem_ld32_nowait(tS, sv);
-      tmem_ld32_nowait(tS + 32, sv + 32);
-      tmem_ld_wait();
-      if (!full) {
-#pragma unroll
-        for (int i = 0; i < KH; ++i)
-          if (kbase + i >= Lk) sv[i] = __float_as_uint(-INFINITY);
-      }
-      float pm[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) pm[j] = __uint_as_float(sv[j]);
-#pragma unroll
-      for (int i = 8; i < KH; ++i) pm[i & 7] = fmaxf(pm[i & 7], __uint_as_float(sv[i]));
-      const float hmax = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                               fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
-      // exchange the half-row maxima with the other warpgroup
-      float* xp = xch + (kt & 1) * 2 * AT_BM;
-      xp[half * AT_BM + row] = hmax;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(su32(&xbar[kt & 1]));
-      if (!warp_wait(su32(&xbar[kt & 1]), (kt >> 1) & 1, abort_flag, err, 22)) {
-        ok = false;
-        break;
-      }
-      const float mt = fmaxf(hmax, xp[(half ^ 1) * AT_BM + row]) * scale_log2;
-      if (kt > 0) {
-        const bool need = mt > m + 8.f;
-        if (__any_sync(0xffffffffu, need)) {
-          // P V of the previous tile must be complete before O is rescaled.  At
-          // least P V of tile kt-2 has completed (S(kt) was issued after it),
-          // and P V of tile kt needs this warp's P, so the parity names tile kt-1.
-          if (!warp_wait(su32(o_done), (kt - 1) & 1, abort_flag, err, 18)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const float alpha = need ? exp2_approx(m - mt) : 1.f;
-          if (need) {
-            m = mt;
-            l *= alpha;
-          }
-          uint32_t r[32];
-#pragma unroll 1
-          for (int c = 0; c < HD / 64; ++c) {
-            tmem_ld32(tO + c * 32, r);
-#pragma unroll
-            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-            tmem_st32(tO + c * 32, r);
-          }
-          tmem_st_wait();
+    while (ok && it.next(item, kt0, kt1)) {
+      const int ob = si & 1;
+      const uint32_t tO = tmem_base + lane_off + (uint32_t)(ob * HD + half * (HD / 2));
+      float m = -INFINITY, l = 0.f;
+      for (int kt = kt0; kt < kt1; ++kt, ++g, ++e) {
+        const int sb = g & 1;
+        if (!warp_wait(su32(&s_full[sb]), (g >> 1) & 1, abort_flag, err, 17)) {
+          ok = false;
+          break;
         }
-      } else {
-        m = mt;
-      }
-      // P = exp2(S * scale - m) for this half, two keys per TMEM column (the
-      // lower key in the low 16 bits), over this half's first 32 S columns.
-      float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      const float nm = -m;
-      uint32_t pk[KH / 2];
+        tc_fence_after();
+        const uint32_t tS =
+            tmem_base + lane_off + S::TM_S0 + (uint32_t)(sb * AT_BN) + (uint32_t)(half * AT_KH);
+        const int kbase = kt * AT_BN + half * AT_KH;
+        const bool full = kbase + AT_KH <= Lk;  // no key of this half-tile is past Lk
+        uint32_t sv[AT_KH];                      // this row of S, this half of the tile
+        tmem_ld32_nowait(tS, sv);
+        tmem_ld32_nowait(tS + 32, sv + 32);
+        tmem_ld_wait();
+        if (!full) {
 #pragma unroll
-      for (int i = 0; i < KH / 2; ++i) {
-        const float p0 = exp2_approx(fmaf(__uint_as_float(sv[2 * i]), scale_log2, nm));
-        const float p1 = exp2_approx(fmaf(__uint_as_float(sv[2 * i + 1]), scale_log2, nm));
-        ps[(2 * i) & 7] += p0;
-        ps[(2 * i + 1) & 7] += p1;
-        pk[i] = pack_bf16x2(p0, p1);
+          for (int i = 0; i < AT_KH; ++i)
+            if (kbase + i >= Lk) sv[i] = __float_as_uint(-INFINITY);
+        }
+        float pm[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) pm[j] = __uint_as_float(sv[j]);
+#pragma unroll
+        for (int i = 8; i < AT_KH; ++i) pm[i & 7] = fmaxf(pm[i & 7], __uint_as_float(sv[i]));
+        const float hmax = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                                 fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+        // exchange the half-row maxima with the other warpgroup
+        float* xp = xch + (e & 1) * 2 * AT_BM;
+        xp[half * AT_BM + row] = hmax;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(su32(&xbar[e & 1]));
+        if (!warp_wait(su32(&xbar[e & 1]), (e >> 1) & 1, abort_flag, err, 22)) {
+          ok = false;
+          break;
+        }
+        // finite: the first key of every key tile is valid
+        const float mt = fmaxf(hmax, xp[(half ^ 1) * AT_BM + row]) * scale_log2;
+        if (kt > kt0) {
+          const bool need = mt > m + 8.f;
+          if (__any_sync(0xffffffffu, need)) {
+            // P V of the previous tile must be complete before O is rescaled.  That
+            // of tile g-2 has completed (S(g) was issued after it), and that of
+            // tile g needs this warp's P, so the parity names tile g-1.
+            if (!warp_wait(su32(o_done), (g - 1) & 1, abort_flag, err, 18)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const float alpha = need ? exp2_approx(m - mt) : 1.f;
+            if (need) {
+              m = mt;
+              l *= alpha;
+            }
+            uint32_t r[32];
+#pragma unroll 1
+            for (int cc = 0; cc < HD / 64; ++cc) {
+              tmem_ld32(tO + cc * 32, r);
+#pragma unroll
+              for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+              tmem_st32(tO + cc * 32, r);
+            }
+          }
+        } else {
+          m = mt;
+        }
+        // P = exp2(S * scale - m) for this half, two keys per TMEM column (the
+        // lower key in the low 16 bits), over this half's first 32 S columns.
+        float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        const float nm = -m;
+        uint32_t pk[AT_KH / 2];
+#pragma unroll
+        for (int i = 0; i < AT_KH / 2; ++i) {
+          const float p0 = exp2_approx(fmaf(__uint_as_float(sv[2 * i]), scale_log2, nm));
+          const float p1 = exp2_approx(fmaf(__uint_as_float(sv[2 * i + 1]), scale_log2, nm));
+          ps[(2 * i) & 7] += p0;
+          ps[(2 * i + 1) & 7] += p1;
+          pk[i] = pack_bf16x2(p0, p1);
+        }
+        tmem_st32(tS, pk);
+        l += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(su32(&p_full[sb]));
       }
-      tmem_st32(tS, pk);
-      l += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
-      tmem_st_wait();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(su32(&p_full[kt & 1]));
-    }
-    // Combine the two halves' sums (one more exchange round), then O / l.
-    bool fin = ok;
-    if (fin) {
-      float* xp = xch + (nkt & 1) * 2 * AT_BM;
+      if (!ok) break;
+      // End of the segment: combine the two groups' row sums, then read this
+      // group's half of O once every P V of the segment has completed.
+      float* xp = xch + (e & 1) * 2 * AT_BM;
       xp[half * AT_BM + row] = l;
       __syncwarp();
-      if (lane == 0) mbar_arrive(su32(&xbar[nkt & 1]));
-      fin = warp_wait(su32(&xbar[nkt & 1]), (nkt >> 1) & 1, abort_flag, err, 23);
-      if (fin) l += xp[(half ^ 1) * AT_BM + row];
-    }
-    if (fin && warp_wait(su32(done), 0, abort_flag, err, 19)) {
+      if (lane == 0) mbar_arrive(su32(&xbar[e & 1]));
+      if (!warp_wait(su32(&xbar[e & 1]), (e >> 1) & 1, abort_flag, err, 23)) break;
+      const float lt = l + xp[(half ^ 1) * AT_BM + row];
+      ++e;
+      if (!warp_wait(su32(&o_full[ob]), (si >> 1) & 1, abort_flag, err, 19)) break;
       tc_fence_after();
-      const float inv = 1.f / l;
-      const int qrow = q0 + row;
-      bf16* orow = O + (((int64_t)sq * Lq + qrow) * H + hq) * HD + half * (HD / 2);
-      uint32_t r2[32];
-#pragma unroll 1
-      for (int c = 0; c < HD / 64; ++c) {
-        tmem_ld32(tO + c * 32, r2);
-        if (qrow < Lq) {
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            uint4 v;
-            v.x = pack_bf16x2(__uint_as_float(r2[8 * j]) * inv, __uint_as_float(r2[8 * j + 1]) * inv);
-            v.y = pack_bf16x2(__uint_as_float(r2[8 * j + 2]) * inv, __uint_as_float(r2[8 * j + 3]) * inv);
-            v.z = pack_bf16x2(__uint_as_float(r2[8 * j + 4]) * inv, __uint_as_float(r2[8 * j + 5]) * inv);
-            v.w = pack_bf16x2(__uint_as_float(r2[8 * j + 6]) * inv, __uint_as_float(r2[8 * j + 7]) * inv);
-            *reinterpret_cast<uint4*>(orow + c * 32 + 8 * j) = v;
-          }
-        }
-      }
+      if (!segment_output<HD>(tO, m, lt, item, kt0, kt1, KT, QT, H, Lq, U, O, half, row, lane,
+                              wi, sk, err, abort_flag))
+        break;
+      // This O buffer may now take the segment after next.
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(su32(&o_empty[ob]));
+      ++si;
     }
   }
 
@@ -383,6 +614,15 @@ bool make_tmap_op(CUtensorMap* tm, const AttnOperand& op, int hd, int L, int H, 
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+std::atomic<int> g_attn_schedule{0};
+
+// Schedule by a makespan model in key-tile units: data-parallel costs
+// ceil(items / G) x (KT + AT_OV), stream-K U / G + items / G x AT_OV + AT_FIX,
+// where AT_OV is the per-item cost of loading Q and writing the output and
+// AT_FIX the fix-up of a split item (publish, counter round trips, combine).
+// Stream-K must win by 3 %: near-ties measured slower.
+constexpr double AT_OV = 1.5, AT_FIX = 6.0;
+
 template <int HD>
 cudaError_t launch_attn_tc(const AttnOperand& Q, const AttnOperand& K, const AttnOperand& V,
                            void* O, int S_, int H, int Lq, int Lk, cudaStream_t s) {
@@ -400,18 +640,39 @@ cudaError_t launch_attn_tc(const AttnOperand& Q, const AttnOperand& K, const Att
   cudaError_t e = cudaFuncSetAttribute(k_attn_tc<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)S1::SMEM);
   if (e != cudaSuccess) return e;
-  dim3 grid((Lq + AT_BM - 1) / AT_BM, S_ * H);
+  const int QT = (Lq + AT_BM - 1) / AT_BM, KT = (Lk + AT_BN - 1) / AT_BN;
+  const int64_t items = (int64_t)S_ * H * QT;
+  if (items > (1 << 26)) return cudaErrorInvalidValue;
+  const int G = num_sms();
+  int grid = items < G ? (int)items : G;
+  AtSk sk = {nullptr, nullptr, 0};
+  const int mode = g_attn_schedule.load();
+  if (mode != 1) {
+    const int64_t U = items * KT, per = U / G;
+    const bool spans_ok = per > 0 && 1 + (KT - 1 + per - 1) / per <= AT_MAX_PARTS;
+    const double dp_cost = (double)((items + G - 1) / G) * (KT + AT_OV);
+    const double sk_cost = (double)U / G + (double)items / G * AT_OV + AT_FIX;
+    if (spans_ok && (mode == 2 || sk_cost < 0.97 * dp_cost) &&
+        sk_scratch(s, (size_t)8 * items, (size_t)2 * G * S1::SLOT, &sk.cnt, &sk.ws)) {
+      sk.units = U;
+      grid = G;
+    } else {
+      sk = {nullptr, nullptr, 0};
+    }
+  }
   count_launch();
   return launch_pdl(k_attn_tc<HD>, grid, AT_THREADS, S1::SMEM, s, tq, tk, tv, (bf16*)O, H, Lq, Lk,
-                    scale_log2, q_tok, k_tok, err);
+                    scale_log2, q_tok, k_tok, err, (int)items, sk);
 }
 
 }  // namespace
 
+void set_attention_schedule(int mode) { g_attn_schedule.store(mode); }
+
 cudaError_t attention_bf16(const AttnOperand& Q, const AttnOperand& K, const AttnOperand& V,
                            void* O, int S, int H, int Lq, int Lk, int hd, cudaStream_t s) {
   if (S <= 0 || Lq <= 0) return cudaSuccess;
-  if (Lk <= 0 || S * H > 65535) return cudaErrorInvalidValue;
+  if (Lk <= 0) return cudaErrorInvalidValue;
   if ((((uintptr_t)Q.ptr) | ((uintptr_t)K.ptr) | ((uintptr_t)V.ptr) | ((uintptr_t)O)) & 15)
     return cudaErrorMisalignedAddress;
   if (hd == 128) return launch_attn_tc<128>(Q, K, V, O, S, H, Lq, Lk, s);

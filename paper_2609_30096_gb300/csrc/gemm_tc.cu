@@ -80,52 +80,6 @@ struct SkArgs {
   int64_t units;  // work tiles * k-blocks
 };
 
-// Worker (cluster) whose share [w U / G, (w+1) U / G) holds unit u.
-__device__ __forceinline__ int sk_worker_of(int64_t u, int64_t U, int G) {
-  return (int)(((u + 1) * G + U - 1) / U) - 1;
-}
-
-// Segment sequence of worker w of G: (work tile, first k-block, end k-block).
-struct SegIter {
-  int64_t u, u1;
-  int tile, stride, num_tiles, nk;
-  bool sk;
-  __device__ SegIter(bool sk_, int64_t U, int num_tiles_, int nk_, int w, int G) {
-    sk = sk_;
-    num_tiles = num_tiles_;
-    nk = nk_;
-    u = (int64_t)w * U / G;
-    u1 = (int64_t)(w + 1) * U / G;
-    tile = w;
-    stride = G;
-  }
-  // True once the segment just returned is the worker's last.
-  __device__ bool done() const { return sk ? u >= u1 : tile >= num_tiles; }
-  __device__ bool next(int& t, int& k0, int& k1) {
-    if (sk) {
-      if (u >= u1) return false;
-      t = (int)(u / nk);
-      k0 = (int)(u - (int64_t)t * nk);
-      const int64_t left = u1 - u;
-      k1 = left < (int64_t)(nk - k0) ? k0 + (int)left : nk;
-      u += k1 - k0;
-      return true;
-    }
-    if (tile >= num_tiles) return false;
-    t = tile;
-    k0 = 0;
-    k1 = nk;
-    tile += stride;
-    return true;
-  }
-};
-
-__device__ __forceinline__ int ld_acquire(const int* p) {
-  int v;
-  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-
 constexpr int SK_MAX_PARTS = 4;     // the host only picks stream-K when no tile spans more workers
 // Makespan-model cost of the stream-K fix-up (publishing a partial tile, the
 // counter round trips and the final combine: about 8 us), in the model's units
@@ -577,46 +531,6 @@ bool make_tmap(CUtensorMap* tm, CUtensorMapDataType dt, size_t esize, const void
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Stream-K counters and partial-sum slots, one set per (device, stream): GEMMs
-// on one stream run one after another, so they can share them.
-struct SkScratch {
-  int* cnt = nullptr;
-  size_t ncnt = 0;
-  float* ws = nullptr;
-  size_t nws = 0;
-};
-std::mutex g_sk_mu;
-std::map<std::pair<int, cudaStream_t>, SkScratch> g_sk;
-
-// Returns false (and leaves *out empty) if the buffers cannot be had.
-bool sk_scratch(cudaStream_t s, size_t ncnt, size_t nws, SkArgs* out) {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return false;
-  std::lock_guard<std::mutex> lk(g_sk_mu);
-  SkScratch& sc = g_sk[std::make_pair(dev, s)];
-  if (sc.ncnt < ncnt || sc.nws < nws) {
-    if (cudaStreamSynchronize(s) != cudaSuccess) return false;
-    cudaFree(sc.cnt);
-    cudaFree(sc.ws);
-    sc = SkScratch();
-    const size_t nc = ncnt > 4096 ? ncnt : 4096, nw = nws;
-    if (cudaMalloc(&sc.cnt, nc * sizeof(int)) != cudaSuccess ||
-        cudaMalloc(&sc.ws, nw * sizeof(float)) != cudaSuccess ||
-        cudaMemsetAsync(sc.cnt, 0, nc * sizeof(int), s) != cudaSuccess) {
-      cudaGetLastError();
-      cudaFree(sc.cnt);
-      cudaFree(sc.ws);
-      sc = SkScratch();
-      return false;
-    }
-    sc.ncnt = nc;
-    sc.nws = nw;
-  }
-  out->cnt = sc.cnt;
-  out->ws = sc.ws;
-  return true;
-}
-
 // Concurrently resident workers (CTAs, or clusters of CL CTAs) of one kernel
 // instantiation on the current device, looked up once.
 template <int BN, int STAGES, int CL>
@@ -678,7 +592,7 @@ cudaError_t launch_tc(const void* A, const void* W, const GemmArgs& g, bool stre
   SkArgs sk = {nullptr, nullptr, 0};
   if (stream_k) {
     sk.units = (int64_t)tiles * (g.K / BK);
-    if (sk_scratch(s, (size_t)4 * tiles * CL, (size_t)2 * wmax * CL * BM * BN, &sk))
+    if (sk_scratch(s, (size_t)4 * tiles * CL, (size_t)2 * wmax * CL * BM * BN, &sk.cnt, &sk.ws))
       workers = wmax;
     else
       sk = {nullptr, nullptr, 0};
@@ -749,6 +663,49 @@ EncodeTiledFn encode_tiled_fn() {
   }();
   return fn;
 }
+
+namespace {
+// Stream-K counters and partial-sum slots, one set per (device, stream): the
+// kernels of one stream run one after another and leave every counter at zero,
+// so the GEMM and attention launches of a stream share them.
+struct SkScratch {
+  int* cnt = nullptr;
+  size_t ncnt = 0;
+  float* ws = nullptr;
+  size_t nws = 0;
+};
+std::mutex g_sk_mu;
+std::map<std::pair<int, cudaStream_t>, SkScratch> g_sk;
+}  // namespace
+
+bool sk_scratch(cudaStream_t s, size_t ncnt, size_t nws, int** cnt, float** ws) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  std::lock_guard<std::mutex> lk(g_sk_mu);
+  SkScratch& sc = g_sk[std::make_pair(dev, s)];
+  if (sc.ncnt < ncnt || sc.nws < nws) {
+    if (cudaStreamSynchronize(s) != cudaSuccess) return false;
+    cudaFree(sc.cnt);
+    cudaFree(sc.ws);
+    sc = SkScratch();
+    const size_t nc = ncnt > 4096 ? ncnt : 4096, nw = nws;
+    if (cudaMalloc(&sc.cnt, nc * sizeof(int)) != cudaSuccess ||
+        cudaMalloc(&sc.ws, nw * sizeof(float)) != cudaSuccess ||
+        cudaMemsetAsync(sc.cnt, 0, nc * sizeof(int), s) != cudaSuccess) {
+      cudaGetLastError();
+      cudaFree(sc.cnt);
+      cudaFree(sc.ws);
+      sc = SkScratch();
+      return false;
+    }
+    sc.ncnt = nc;
+    sc.nws = nw;
+  }
+  *cnt = sc.cnt;
+  *ws = sc.ws;
+  return true;
+}
+
 
 namespace {
 std::atomic<int> g_schedule{0};

@@ -85,6 +85,10 @@ cudaError_t gemm_f32(const float* A, const float* W, const GemmArgs& g, cudaStre
 // bf16 tcgen05 GEMM: A bf16 [M,K] and W bf16 [N,K], fp32 accumulation in TMEM.
 // Requires K % 64 == 0, N % 32 == 0 and 16-byte aligned A, W and out.
 cudaError_t gemm_bf16_tc(const void* A, const void* W, const GemmArgs& g, cudaStream_t s);
+// Stream-K counters (zero between launches) and fp32 partial-sum slots of the
+// stream, grown on demand (a growth synchronizes the stream).  False if they
+// cannot be allocated.
+bool sk_scratch(cudaStream_t s, size_t ncnt, size_t nws, int** cnt, float** ws);
 // 0 auto, 1 data-parallel, 2 stream-K where the shape allows it; + 4: W tiles
 // shared by two-CTA clusters through TMA multicast.
 void set_gemm_schedule(int mode);
@@ -107,6 +111,8 @@ inline AttnOperand token_major(const void* p, int L, int ld, int hd) {
 // O [S, Lq, H, hd] (token-major) = softmax(Q K^T / sqrt(hd)) V.
 cudaError_t attention_f32(const AttnOperand& Q, const AttnOperand& K, const AttnOperand& V,
                           float* O, int S, int H, int Lq, int Lk, int hd, cudaStream_t s);
+// 0 auto, 1 data-parallel, 2 stream-K where the shape allows it.
+void set_attention_schedule(int mode);
 cudaError_t attention_bf16(const AttnOperand& Q, const AttnOperand& K, const AttnOperand& V,
                            void* O, int S, int H, int Lq, int Lk, int hd, cudaStream_t s);
 

@@ -295,6 +295,54 @@ __device__ __forceinline__ float exp2_approx(float x) {
   return y;
 }
 
+// Stream-K work split: U units (a work tile's k-blocks, or a query tile's key
+// tiles, in order) shared out as G contiguous ranges.
+// Worker whose share [w U / G, (w+1) U / G) holds unit u.
+__device__ __forceinline__ int sk_worker_of(int64_t u, int64_t U, int G) {
+  return (int)(((u + 1) * G + U - 1) / U) - 1;
+}
+
+// Segment sequence of worker w of G: (work tile, first k-block, end k-block).
+struct SegIter {
+  int64_t u, u1;
+  int tile, stride, num_tiles, nk;
+  bool sk;
+  __device__ SegIter(bool sk_, int64_t U, int num_tiles_, int nk_, int w, int G) {
+    sk = sk_;
+    num_tiles = num_tiles_;
+    nk = nk_;
+    u = (int64_t)w * U / G;
+    u1 = (int64_t)(w + 1) * U / G;
+    tile = w;
+    stride = G;
+  }
+  // True once the segment just returned is the worker's last.
+  __device__ bool done() const { return sk ? u >= u1 : tile >= num_tiles; }
+  __device__ bool next(int& t, int& k0, int& k1) {
+    if (sk) {
+      if (u >= u1) return false;
+      t = (int)(u / nk);
+      k0 = (int)(u - (int64_t)t * nk);
+      const int64_t left = u1 - u;
+      k1 = left < (int64_t)(nk - k0) ? k0 + (int)left : nk;
+      u += k1 - k0;
+      return true;
+    }
+    if (tile >= num_tiles) return false;
+    t = tile;
+    k0 = 0;
+    k1 = nk;
+    tile += stride;
+    return true;
+  }
+};
+
+__device__ __forceinline__ int ld_acquire(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
 }  // namespace tc
 
 // Host: cuTensorMapEncodeTiled through the runtime's driver entry point.

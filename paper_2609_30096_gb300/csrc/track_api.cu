@@ -737,6 +737,13 @@ int track_gemm_schedule(int mode) {
   return TRACK_OK;
 }
 
+int track_attention_schedule(int mode) {
+  if (mode < TRACK_GEMM_AUTO || mode > TRACK_GEMM_STREAM_K)
+    return fail(TRACK_EINVAL, "unknown attention schedule");
+  set_attention_schedule(mode);
+  return TRACK_OK;
+}
+
 int track_profile_enable(int enable) {
   g_prof_on.store(enable != 0);
   return TRACK_OK;

@@ -112,3 +112,12 @@ def test_gemm_schedule_modes(T):
         with pytest.raises(T.TrackError) as e:
             T.track_gemm_schedule(bad)
         assert e.value.code == T.TRACK_EINVAL
+
+
+def test_attention_schedule_modes(T):
+    for mode in (T.GEMM_DATA_PARALLEL, T.GEMM_STREAM_K, T.GEMM_AUTO):
+        T.track_attention_schedule(mode)
+    for bad in (-1, 3, T.GEMM_STREAM_K | T.GEMM_MULTICAST):
+        with pytest.raises(T.TrackError) as e:
+            T.track_attention_schedule(bad)
+        assert e.value.code == T.TRACK_EINVAL

@@ -256,6 +256,64 @@ def test_attention_growing_logits(T, hd):
     assert rel_l2(O.float().cpu().numpy(), _attn_ref(Q, K, V)) < 1e-2
 
 
+# Both attention schedules at shapes where stream-K splits query tiles over 2
+# (bench shape, ragged keys, hd 64), 3 and 4 CTAs; each run twice for bits.
+ATTN_SCHED_CASES = [
+    (1, 12, 3510, 3510, 128),
+    (4, 16, 1000, 700, 128),
+    (1, 4, 2400, 2000, 128),
+    (1, 6, 1100, 2000, 128),
+    (2, 40, 600, 512, 64),
+]
+
+
+@pytest.fixture(params=["dp", "sk"])
+def attn_schedule(T, request):
+    T.track_attention_schedule(T.GEMM_DATA_PARALLEL if request.param == "dp" else T.GEMM_STREAM_K)
+    yield request.param
+    T.track_attention_schedule(T.GEMM_AUTO)
+
+
+@pytest.mark.parametrize("S,H,Lq,Lk,hd", ATTN_SCHED_CASES)
+def test_attention_schedules(T, attn_schedule, S, H, Lq, Lk, hd):
+    rng = np.random.default_rng(Lq * 5 + Lk + hd + H)
+    Q = dit.round_bf16(rng.normal(size=(S, H, Lq, hd)).astype(np.float32))
+    K = dit.round_bf16(rng.normal(size=(S, H, Lk, hd)).astype(np.float32))
+    V = dit.round_bf16(rng.normal(size=(S, H, Lk, hd)).astype(np.float32))
+    Qd, Kd, Vd = dev_bf16(Q), dev_bf16(K), dev_bf16(V)
+    outs = []
+    for _ in range(2):
+        O = torch.zeros((S, Lq, H, hd), dtype=torch.bfloat16, device=DEV)
+        T.track_attention(T.BF16, Qd, Kd, Vd, O)
+        T.track_sync()
+        outs.append(O.float().cpu().numpy())
+    assert np.array_equal(outs[0], outs[1])
+    rows = rng.choice(Lq, min(Lq, 48), replace=False)
+    ref = _attn_ref(Q[:, :, rows], K, V)
+    assert rel_l2(outs[0][:, rows], ref) < 1e-2
+
+
+@pytest.mark.parametrize("hd", [64, 128])
+def test_attention_growing_logits_split(T, hd):
+    # Stream-K with query tiles split over up to four CTAs whose parts reach
+    # very different row maxima: the combine's 2^(m_p - M) weights matter.
+    rng = np.random.default_rng(hd + 17)
+    S, H, Lq, Lk = 1, 8, 1000, 2000
+    ramp = (1.0 + 4.0 * np.arange(Lk) / Lk)[None, None, :, None]
+    Q = dit.round_bf16((4.0 * rng.normal(size=(S, H, Lq, hd))).astype(np.float32))
+    K = dit.round_bf16((ramp * rng.normal(size=(S, H, Lk, hd))).astype(np.float32))
+    V = dit.round_bf16(rng.normal(size=(S, H, Lk, hd)).astype(np.float32))
+    T.track_attention_schedule(T.GEMM_STREAM_K)
+    try:
+        O = torch.zeros((S, Lq, H, hd), dtype=torch.bfloat16, device=DEV)
+        T.track_attention(T.BF16, dev_bf16(Q), dev_bf16(K), dev_bf16(V), O)
+        T.track_sync()
+    finally:
+        T.track_attention_schedule(T.GEMM_AUTO)
+    rows = rng.choice(Lq, 64, replace=False)
+    assert rel_l2(O.float().cpu().numpy()[:, rows], _attn_ref(Q[:, :, rows], K, V)) < 1e-2
+
+
 def test_attention_single_key_returns_value_row(T):
     rng = np.random.default_rng(5)
     Q = rng.normal(size=(1, 2, 70, 64)).astype(np.float32)
