@@ -236,6 +236,23 @@ int track_sample(track_model* large, track_model* small, const uint8_t* policy,
                  const float* sigmas, int n_steps, float* x, int B, const float* cond,
                  const float* uncond, float cfg_scale, track_stream s);
 
+/* track_sample through a CUDA graph.  It computes the same values bit for bit,
+ * with the text projection of cond/uncond recomputed on every call.  The
+ * library keeps up to 32 recorded graphs, keyed by every argument (models,
+ * policy and sigma values, pointers, B, cfg_scale, stream).  The first call
+ * with a key runs eagerly and sizes every buffer the graph will address.  The
+ * second call records the loop on s and instantiates it.  Later calls replay
+ * it with one launch, so host launch time no longer paces the GPU.  Replays
+ * read the current contents of x, cond and uncond.  A graph is dropped when
+ * a model it uses is destroyed or a buffer it addresses is reallocated.
+ * s must be a created stream: EINVAL for the legacy default stream (it cannot
+ * be recorded).  Kernel timing (track_profile_enable) sees none of the
+ * replayed kernels.  This is a host-side mechanism; the paper has no
+ * counterpart. */
+int track_sample_graph(track_model* large, track_model* small, const uint8_t* policy,
+                       const float* sigmas, int n_steps, float* x, int B, const float* cond,
+                       const float* uncond, float cfg_scale, track_stream s);
+
 /* ---- building blocks (the denoiser's kernels, for tests and benchmarks) --- */
 
 /* Y = X W^T + bias with an epilogue (TRACK_EPI_*).  dtype selects the kernel:

@@ -83,6 +83,7 @@ def lib():
         "track_policy_random_k": (_I, [_I, _I, ctypes.c_uint64, _P]),
         "track_calibrate": (_I, [_P, _P, _P, _I, _P, _P, _F, _P, _I, _F, _P, _P]),
         "track_sample": (_I, [_P, _P, _P, _P, _I, _P, _I, _P, _P, _F, _P]),
+        "track_sample_graph": (_I, [_P, _P, _P, _P, _I, _P, _I, _P, _P, _F, _P]),
         "track_linear": (_I, [_I, _P, _P, _P, _I, _I, _I, _I, _P, _P, _I, _P]),
         "track_attention": (_I, [_I, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P]),
     }
@@ -364,6 +365,19 @@ def track_sample(large: Model, small: Model, policy, sigmas, x, cond, uncond, cf
     _check(lib().track_sample(large.handle, small.handle, pol.ctypes.data, sig.ctypes.data,
                               pol.shape[0], _ptr(x), x.shape[0], _ptr(cond), _ptr(uncond),
                               cfg_scale, _stream(stream)))
+    return x
+
+
+def track_sample_graph(large: Model, small: Model, policy, sigmas, x, cond, uncond, cfg_scale,
+                       stream=None):
+    """track_sample replayed from a recorded CUDA graph (first call eager, second records)."""
+    pol = np.ascontiguousarray(policy, dtype=np.uint8)
+    sig = np.ascontiguousarray(sigmas, dtype=np.float32)
+    if pol.shape[0] != sig.shape[0] - 1:
+        raise ValueError("policy needs one entry per step")
+    _check(lib().track_sample_graph(large.handle, small.handle, pol.ctypes.data, sig.ctypes.data,
+                                    pol.shape[0], _ptr(x), x.shape[0], _ptr(cond), _ptr(uncond),
+                                    cfg_scale, _stream(stream)))
     return x
 
 

@@ -676,7 +676,10 @@ struct SkScratch {
 };
 std::mutex g_sk_mu;
 std::map<std::pair<int, cudaStream_t>, SkScratch> g_sk;
+std::atomic<uint64_t> g_sk_gen{0};
 }  // namespace
+
+uint64_t sk_scratch_generation() { return g_sk_gen.load(); }
 
 bool sk_scratch(cudaStream_t s, size_t ncnt, size_t nws, int** cnt, float** ws) {
   int dev = 0;
@@ -684,6 +687,7 @@ bool sk_scratch(cudaStream_t s, size_t ncnt, size_t nws, int** cnt, float** ws) 
   std::lock_guard<std::mutex> lk(g_sk_mu);
   SkScratch& sc = g_sk[std::make_pair(dev, s)];
   if (sc.ncnt < ncnt || sc.nws < nws) {
+    g_sk_gen.fetch_add(1);
     if (cudaStreamSynchronize(s) != cudaSuccess) return false;
     cudaFree(sc.cnt);
     cudaFree(sc.ws);

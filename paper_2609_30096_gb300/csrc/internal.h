@@ -89,6 +89,8 @@ cudaError_t gemm_bf16_tc(const void* A, const void* W, const GemmArgs& g, cudaSt
 // stream, grown on demand (a growth synchronizes the stream).  False if they
 // cannot be allocated.
 bool sk_scratch(cudaStream_t s, size_t ncnt, size_t nws, int** cnt, float** ws);
+// Bumped whenever any stream-K scratch is reallocated (recorded graphs hold its addresses).
+uint64_t sk_scratch_generation();
 // 0 auto, 1 data-parallel, 2 stream-K where the shape allows it; + 4: W tiles
 // shared by two-CTA clusters through TMA multicast.
 void set_gemm_schedule(int mode);

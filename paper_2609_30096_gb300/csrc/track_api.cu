@@ -90,12 +90,15 @@ static std::atomic<bool> g_prof_on{false};
 static std::vector<ProfRec> g_prof;
 static std::vector<std::pair<cudaEvent_t, cudaEvent_t>> g_prof_pool;
 
+// True on a thread while it records a CUDA graph (no event brackets then).
+static thread_local bool g_capturing = false;
+
 struct ProfScope {
   bool on = false;
   ProfRec r;
   cudaStream_t s;
   ProfScope(int cls, double flops, cudaStream_t st) : s(st) {
-    if (!g_prof_on.load(std::memory_order_relaxed)) return;
+    if (g_capturing || !g_prof_on.load(std::memory_order_relaxed)) return;
     std::lock_guard<std::mutex> lk(g_prof_mu);
     if (!g_prof_pool.empty()) {
       r.a = g_prof_pool.back().first;
@@ -223,6 +226,7 @@ struct track_model {
   const float* c_uncond = nullptr;
   int c_nseq = -1;
   bool c_valid = false;
+  uint64_t ws_gen = 0;  // bumped whenever the workspace is reallocated (graphs hold its addresses)
 };
 
 namespace track {
@@ -388,6 +392,7 @@ static int ensure_workspace(track_model* m, int nseq) {
   w.base = nullptr;
   w.cap = 0;
   m->c_valid = false;
+  ++m->ws_gen;
   const track_arch& a = m->a;
   const int64_t d = a.dim, F = a.ffn, Lt = a.text_len, Dt = a.text_dim;
   const int64_t M = (int64_t)nseq * m->L_tok, Mt = (int64_t)nseq * Lt;
@@ -552,7 +557,7 @@ static int forward(track_model* m, const float* x, int B, int nseq, float t, con
   const track_arch& a = m->a;
   TRACK_TRY(ensure_workspace(m, nseq));
   Workspace& w = m->ws;
-  const int d = a.dim, F = a.ffn, L = m->L_tok, H = a.heads;
+  const int d = a.dim, F = a.ffn, L = m->L_tok;
   const int M = nseq * L;
   const size_t es = m->esz;
 
@@ -821,10 +826,13 @@ static int model_alloc(const track_arch* arch, track_model** out, track_model** 
   return TRACK_OK;
 }
 
+static void drop_graphs_of(const track_model* m);
+
 int track_model_destroy(track_model* m) {
   if (m == nullptr) return TRACK_OK;
   set_device(m);
   cudaDeviceSynchronize();
+  drop_graphs_of(m);
   free_workspace(m->ws);
   if (m->wbuf) cudaFree(m->wbuf);
   if (m->rope_tab) cudaFree(m->rope_tab);
@@ -1062,6 +1070,150 @@ int track_sample(track_model* large, track_model* small, const uint8_t* policy, 
     TRACK_TRY(denoise_step_impl(m, x, B, sigmas[i], sigmas[i + 1], cond, uncond, cfg_scale,
                                 (cudaStream_t)s));
   }
+  return TRACK_OK;
+}
+
+// ---------------------------------------------------------------- routed loop as a CUDA graph
+namespace {
+struct GraphEntry {
+  track_model *L, *S;
+  std::string policy;
+  std::vector<float> sigmas;
+  float* x;
+  int B;
+  const float *cond, *uncond;
+  float w;
+  cudaStream_t s;
+  int dev;
+  uint64_t gen_L, gen_S, gen_sk;  // allocations the graph's addresses come from
+  cudaGraphExec_t exec = nullptr;
+  int64_t launches = 0;  // kernels recorded in the graph
+};
+std::mutex g_graph_mu;
+std::vector<GraphEntry> g_graphs;
+constexpr size_t kMaxGraphs = 32;
+
+bool same_call(const GraphEntry& e, const GraphEntry& k) {
+  return e.L == k.L && e.S == k.S && e.policy == k.policy && e.sigmas == k.sigmas && e.x == k.x &&
+         e.B == k.B && e.cond == k.cond && e.uncond == k.uncond && e.w == k.w && e.s == k.s &&
+         e.dev == k.dev;
+}
+
+void drop_graph(GraphEntry& e) {
+  if (e.exec) cudaGraphExecDestroy(e.exec);
+  e.exec = nullptr;
+}
+
+// The routed loop of Eq. 3 with the text projection always recomputed.
+int sample_loop(track_model* large, track_model* small, const uint8_t* policy,
+                const float* sigmas, int n_steps, float* x, int B, const float* cond,
+                const float* uncond, float cfg_scale, cudaStream_t s) {
+  large->c_valid = false;
+  small->c_valid = false;
+  for (int i = 0; i < n_steps; ++i) {
+    track_model* m = policy[i] ? small : large;
+    TRACK_TRY(denoise_step_impl(m, x, B, sigmas[i], sigmas[i + 1], cond, uncond, cfg_scale, s));
+  }
+  return TRACK_OK;
+}
+}  // namespace
+
+// Drops every recorded graph that uses model m.
+static void drop_graphs_of(const track_model* m) {
+  std::lock_guard<std::mutex> lk(g_graph_mu);
+  for (size_t i = 0; i < g_graphs.size();) {
+    if (g_graphs[i].L == m || g_graphs[i].S == m) {
+      drop_graph(g_graphs[i]);
+      g_graphs.erase(g_graphs.begin() + (long)i);
+    } else {
+      ++i;
+    }
+  }
+}
+
+int track_sample_graph(track_model* large, track_model* small, const uint8_t* policy,
+                       const float* sigmas, int n_steps, float* x, int B, const float* cond,
+                       const float* uncond, float cfg_scale, track_stream s) {
+  if (!large || !small) return fail(TRACK_EINVAL, "model is NULL");
+  if (track_models_compatible(large, small) != 1)
+    return fail(TRACK_EINVAL, "models are not a compatible pair");
+  if (!policy || !sigmas || n_steps < 1) return fail(TRACK_EINVAL, "bad arguments");
+  if ((cudaStream_t)s == nullptr || (cudaStream_t)s == cudaStreamLegacy)
+    return fail(TRACK_EINVAL, "a CUDA graph cannot be recorded on the legacy default stream");
+  TRACK_TRY(check_denoise_args(large, x, B, cond, uncond, cfg_scale, x));
+  TRACK_TRY(set_device(large));
+  const cudaStream_t st = (cudaStream_t)s;
+  GraphEntry key;
+  key.L = large; key.S = small;
+  key.policy.assign((const char*)policy, (size_t)n_steps);
+  key.sigmas.assign(sigmas, sigmas + n_steps + 1);
+  key.x = x; key.B = B; key.cond = cond; key.uncond = cfg_scale == 1.f ? nullptr : uncond;
+  key.w = cfg_scale; key.s = st; key.dev = large->dev;
+  cudaGraphExec_t exec = nullptr;
+  int64_t nlaunch = 0;
+  bool warm = false;
+  {
+    std::lock_guard<std::mutex> lk(g_graph_mu);
+    for (size_t i = 0; i < g_graphs.size(); ++i) {
+      GraphEntry& e = g_graphs[i];
+      if (!same_call(e, key)) continue;
+      if (e.gen_L != large->ws_gen || e.gen_S != small->ws_gen ||
+          e.gen_sk != sk_scratch_generation()) {  // an address it holds was freed
+        drop_graph(e);
+        g_graphs.erase(g_graphs.begin() + (long)i);
+        break;
+      }
+      warm = true;
+      exec = e.exec;
+      nlaunch = e.launches;
+      break;
+    }
+  }
+  if (!warm) {
+    // First call with these arguments: run eagerly, which also sizes every
+    // buffer the graph will address.
+    TRACK_TRY(sample_loop(large, small, policy, sigmas, n_steps, x, B, cond, uncond, cfg_scale, st));
+    key.gen_L = large->ws_gen;
+    key.gen_S = small->ws_gen;
+    key.gen_sk = sk_scratch_generation();
+    std::lock_guard<std::mutex> lk(g_graph_mu);
+    if (g_graphs.size() >= kMaxGraphs) {
+      drop_graph(g_graphs.front());
+      g_graphs.erase(g_graphs.begin());
+    }
+    g_graphs.push_back(key);
+    return TRACK_OK;
+  }
+  if (exec == nullptr) {
+    // Second call: record the loop (kernels are recorded, not run) and instantiate it.
+    cudaGraph_t graph = nullptr;
+    TRACK_CUDA(cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal));
+    g_capturing = true;
+    const int64_t n0 = track_launch_count();
+    const int rc =
+        sample_loop(large, small, policy, sigmas, n_steps, x, B, cond, uncond, cfg_scale, st);
+    nlaunch = track_launch_count() - n0;
+    g_capturing = false;
+    const cudaError_t ce = cudaStreamEndCapture(st, &graph);
+    large->c_valid = small->c_valid = false;  // the recorded projection has not run yet
+    if (rc != TRACK_OK) {
+      if (graph) cudaGraphDestroy(graph);
+      return rc;
+    }
+    if (ce != cudaSuccess) return fail(TRACK_ECUDA, std::string("graph capture: ") + cudaGetErrorString(ce));
+    const cudaError_t ie = cudaGraphInstantiate(&exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (ie != cudaSuccess) return fail(TRACK_ECUDA, std::string("graph instantiate: ") + cudaGetErrorString(ie));
+    g_launches.fetch_sub(nlaunch, std::memory_order_relaxed);  // recorded, not launched
+    std::lock_guard<std::mutex> lk(g_graph_mu);
+    for (GraphEntry& e : g_graphs)
+      if (same_call(e, key)) {
+        e.exec = exec;
+        e.launches = nlaunch;
+      }
+  }
+  TRACK_CUDA(cudaGraphLaunch(exec, st));
+  count_launch((int)nlaunch);
   return TRACK_OK;
 }
 

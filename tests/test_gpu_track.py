@@ -175,6 +175,44 @@ def test_routed_sampling_follows_the_oracle(T, tiny, calib_inputs, oracle_calibr
     assert cnt == {"L": 2 * 2 * int((pol == 0).sum()), "S": 2 * 2 * int(pol.sum())}
 
 
+def test_graph_replay_matches_eager(T, tiny):
+    # First call eager, second records and replays, later calls replay: every
+    # call must equal an eager run bit for bit, with the buffers' current
+    # contents (new latent values each call, same pointer) and the same kernels.
+    prec, P = tiny
+    pol = np.array([0, 1, 1, 0, 1, 0, 0, 1][:WL.steps], np.uint8)
+    x, c, u = synth.evaluation_inputs(WL.large, 3, 2, with_uncond=True)
+    sig = track.schedule(WL.steps, WL.shift)
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        cd, ud, xg = dev(c), dev(u), dev(x)
+        for call in range(4):
+            x_in = torch.from_numpy((x * (1.0 + 0.25 * call)).astype(np.float32)).cuda()
+            xg.copy_(x_in)
+            n0 = T.track_launch_count()
+            T.track_sample_graph(P.L, P.S, pol, sig, xg, cd, ud, WL.cfg, stream=s.cuda_stream)
+            n_graph = T.track_launch_count() - n0
+            xe = x_in.clone()
+            T.track_invalidate_ctx(P.L)
+            T.track_invalidate_ctx(P.S)
+            n0 = T.track_launch_count()
+            T.track_sample(P.L, P.S, pol, sig, xe, cd, ud, WL.cfg, stream=s.cuda_stream)
+            n_eager = T.track_launch_count() - n0
+            T.track_sync(s.cuda_stream)
+            assert torch.equal(xg, xe), call
+            assert n_graph == n_eager, call
+        # a different policy is a different graph (eager first), still exact
+        xg.copy_(dev(x))
+        T.track_sample_graph(P.L, P.S, 1 - pol, sig, xg, cd, ud, WL.cfg, stream=s.cuda_stream)
+        xe = dev(x)
+        T.track_sample(P.L, P.S, 1 - pol, sig, xe, cd, ud, WL.cfg, stream=s.cuda_stream)
+        T.track_sync(s.cuda_stream)
+        assert torch.equal(xg, xe)
+    with pytest.raises(T.TrackError) as e:   # the legacy default stream cannot be recorded
+        T.track_sample_graph(P.L, P.S, pol, sig, dev(x), dev(c), dev(u), WL.cfg, stream=0)
+    assert e.value.code == T.TRACK_EINVAL
+
+
 def test_argument_errors(T, tiny, calib_inputs):
     prec, P = tiny
     x, c, u = calib_inputs
