@@ -46,6 +46,41 @@ def euler_update(x, p, sigma_t, sigma_next):
     return x + (float(sigma_next) - float(sigma_t)) * np.asarray(p, dtype=np.float64)
 
 
+def multistep_update(i: int, x, p, state, sigmas):
+    """Scheduler update S(x_{t_i}, p, t_i, h_i) of Eq. 2 with a history h_i: a
+    second-order predictor-corrector for the flow-matching ODE dx/dsigma = v.
+
+    Sec. 3.1 lets S carry any history a multistep solver needs, and TRACK keeps
+    its evolution unchanged while switching models; the pipelines' sampler
+    (UniPC) is named but not written out.  Reading used here, with
+    h_i = sigma_{i+1} - sigma_i and v_i = p, the guided prediction the routed
+    model made at the latent x_i it was given:
+      corrector (i >= 1): xc_i = xc_{i-1} + (h_{i-1} / 2) (v_{i-1} + v_i)
+                          (trapezoid over [sigma_{i-1}, sigma_i]);  xc_0 = x_0;
+      predictor:          x_{i+1} = xc_i + h_i v_i                       (i = 0)
+                          x_{i+1} = xc_i + h_i ((1 + r/2) v_i - (r/2) v_{i-1}),
+                          r = h_i / h_{i-1}                              (i >= 1)
+                          (v extrapolated linearly from the last two steps).
+    The one evaluation at the predicted x_i serves both the corrector of step
+    i and the predictor of step i+1, so the scheme costs one denoiser call per
+    step, whichever model makes it.  state = h_i = (xc_{i-1}, v_{i-1}), None
+    at i = 0.  Returns (x_{i+1}, h_{i+1}) in fp64.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    v = np.asarray(p, dtype=np.float64)
+    h = float(sigmas[i + 1]) - float(sigmas[i])
+    if state is None:
+        xc = x
+        x_next = xc + h * v
+    else:
+        xc_prev, v_prev = state
+        h_prev = float(sigmas[i]) - float(sigmas[i - 1])
+        xc = xc_prev + 0.5 * h_prev * (v_prev + v)
+        r = h / h_prev
+        x_next = xc + h * ((1.0 + 0.5 * r) * v - 0.5 * r * v_prev)
+    return x_next, (xc, v)
+
+
 # ---------------------------------------------------------------------------
 # Guidance (Eq. 1)
 # ---------------------------------------------------------------------------
@@ -229,6 +264,18 @@ def calibrate(large, small, x_T, conds, unconds, w, sigmas, eps: float = 1e-8):
             x = euler_update(x, p_l, sigmas[k], sigmas[k + 1])
         finals.append(x)
     return r, np.stack(finals)
+
+
+def sample_routed_multistep(large, small, policy, x_T, cond, uncond, w, sigmas, counter=None):
+    """Eq. 3 with the multistep scheduler: the history h_i evolves exactly as in
+    an all-large run, whichever model supplied each p (Sec. 3.1)."""
+    x = np.asarray(x_T, dtype=np.float64)
+    state = None
+    for i in range(len(sigmas) - 1):
+        m = small if policy[i] else large
+        p = guided_prediction(m, x, sigmas[i], cond, uncond, w, counter)
+        x, state = multistep_update(i, x, p, state, sigmas)
+    return x
 
 
 def sample_routed(large, small, policy, x_T, cond, uncond, w, sigmas, counter=None):

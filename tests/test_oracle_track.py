@@ -266,3 +266,120 @@ def test_equal_budget_policies():
     for seed in range(4000):
         counts += track.random_k_policy(n, k, seed)
     assert np.allclose(counts / 4000, k / n, atol=0.03)
+
+
+# ---------------------------------------------------------------------------
+# Multistep scheduler with history h_i (Eq. 2), routed (Sec. 3.1)
+# ---------------------------------------------------------------------------
+
+
+def _drive(update, field, sig, x0):
+    """Runs a scheduler update over the grid with v_i = field(x_i, sigma_i)."""
+    x, state = np.asarray(x0, np.float64), None
+    for i in range(len(sig) - 1):
+        x, state = update(i, x, field(x, float(sig[i])), state, sig)
+    return x
+
+
+@pytest.mark.parametrize("n,shift", [(2, 5.0), (4, 5.0), (7, 3.0), (50, 5.0)])
+def test_multistep_integrates_sigma_linear_fields_exactly(n, shift):
+    # For v = a + b*sigma the ODE integral is x_0 + a*(s_N - s_0) + b*(s_N^2 - s_0^2)/2:
+    # the trapezoid corrector and the linear-extrapolation predictor are both exact
+    # for a linear integrand, on the shifted (non-uniform) grid.  Euler is not.
+    rng = np.random.default_rng(n)
+    a, b, x0 = rng.normal(size=(3, 17))
+    sig = track.schedule(n, shift)
+    s0, sN = float(sig[0]), float(sig[-1])
+    exact = x0 + a * (sN - s0) + b * (sN * sN - s0 * s0) / 2
+    got = _drive(track.multistep_update, lambda x, s: a + b * s, sig, x0)
+    assert np.allclose(got, exact, rtol=0, atol=1e-12)
+    if n > 1:
+        euler = _drive(lambda i, x, p, st, sg: (track.euler_update(x, p, sg[i], sg[i + 1]), None),
+                       lambda x, s: a + b * s, sig, x0)
+        assert np.max(np.abs(euler - exact)) > 1e-3
+
+
+def test_multistep_is_second_order():
+    # dx/dsigma = lam * x from sigma = 1 to 0: x_N = x_0 * exp(-lam).  The global
+    # error falls 4x per halving of the step (the model is evaluated at the
+    # predicted latent, as the scheme prescribes); Euler's falls 2x.
+    lam, x0 = 1.3, np.array([0.7, -1.1])
+    exact = x0 * math.exp(-lam)
+    def err(upd, n):
+        return np.max(np.abs(_drive(upd, lambda x, s: lam * x, track.schedule(n, 1.0), x0) - exact))
+    e = [err(track.multistep_update, n) for n in (64, 128, 256)]
+    assert 3.6 < e[0] / e[1] < 4.4 and 3.6 < e[1] / e[2] < 4.4
+    eu = lambda i, x, p, st, sg: (track.euler_update(x, p, sg[i], sg[i + 1]), None)
+    assert 1.8 < err(eu, 64) / err(eu, 128) < 2.2
+
+
+def test_multistep_single_step_and_constant_field():
+    rng = np.random.default_rng(3)
+    x0, c = rng.normal(size=(2, 5))
+    sig = track.schedule(1, 5.0)
+    one = _drive(track.multistep_update, lambda x, s: c, sig, x0)
+    assert np.array_equal(one, track.euler_update(x0, c, sig[0], sig[1]))   # no history yet
+    for n in (3, 9):
+        got = _drive(track.multistep_update, lambda x, s: c, track.schedule(n, 5.0), x0)
+        assert np.allclose(got, x0 - c, rtol=0, atol=1e-14)                 # sum of steps = -1
+
+
+def test_multistep_history_survives_model_switches(samples):
+    # Two distinct model objects computing the same function: any routing must give
+    # the single-model trajectory, which fails if a switch touched the history.
+    L = dit.DiT(ARCH_L, synth.make_weights(ARCH_L, 11), name="L")
+    S = dit.DiT(ARCH_L, synth.make_weights(ARCH_L, 11), name="S")
+    x, c, u = samples
+    sig = track.schedule(5, 5.0)
+    ref = track.sample_routed_multistep(L, S, np.zeros(5, np.uint8), x[0], c[0], u[0], 5.0, sig)
+    cnt = {}
+    got = track.sample_routed_multistep(L, S, np.uint8([0, 1, 1, 0, 1]), x[0], c[0], u[0], 5.0,
+                                        sig, counter=cnt)
+    assert np.array_equal(got, ref)
+    assert cnt == {"L": 2 * 2, "S": 3 * 2}     # still exactly one model per step
+
+
+def test_multistep_mutants_are_caught(samples):
+    # Plausible slips each fail one of the pins above.
+    L = dit.DiT(ARCH_L, synth.make_weights(ARCH_L, 11), name="L")
+    S = dit.DiT(ARCH_L, synth.make_weights(ARCH_L, 11), name="S")
+    x, c, u = samples
+    sig = track.schedule(5, 5.0)
+    # (1) history reset whenever the model changes
+    def reset_on_switch(pol):
+        xx, st, prev = np.asarray(x[0], np.float64), None, None
+        for i in range(5):
+            m = S if pol[i] else L
+            if prev is not None and m is not prev:
+                st = None
+            p = track.guided_prediction(m, xx, sig[i], c[0], u[0], 5.0)
+            if st is None and i > 0:   # restart: Euler from here, as a fresh scheduler would
+                xx, st = xx + (float(sig[i + 1]) - float(sig[i])) * p, (xx, p)
+            else:
+                xx, st = track.multistep_update(i, xx, p, st, sig)
+            prev = m
+        return xx
+    ref = track.sample_routed_multistep(L, S, np.zeros(5, np.uint8), x[0], c[0], u[0], 5.0, sig)
+    assert not np.array_equal(reset_on_switch(np.uint8([0, 1, 1, 0, 1])), ref)
+    # (2) step ratio inverted, (3) corrector dropped: the sigma-linear pin fails
+    rng = np.random.default_rng(0)
+    a, b, x0 = rng.normal(size=(3, 9))
+    g = track.schedule(6, 5.0)
+    exact = x0 + a * (float(g[-1]) - float(g[0])) + b * (float(g[-1]) ** 2 - float(g[0]) ** 2) / 2
+    def inverted(i, xx, p, st, sg):
+        if st is None:
+            return xx + (float(sg[i + 1]) - float(sg[i])) * p, (xx, p)
+        xc_prev, v_prev = st
+        hp, h = float(sg[i]) - float(sg[i - 1]), float(sg[i + 1]) - float(sg[i])
+        xc = xc_prev + 0.5 * hp * (v_prev + p)
+        r = hp / h
+        return xc + h * ((1 + r / 2) * p - (r / 2) * v_prev), (xc, p)
+    def no_corrector(i, xx, p, st, sg):
+        if st is None:
+            return xx + (float(sg[i + 1]) - float(sg[i])) * p, (xx, p)
+        _, v_prev = st
+        hp, h = float(sg[i]) - float(sg[i - 1]), float(sg[i + 1]) - float(sg[i])
+        r = h / hp
+        return xx + h * ((1 + r / 2) * p - (r / 2) * v_prev), (xx, p)
+    for wrong in (inverted, no_corrector):
+        assert np.max(np.abs(_drive(wrong, lambda xx, s: a + b * s, g, x0) - exact)) > 1e-4
