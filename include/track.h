@@ -236,6 +236,30 @@ int track_sample(track_model* large, track_model* small, const uint8_t* policy,
                  const float* sigmas, int n_steps, float* x, int B, const float* cond,
                  const float* uncond, float cfg_scale, track_stream s);
 
+/* Eq. 2 with a scheduler history h_i (Sec. 3.1 allows any multistep solver and
+ * TRACK keeps its state evolution unchanged across model switches): one step
+ * of the second-order predictor-corrector for dx/dsigma = v.  With
+ * h_i = sigmas[i+1] - sigmas[i] and r = h_i / h_{i-1}:
+ *   i = 0:  xc = x,                                x <- xc + h_i v
+ *   i > 0:  xc = xc' + (h_{i-1}/2) (v' + v),       x <- xc + h_i ((1 + r/2) v - (r/2) v')
+ * where (xc', v') is the history from step i-1; then the history becomes
+ * (xc, v).  x: device fp32 [n] in/out (in: the latent the model saw at step
+ * i, out: the next one); v: device fp32 [n], the guided prediction made at x;
+ * state: device fp32 [2 n], the corrected latent then the previous velocity,
+ * caller-owned, read only for i > 0.  sigmas: host (n_steps + 1).  EINVAL for
+ * i outside [0, n_steps) or v aliasing x or state.  The paper gives no
+ * formulas for its pipelines' UniPC sampler; this scheme is the reading used. */
+int track_multistep_step(float* x, const float* v, float* state, int64_t n, const float* sigmas,
+                         int n_steps, int i, track_stream s);
+
+/* Eq. 3 over the multistep scheduler of track_multistep_step: policy[i] picks
+ * the model for step i, and the history runs through switches untouched.
+ * state: device fp32 [2, B, C, F, H, W] scratch, caller-owned (contents on
+ * entry ignored; on return, the history after the last step). */
+int track_sample_multistep(track_model* large, track_model* small, const uint8_t* policy,
+                           const float* sigmas, int n_steps, float* x, int B, const float* cond,
+                           const float* uncond, float cfg_scale, float* state, track_stream s);
+
 /* track_sample through a CUDA graph.  It computes the same values bit for bit,
  * with the text projection of cond/uncond recomputed on every call.  The
  * library keeps up to 32 recorded graphs, keyed by every argument (models,

@@ -84,6 +84,8 @@ def lib():
         "track_calibrate": (_I, [_P, _P, _P, _I, _P, _P, _F, _P, _I, _F, _P, _P]),
         "track_sample": (_I, [_P, _P, _P, _P, _I, _P, _I, _P, _P, _F, _P]),
         "track_sample_graph": (_I, [_P, _P, _P, _P, _I, _P, _I, _P, _P, _F, _P]),
+        "track_multistep_step": (_I, [_P, _P, _P, ctypes.c_int64, _P, _I, _I, _P]),
+        "track_sample_multistep": (_I, [_P, _P, _P, _P, _I, _P, _I, _P, _P, _F, _P, _P]),
         "track_linear": (_I, [_I, _P, _P, _P, _I, _I, _I, _I, _P, _P, _I, _P]),
         "track_attention": (_I, [_I, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P]),
     }
@@ -366,6 +368,34 @@ def track_sample(large: Model, small: Model, policy, sigmas, x, cond, uncond, cf
                               pol.shape[0], _ptr(x), x.shape[0], _ptr(cond), _ptr(uncond),
                               cfg_scale, _stream(stream)))
     return x
+
+
+def track_multistep_step(x, v, state, sigmas, i, stream=None):
+    """Step i of the history-carrying scheduler on device fp32 tensors; state has 2 * x.numel()."""
+    sig = np.ascontiguousarray(sigmas, dtype=np.float32)
+    n = x.numel()
+    if state.numel() != 2 * n or v.numel() != n:
+        raise ValueError("state must hold 2 * n floats and v n floats")
+    _check(lib().track_multistep_step(_ptr(x), _ptr(v), _ptr(state), n, sig.ctypes.data,
+                                      sig.shape[0] - 1, int(i), _stream(stream)))
+    return x
+
+
+def track_sample_multistep(large: Model, small: Model, policy, sigmas, x, cond, uncond, cfg_scale,
+                           state=None, stream=None):
+    """Eq. 3 over the multistep scheduler; returns (x, state)."""
+    import torch
+    pol = np.ascontiguousarray(policy, dtype=np.uint8)
+    sig = np.ascontiguousarray(sigmas, dtype=np.float32)
+    if pol.shape[0] != sig.shape[0] - 1:
+        raise ValueError("policy needs one entry per step")
+    if state is None:
+        state = torch.empty((2,) + tuple(x.shape), dtype=torch.float32, device=x.device)
+    _check(lib().track_sample_multistep(large.handle, small.handle, pol.ctypes.data,
+                                        sig.ctypes.data, pol.shape[0], _ptr(x), x.shape[0],
+                                        _ptr(cond), _ptr(uncond), cfg_scale, _ptr(state),
+                                        _stream(stream)))
+    return x, state
 
 
 def track_sample_graph(large: Model, small: Model, policy, sigmas, x, cond, uncond, cfg_scale,

@@ -161,6 +161,11 @@ cudaError_t head_unpatchify(const float* xres, int nseq, int L, int d, const flo
 cudaError_t cfg_combine(const float* fc, const float* fu, int64_t n, float w, float* p,
                         cudaStream_t s);
 cudaError_t euler_step(float* x, const float* v, int64_t n, float dsig, cudaStream_t s);
+// Step i of the second-order predictor-corrector scheduler (Eq. 2 with history):
+// x (the latent the model saw) becomes x_{i+1}; (xc, vp) is the history,
+// read for i > 0 and rewritten.  sigmas: host.
+cudaError_t multistep_step(float* x, const float* v, float* xc, float* vp, int64_t n,
+                           const float* sigmas, int i, cudaStream_t s);
 cudaError_t cfg_euler(float* x, const float* fc, const float* fu, int64_t n, float w, float dsig,
                       cudaStream_t s);
 // Eq. 4: partial sums then a fixed-order final combine; scratch holds B*nblk*2 floats.

@@ -1131,6 +1131,42 @@ static void drop_graphs_of(const track_model* m) {
   }
 }
 
+int track_multistep_step(float* x, const float* v, float* state, int64_t n, const float* sigmas,
+                         int n_steps, int i, track_stream s) {
+  if (!x || !v || !state || !sigmas) return fail(TRACK_EINVAL, "NULL pointer");
+  if (n < 0 || n_steps < 1 || i < 0 || i >= n_steps) return fail(TRACK_EINVAL, "bad step index");
+  if ((((uintptr_t)x) | ((uintptr_t)v) | ((uintptr_t)state)) & 15)
+    return fail(TRACK_EINVAL, "device pointers must be 16-byte aligned");
+  if (v == x || v == state || v == state + n) return fail(TRACK_EINVAL, "v may not alias x or state");
+  LAUNCH(multistep_step(x, v, state, state + n, n, sigmas, i, (cudaStream_t)s));
+  return TRACK_OK;
+}
+
+int track_sample_multistep(track_model* large, track_model* small, const uint8_t* policy,
+                           const float* sigmas, int n_steps, float* x, int B, const float* cond,
+                           const float* uncond, float cfg_scale, float* state, track_stream s) {
+  if (!large || !small) return fail(TRACK_EINVAL, "model is NULL");
+  if (track_models_compatible(large, small) != 1)
+    return fail(TRACK_EINVAL, "models are not a compatible pair");
+  if (!policy || !sigmas || n_steps < 1 || !state) return fail(TRACK_EINVAL, "bad arguments");
+  if (((uintptr_t)state) & 15) return fail(TRACK_EINVAL, "state must be 16-byte aligned");
+  TRACK_TRY(check_denoise_args(large, x, B, cond, uncond, cfg_scale, x));
+  TRACK_TRY(set_device(large));
+  const cudaStream_t st = (cudaStream_t)s;
+  const int64_t n = (int64_t)B * large->latent_n;
+  const int nseq = cfg_scale == 1.f ? B : 2 * B;
+  for (int i = 0; i < n_steps; ++i) {
+    track_model* m = policy[i] ? small : large;
+    TRACK_TRY(ensure_workspace(m, nseq));
+    float* p = m->ws.fout;
+    TRACK_TRY(forward(m, x, B, nseq, 1000.f * sigmas[i], cond, cfg_scale == 1.f ? nullptr : uncond,
+                      p, st));
+    if (cfg_scale != 1.f) LAUNCH(cfg_combine(p, p + n, n, cfg_scale, p, st));  // in place
+    LAUNCH(multistep_step(x, p, state, state + n, n, sigmas, i, st));
+  }
+  return TRACK_OK;
+}
+
 int track_sample_graph(track_model* large, track_model* small, const uint8_t* policy,
                        const float* sigmas, int n_steps, float* x, int B, const float* cond,
                        const float* uncond, float cfg_scale, track_stream s) {

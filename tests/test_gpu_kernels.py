@@ -327,6 +327,29 @@ def test_attention_single_key_returns_value_row(T):
         assert np.array_equal(got[0, :, h, :], np.repeat(V[0, h], 70, 0))
 
 
+# ---------------------------------------------------------------- multistep scheduler (Eq. 2)
+@pytest.mark.parametrize("n", [1, 3, 4096 + 3, 2_096_640])
+def test_multistep_step_matches_oracle(T, n):
+    rng = np.random.default_rng(n + 5)
+    sig = track.schedule(4, 5.0)
+    x = rng.normal(size=n).astype(np.float32)
+    xd = dev_f32(x)
+    state = torch.full((2 * n,), float("nan"), device=DEV)   # step 0 must not read it
+    xr, st = x.astype(np.float64), None
+    for i in range(4):
+        v = rng.normal(size=n).astype(np.float32)
+        T.track_multistep_step(xd, dev_f32(v), state, sig, i)
+        T.track_sync()
+        xr, st = track.multistep_update(i, xr, v, st, sig)
+        assert rel_l2(xd.cpu().numpy(), xr) < 1e-6
+        xr = xd.cpu().numpy().astype(np.float64)   # continue from the GPU's own values
+        st = tuple(a.cpu().numpy().astype(np.float64) for a in state.view(2, n))
+    with pytest.raises(T.TrackError):
+        T.track_multistep_step(xd, xd, state, sig, 0)          # v aliases x
+    with pytest.raises(T.TrackError):
+        T.track_multistep_step(xd, dev_f32(x), state, sig, 4)  # step index out of range
+
+
 # ---------------------------------------------------------------- guidance, Euler, Eq. 4
 @pytest.mark.parametrize("n", [1, 3, 4096 + 3, 2_096_640])
 def test_guidance_and_euler(T, n):

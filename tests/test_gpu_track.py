@@ -175,6 +175,41 @@ def test_routed_sampling_follows_the_oracle(T, tiny, calib_inputs, oracle_calibr
     assert cnt == {"L": 2 * 2 * int((pol == 0).sum()), "S": 2 * 2 * int(pol.sum())}
 
 
+def test_multistep_routed_sampling_follows_the_oracle(T, tiny, calib_inputs, oracle_calibration):
+    prec, P = tiny
+    _, _, r_ref = oracle_calibration
+    pol = track.topk_policy(track.mean_score(r_ref), WL.k)
+    x, c, u = synth.evaluation_inputs(WL.large, 0, 2, with_uncond=True)
+    sig = track.schedule(WL.steps, WL.shift)
+    xd = dev(x)
+    T.track_sample_multistep(P.L, P.S, pol, sig, xd, dev(c), dev(u), WL.cfg)
+    T.track_sync()
+    for j in range(2):
+        ref = track.sample_routed_multistep(P.oL, P.oS, pol, x[j], c[j], u[j], WL.cfg, sig)
+        assert rel_l2(xd[j].cpu().numpy(), ref) < (1e-3 if prec == "fp32" else 5e-2)
+    # the history is kept across switches: differs from the Euler trajectory
+    xe = dev(x)
+    T.track_sample(P.L, P.S, pol, sig, xe, dev(c), dev(u), WL.cfg)
+    T.track_sync()
+    assert not torch.equal(xe, xd)
+
+
+def test_multistep_identities_bit_exact(T, calib_inputs):
+    # Two distinct models with identical weights: any routing reproduces the
+    # single-model trajectory bit for bit (a history reset at a switch would not).
+    P = Pair(T, "fp32", small_seed=synth.SEED_LARGE, small_arch=WL.large)
+    x, c, u = calib_inputs
+    sig = track.schedule(WL.steps, WL.shift)
+    ref = dev(x[:2])
+    T.track_sample_multistep(P.L, P.S, np.zeros(WL.steps, np.uint8), sig, ref, dev(c[:2]),
+                             dev(u[:2]), WL.cfg)
+    got = dev(x[:2])
+    pol = np.array([0, 1, 1, 0, 1, 0, 1, 1][:WL.steps], np.uint8)
+    T.track_sample_multistep(P.L, P.S, pol, sig, got, dev(c[:2]), dev(u[:2]), WL.cfg)
+    T.track_sync()
+    assert torch.equal(got, ref)
+
+
 def test_graph_replay_matches_eager(T, tiny):
     # First call eager, second records and replays, later calls replay: every
     # call must equal an eager run bit for bit, with the buffers' current
