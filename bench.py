@@ -431,6 +431,24 @@ def run_ours(args):
         prime(pol)
         t, _ = timed(step_device, pol, nsw)
         equal_budget[name] = {"ms": t / nsw, "policy": "".join("S" if p else "L" for p in pol)}
+    # The same routed and all-large trajectories over the history-carrying
+    # multistep scheduler (Eq. 2 with h_i), launched kernel by kernel.
+    ms_state = torch.empty(2 * xd.numel(), dtype=torch.float32, device=dev)
+
+    def step_multistep(pol):
+        xd.copy_(x_init)
+        T.track_invalidate_ctx(L)
+        T.track_invalidate_ctx(S)
+        T.track_sample_multistep(L, S, pol, sig, xd, cd, ud, w, state=ms_state, stream=sid)
+
+    multistep = {}
+    for name, pol in (("routed", policy), ("all_large", all_l)):
+        step_multistep(pol)
+        t, _ = timed(step_multistep, pol, nsw)
+        multistep[name + "_ms"] = t / nsw
+    multistep["speedup"] = multistep["all_large_ms"] / multistep["routed_ms"]
+    multistep["scheduler"] = "second-order predictor-corrector with history (Eq. 2 h_i)"
+
     for _ in range(max(1, args.warmup // 2)):
         step_e2e(policy)
     ms_e2e, _ = timed(step_e2e, policy, args.steps)
@@ -505,6 +523,7 @@ def run_ours(args):
             "latency_vs_k": sweep,
             "cost_model": {"C_large_ms": c_l, "C_small_ms": c_s, "max_rel_err": cost_err},
             "equal_budget_K": wl.k, "equal_budget": equal_budget,
+            "multistep": multistep,
             "score_map": [float(v) for v in q],
             "roofline": roof,
             "cpu_baseline": cpu,
@@ -568,14 +587,20 @@ def run_kernel(args):
                       lambda: T.track_attention(T.BF16, Q, Kc, Vc, O)))
     elif args.kernel == "hbm":
         # HBM-bound kernels of the public C ABI, algorithmic bytes per call: fused
-        # guidance + Euler update 16 B/elem (read f_c, f_u, x; write x), Eq. 4
-        # reduction 8 B/elem (read p_L, p_S).  The normalization kernels inside the
-        # denoiser are measured in place by the full benchmark.
+        # guidance + Euler update 16 B/elem (read f_c, f_u, x; write x), multistep
+        # update 28 B/elem (read x, v and the two history arrays; write x and the
+        # history), Eq. 4 reduction 8 B/elem (read p_L, p_S).  The normalization
+        # kernels inside the denoiser are measured in place by the full benchmark.
         n480 = 16 * 21 * 60 * 104
         for label, n in (("480p latent x2 (CFG batch)", 2 * n480), ("1 Gi elements", 1 << 30)):
             fc, fu, xx = (torch.randn(n, device="cuda") for _ in range(3))
             cases.append(("cfg_euler", f"{label}: n={n}", 16.0 * n,
                           lambda fc=fc, fu=fu, xx=xx: T.track_cfg_step(xx, fc, fu, 5.0, 0.5, 0.45)))
+            st = torch.zeros(2 * n, device="cuda")
+            sg = T.track_schedule(4, 5.0)
+            T.track_multistep_step(xx, fc, st, sg, 0)      # history for the timed step 1
+            cases.append(("multistep", f"{label}: n={n}", 28.0 * n,
+                          lambda xx=xx, fc=fc, st=st, sg=sg: T.track_multistep_step(xx, fc, st, sg, 1)))
             B = 2 if n == 2 * n480 else 8
             acc = torch.zeros(B, device="cuda")
             cases.append(("disagreement", f"{label}: B={B} n={n // B}", 8.0 * n,
