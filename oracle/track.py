@@ -113,6 +113,61 @@ def disagreement(p_large, p_small, eps: float = 1e-8) -> float:
     return num / den
 
 
+def band_index(k: int, n: int) -> int:
+    """|signed frequency| of DFT bin k of an n-point transform (numpy's fftfreq * n)."""
+    return min(k, n - k)
+
+
+def spatial_band(kh: int, kw: int, H: int, W: int) -> int:
+    """Band 0/1/2 (low/mid/high) of spatial bin (kh, kw): the radius of the normalized
+    frequency (|kh|/H, |kw|/W) in units of Nyquist (0.5) against 1/3 and 2/3, decided
+    in integer arithmetic: rho^2 = 4 (kh^2/H^2 + kw^2/W^2)."""
+    a, b = band_index(kh, H), band_index(kw, W)
+    num = 4 * (a * a * W * W + b * b * H * H)   # rho^2 * H^2 W^2
+    den = H * H * W * W
+    if 9 * num < den:
+        return 0
+    if 9 * num < 4 * den:
+        return 1
+    return 2
+
+
+def temporal_band(kf: int, F: int) -> int:
+    """Band 0/1/2 of temporal bin kf: |kf|/F in units of Nyquist against 1/3 and 2/3."""
+    a = band_index(kf, F)
+    if 6 * a < F:
+        return 0
+    if 3 * a < F:
+        return 1
+    return 2
+
+
+def band_disagreement(p_large, p_small, eps: float = 1e-8) -> np.ndarray:
+    """Sec. 4.4: Eq. 4's disagreement split over frequency bands with an orthonormal
+    Fourier transform, for one sample of shape [C, F, H, W].
+
+    D = p_S - p_L is transformed over (F, H, W) per channel (orthonormal, so
+    sum |D^|^2 = sum D^2); each bin's energy goes to one spatial band (radius of
+    the (h, w) frequency in units of Nyquist: low < 1/3 <= mid < 2/3 <= high) and
+    one temporal band (|f| frequency, same thirds).  The paper gives no band
+    edges; these are the reading used.  Returns [6]: spatial low/mid/high then
+    temporal low/mid/high, each sqrt(band energy) / max(||p_L||, eps), so that
+    the squares of each triple add up to r^2 of Eq. 4.
+    """
+    pl = np.asarray(p_large, dtype=np.float64)
+    d = np.asarray(p_small, dtype=np.float64) - pl
+    C, F, H, W = d.shape
+    e2 = np.abs(np.fft.fftn(d, axes=(1, 2, 3), norm="ortho")) ** 2
+    sp = np.array([[spatial_band(kh, kw, H, W) for kw in range(W)] for kh in range(H)])
+    tb = np.array([temporal_band(kf, F) for kf in range(F)])
+    out = np.zeros(6)
+    for band in range(3):
+        out[band] = e2[:, :, sp == band].sum()
+        out[3 + band] = e2[:, tb == band, :, :].sum()
+    den = max(math.sqrt(float(np.dot(pl.ravel(), pl.ravel()))), eps)
+    return np.sqrt(out) / den
+
+
 def mean_score(r) -> np.ndarray:
     """Eq. 5: q_k = (1/M) sum_j r_{j,k}; r has shape [M, N].  Returned as fp32."""
     r = np.asarray(r, dtype=np.float64)

@@ -383,3 +383,82 @@ def test_multistep_mutants_are_caught(samples):
         return xx + h * ((1 + r / 2) * p - (r / 2) * v_prev), (xx, p)
     for wrong in (inverted, no_corrector):
         assert np.max(np.abs(_drive(wrong, lambda xx, s: a + b * s, g, x0) - exact)) > 1e-4
+
+
+# ---------------------------------------------------------------------------
+# Frequency-band decomposition of the disagreement (Sec. 4.4)
+# ---------------------------------------------------------------------------
+
+
+@pytest.mark.parametrize("shape", [(1, 1, 1, 1), (2, 3, 4, 5), (16, 9, 30, 52), (3, 4, 6, 8)])
+def test_band_disagreement_parseval(shape):
+    # The transform is orthonormal, so each band triple's squares add up to r^2 of Eq. 4.
+    rng = np.random.default_rng(sum(shape))
+    pl, ps = rng.normal(size=(2,) + shape)
+    b = track.band_disagreement(pl, ps)
+    r = track.disagreement(pl, ps)
+    assert b.shape == (6,) and np.all(b >= 0)
+    assert abs(float(np.sum(b[:3] ** 2)) - r * r) < 1e-12 * r * r
+    assert abs(float(np.sum(b[3:] ** 2)) - r * r) < 1e-12 * r * r
+
+
+def test_band_disagreement_brute_force_dft():
+    # A direct triple-loop DFT with the bands decided in floating point (no bin of
+    # this shape sits on a band edge) gives the same numbers.
+    rng = np.random.default_rng(7)
+    C, F, H, W = 2, 3, 4, 7
+    pl, ps = rng.normal(size=(2, C, F, H, W))
+    d = ps - pl
+    e_sp, e_t = np.zeros(3), np.zeros(3)
+    ff, hh, ww = np.meshgrid(np.arange(F), np.arange(H), np.arange(W), indexing="ij")
+    for c in range(C):
+        for kf in range(F):
+            for kh in range(H):
+                for kw in range(W):
+                    ph = np.exp(-2j * np.pi * (kf * ff / F + kh * hh / H + kw * ww / W))
+                    e = abs(np.sum(d[c] * ph)) ** 2 / (F * H * W)
+                    nf, nh, nw = (min(k, n - k) / n for k, n in ((kf, F), (kh, H), (kw, W)))
+                    rho_s, rho_t = math.hypot(nh, nw) / 0.5, nf / 0.5
+                    e_sp[0 if rho_s < 1 / 3 else 1 if rho_s < 2 / 3 else 2] += e
+                    e_t[0 if rho_t < 1 / 3 else 1 if rho_t < 2 / 3 else 2] += e
+    ref = np.sqrt(np.concatenate([e_sp, e_t])) / np.linalg.norm(pl)
+    assert np.allclose(track.band_disagreement(pl, ps), ref, rtol=1e-12, atol=0)
+
+
+@pytest.mark.parametrize("k,band", [(2, 0), (12, 1), (24, 2)])
+def test_band_disagreement_spatial_tone(k, band):
+    # A difference that is a pure horizontal tone of k cycles over W = 52 (radius
+    # 2k/52 of Nyquist) puts all its energy in that spatial band and, being
+    # constant over frames, in the low temporal band.
+    C, F, H, W = 2, 9, 30, 52
+    pl = np.ones((C, F, H, W))
+    tone = np.cos(2 * np.pi * k * np.arange(W) / W)
+    ps = pl + np.broadcast_to(tone, (C, F, H, W))
+    b = track.band_disagreement(pl, ps)
+    r = track.disagreement(pl, ps)
+    assert abs(b[band] - r) < 1e-12 * r and abs(b[3] - r) < 1e-12 * r
+    assert np.sum(np.delete(b[:3], band) ** 2) < 1e-24 * r * r
+
+
+@pytest.mark.parametrize("k,band", [(1, 0), (2, 1), (4, 2)])
+def test_band_disagreement_temporal_tone(k, band):
+    C, F, H, W = 1, 9, 6, 8
+    pl = np.ones((C, F, H, W))
+    tone = np.cos(2 * np.pi * k * np.arange(F) / F)[None, :, None, None]
+    ps = pl + np.broadcast_to(tone, (C, F, H, W))
+    b = track.band_disagreement(pl, ps)
+    r = track.disagreement(pl, ps)
+    assert abs(b[3 + band] - r) < 1e-12 * r and abs(b[0] - r) < 1e-12 * r
+
+
+def test_band_disagreement_special_cases_and_edges():
+    rng = np.random.default_rng(1)
+    pl = rng.normal(size=(3, 4, 6, 8))
+    assert np.all(track.band_disagreement(pl, pl) == 0.0)
+    b = track.band_disagreement(pl, pl + 0.5)            # a constant offset is all DC
+    assert b[1] == b[2] == b[4] == b[5] == 0.0 or max(b[1], b[2], b[4], b[5]) < 1e-12 * b[0]
+    # edges: exactly 1/3 of Nyquist belongs to mid, exactly 2/3 to high
+    assert track.spatial_band(0, 1, 4, 6) == 1          # |kw|/W = 1/6 -> rho = 1/3
+    assert track.spatial_band(0, 2, 4, 6) == 2          # rho = 2/3
+    assert track.temporal_band(1, 6) == 1 and track.temporal_band(2, 6) == 2
+    assert track.temporal_band(5, 6) == 1               # bin 5 of 6 is frequency -1
