@@ -236,6 +236,21 @@ int track_sample(track_model* large, track_model* small, const uint8_t* policy,
                  const float* sigmas, int n_steps, float* x, int B, const float* cond,
                  const float* uncond, float cfg_scale, track_stream s);
 
+/* Sec. 4.4: Eq. 4's disagreement split over frequency bands.  For each sample
+ * b, D = v_S - v_L ([C, F, H, W], fp32) is transformed by the orthonormal 3-D
+ * DFT over (F, H, W) per channel, and every bin's energy |D^|^2 goes to one
+ * spatial band (radius of the (h, w) frequency in units of Nyquist:
+ * low < 1/3 <= mid < 2/3 <= high) and one temporal band (|f| frequency in
+ * units of Nyquist, same thirds); the paper gives no band edges, these are the
+ * reading used.  bands_out[b * 6 + j] = sqrt(E_j) / max(||v_L[b]||, eps):
+ * j = 0..2 spatial low/mid/high, 3..5 temporal low/mid/high (each triple's
+ * squares add up to r^2 of Eq. 4).  v_L, v_S: device fp32 [B, C, F, H, W];
+ * bands_out: device fp32 [B, 6], overwritten.  Deterministic.  Uses scratch
+ * the library keeps per stream (4 B C F H W floats plus partials).
+ * EUNSUPPORTED for an axis longer than 512. */
+int track_band_disagreement(const float* v_L, const float* v_S, int B, int C, int F, int H, int W,
+                            float eps, float* bands_out, track_stream s);
+
 /* Eq. 2 with a scheduler history h_i (Sec. 3.1 allows any multistep solver and
  * TRACK keeps its state evolution unchanged across model switches): one step
  * of the second-order predictor-corrector for dx/dsigma = v.  With

@@ -85,6 +85,7 @@ def lib():
         "track_sample": (_I, [_P, _P, _P, _P, _I, _P, _I, _P, _P, _F, _P]),
         "track_sample_graph": (_I, [_P, _P, _P, _P, _I, _P, _I, _P, _P, _F, _P]),
         "track_multistep_step": (_I, [_P, _P, _P, ctypes.c_int64, _P, _I, _I, _P]),
+        "track_band_disagreement": (_I, [_P, _P, _I, _I, _I, _I, _I, _F, _P, _P]),
         "track_sample_multistep": (_I, [_P, _P, _P, _P, _I, _P, _I, _P, _P, _F, _P, _P]),
         "track_linear": (_I, [_I, _P, _P, _P, _I, _I, _I, _I, _P, _P, _I, _P]),
         "track_attention": (_I, [_I, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P]),
@@ -368,6 +369,18 @@ def track_sample(large: Model, small: Model, policy, sigmas, x, cond, uncond, cf
                               pol.shape[0], _ptr(x), x.shape[0], _ptr(cond), _ptr(uncond),
                               cfg_scale, _stream(stream)))
     return x
+
+
+def track_band_disagreement(v_L, v_S, eps=1e-8, out=None, stream=None):
+    """Sec. 4.4 band split of Eq. 4 for device fp32 [B, C, F, H, W] tensors -> [B, 6]
+    (spatial low/mid/high, temporal low/mid/high)."""
+    import torch
+    B, C, F, H, W = v_L.shape
+    if out is None:
+        out = torch.empty((B, 6), dtype=torch.float32, device=v_L.device)
+    _check(lib().track_band_disagreement(_ptr(v_L), _ptr(v_S), B, C, F, H, W, eps, _ptr(out),
+                                         _stream(stream)))
+    return out
 
 
 def track_multistep_step(x, v, state, sigmas, i, stream=None):

@@ -18,7 +18,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libtrack.so")
 SOURCES = ("elementwise.cu", "gemm_simt.cu", "gemm_tc.cu", "attention.cu", "attn_tc.cu",
-           "track_api.cu", "noalloc.cu")
+           "track_api.cu", "noalloc.cu", "bands.cu")
 ARCH_FLAGS = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE]
 

@@ -168,6 +168,12 @@ cudaError_t multistep_step(float* x, const float* v, float* xc, float* vp, int64
                            const float* sigmas, int i, cudaStream_t s);
 cudaError_t cfg_euler(float* x, const float* fc, const float* fu, int64_t n, float w, float dsig,
                       cudaStream_t s);
+// Sec. 4.4 frequency-band split of Eq. 4 (see bands.cu): out [B, 6] device fp32;
+// scratch holds band_scratch_floats(B, C, F, H, W) floats.
+size_t band_scratch_floats(int B, int C, int F, int H, int W);
+cudaError_t band_disagreement(const float* vL, const float* vS, int B, int C, int F, int H, int W,
+                              float eps, float* out, float* scratch, cudaStream_t s);
+
 // Eq. 4: partial sums then a fixed-order final combine; scratch holds B*nblk*2 floats.
 int disagreement_blocks(int64_t n_per_sample);
 cudaError_t disagreement(const float* vL, const float* vS, int B, int64_t n, float eps,

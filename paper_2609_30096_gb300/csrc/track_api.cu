@@ -689,6 +689,14 @@ static float* stream_scratch(cudaStream_t s, size_t floats) {
   return p;
 }
 
+static int band_impl(const float* vL, const float* vS, int B, int C, int F, int H, int W,
+                     float eps, float* out, cudaStream_t s) {
+  float* scr = stream_scratch(s, band_scratch_floats(B, C, F, H, W));
+  if (scr == nullptr) return fail(TRACK_ENOMEM, "band scratch allocation failed");
+  LAUNCH(band_disagreement(vL, vS, B, C, F, H, W, eps, out, scr, s));
+  return TRACK_OK;
+}
+
 static int disagreement_impl(const float* vL, const float* vS, int B, int64_t n, float eps,
                              float* accum, cudaStream_t s) {
   const int nblk = disagreement_blocks(n);
@@ -1129,6 +1137,15 @@ static void drop_graphs_of(const track_model* m) {
       ++i;
     }
   }
+}
+
+int track_band_disagreement(const float* v_L, const float* v_S, int B, int C, int F, int H, int W,
+                            float eps, float* bands_out, track_stream s) {
+  if (!v_L || !v_S || !bands_out) return fail(TRACK_EINVAL, "NULL pointer");
+  if (B < 0 || C <= 0 || F <= 0 || H <= 0 || W <= 0) return fail(TRACK_EINVAL, "bad shape");
+  if (F > 512 || H > 512 || W > 512) return fail(TRACK_EUNSUPPORTED, "axes longer than 512");
+  if (!(eps >= 0.f)) return fail(TRACK_EINVAL, "eps must be non-negative");
+  return band_impl(v_L, v_S, B, C, F, H, W, eps, bands_out, (cudaStream_t)s);
 }
 
 int track_multistep_step(float* x, const float* v, float* state, int64_t n, const float* sigmas,

@@ -327,6 +327,42 @@ def test_attention_single_key_returns_value_row(T):
         assert np.array_equal(got[0, :, h, :], np.repeat(V[0, h], 70, 0))
 
 
+# ---------------------------------------------------------------- frequency bands (Sec. 4.4)
+@pytest.mark.parametrize("shape", [(1, 16, 9, 30, 52), (2, 3, 4, 5, 7), (3, 1, 1, 1, 1),
+                                   (1, 16, 21, 60, 104)])
+def test_band_disagreement_matches_oracle(T, shape):
+    rng = np.random.default_rng(sum(shape))
+    vl = rng.normal(size=shape).astype(np.float32)
+    vs = (vl + 0.3 * rng.normal(size=shape)).astype(np.float32)
+    outs = []
+    for _ in range(2):
+        out = T.track_band_disagreement(dev_f32(vl), dev_f32(vs))
+        T.track_sync()
+        outs.append(out.cpu().numpy())
+    assert np.array_equal(outs[0], outs[1])                     # deterministic
+    for b in range(shape[0]):
+        ref = track.band_disagreement(vl[b], vs[b])
+        assert np.allclose(outs[0][b], ref, rtol=1e-5, atol=1e-6 * np.max(ref))
+
+
+def test_band_disagreement_tones(T):
+    C, F, H, W = 2, 9, 30, 52
+    vl = np.ones((3, C, F, H, W), np.float32)
+    vs = vl.copy()
+    vs[0] += np.cos(2 * np.pi * 12 * np.arange(W) / W).astype(np.float32)         # spatial mid
+    vs[1] += np.cos(2 * np.pi * 4 * np.arange(F) / F).astype(np.float32)[:, None, None]  # temporal high
+    vs[2] += 0.25                                                                   # DC only
+    out = T.track_band_disagreement(dev_f32(vl), dev_f32(vs)).cpu().numpy()
+    r = [track.disagreement(vl[b], vs[b]) for b in range(3)]
+    assert abs(out[0, 1] - r[0]) < 1e-5 * r[0] and max(out[0, 0], out[0, 2]) < 1e-3 * r[0]
+    assert abs(out[1, 5] - r[1]) < 1e-5 * r[1] and max(out[1, 3], out[1, 4]) < 1e-3 * r[1]
+    assert abs(out[2, 0] - r[2]) < 1e-5 * r[2] and abs(out[2, 3] - r[2]) < 1e-5 * r[2]
+    with pytest.raises(T.TrackError) as e:
+        T.track_band_disagreement(dev_f32(np.ones((1, 1, 1, 1, 600))),
+                                  dev_f32(np.ones((1, 1, 1, 1, 600))))
+    assert e.value.code == T.TRACK_EUNSUPPORTED
+
+
 # ---------------------------------------------------------------- multistep scheduler (Eq. 2)
 @pytest.mark.parametrize("n", [1, 3, 4096 + 3, 2_096_640])
 def test_multistep_step_matches_oracle(T, n):
