@@ -589,8 +589,10 @@ def run_kernel(args):
         # HBM-bound kernels of the public C ABI, algorithmic bytes per call: fused
         # guidance + Euler update 16 B/elem (read f_c, f_u, x; write x), multistep
         # update 28 B/elem (read x, v and the two history arrays; write x and the
-        # history), Eq. 4 reduction 8 B/elem (read p_L, p_S).  The normalization
-        # kernels inside the denoiser are measured in place by the full benchmark.
+        # history), Eq. 4 reduction 8 B/elem (read p_L, p_S), its frequency-band
+        # split 8 B/elem (read p_L, p_S; the three DFT passes keep their complex
+        # intermediates in L2-sized scratch).  The normalization kernels inside the
+        # denoiser are measured in place by the full benchmark.
         n480 = 16 * 21 * 60 * 104
         for label, n in (("480p latent x2 (CFG batch)", 2 * n480), ("1 Gi elements", 1 << 30)):
             fc, fu, xx = (torch.randn(n, device="cuda") for _ in range(3))
@@ -601,6 +603,11 @@ def run_kernel(args):
             T.track_multistep_step(xx, fc, st, sg, 0)      # history for the timed step 1
             cases.append(("multistep", f"{label}: n={n}", 28.0 * n,
                           lambda xx=xx, fc=fc, st=st, sg=sg: T.track_multistep_step(xx, fc, st, sg, 1)))
+            if n == 2 * n480:   # band split (Sec. 4.4) of a 480p CFG pair: reads v_L, v_S
+                bl, bs = fc.view(2, 16, 21, 60, 104), fu.view(2, 16, 21, 60, 104)
+                bo = torch.empty(2, 6, device="cuda")
+                cases.append(("band_split", f"{label}: B=2 [16, 21, 60, 104]", 8.0 * n,
+                              lambda bl=bl, bs=bs, bo=bo: T.track_band_disagreement(bl, bs, out=bo)))
             B = 2 if n == 2 * n480 else 8
             acc = torch.zeros(B, device="cuda")
             cases.append(("disagreement", f"{label}: B={B} n={n // B}", 8.0 * n,

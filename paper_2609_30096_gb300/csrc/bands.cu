@@ -4,8 +4,8 @@
 // frequency in units of Nyquist against 1/3 and 2/3) and one temporal band
 // (|f| frequency, same thirds); band of a bin decided in integer arithmetic.
 //
-// Three separable passes, one output bin per thread, every sum in a fixed
-// order (deterministic):
+// Three separable passes over shared-memory tiles, every sum in a fixed order
+// (deterministic):
 //   pass W  Y1[c,f,h,kw] = sum_w D[c,f,h,w] e^{-2 pi i kw w / W} / sqrt(W), with
 //           per-block partial sums of v_L^2 (the denominator of Eq. 4)
 //   pass H  Y2[c,f,kh,kw] = sum_h Y1[c,f,h,kw] e^{-2 pi i kh h / H} / sqrt(H)
@@ -71,7 +71,12 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
   return t;
 }
 
-// grid (ceil(rows * W / BD_THREADS), B); one thread per (row, kw).
+// Each pass stages a tile in shared memory so every input element is read from
+// global memory once, then each thread forms output bins from the tile.
+constexpr int BD_COLS = 32;     // columns (innermost-axis positions) per H / F tile
+constexpr int BD_ROWS_W = 16;   // rows per W tile
+
+// grid (ceil(rows / BD_ROWS_W), B): a tile of BD_ROWS_W rows of D = v_S - v_L.
 __global__ void __launch_bounds__(BD_THREADS) k_band_w(const float* __restrict__ vL,
                                                        const float* __restrict__ vS,
                                                        float2* __restrict__ Y, int64_t rows,
@@ -80,66 +85,73 @@ __global__ void __launch_bounds__(BD_THREADS) k_band_w(const float* __restrict__
   pdl_release();
   __shared__ float2 tw[BD_MAXN];
   __shared__ float red[BD_THREADS / 32];
+  extern __shared__ float dtile[];  // [BD_ROWS_W][W]
   make_twiddles(tw, W);
-  __syncthreads();
   const int b = blockIdx.y;
   const int64_t per = rows * W;
-  const float* dl = vL + (int64_t)b * per;
-  const float* ds = vS + (int64_t)b * per;
-  const int64_t t = (int64_t)blockIdx.x * BD_THREADS + threadIdx.x;
+  const int64_t r0 = (int64_t)blockIdx.x * BD_ROWS_W;
+  const int nr = (int)(rows - r0 < BD_ROWS_W ? rows - r0 : BD_ROWS_W);
+  const float* dl = vL + (int64_t)b * per + r0 * W;
+  const float* ds = vS + (int64_t)b * per + r0 * W;
   float l2 = 0.f;
-  if (t < per) {
-    const int64_t row = t / W;
-    const int kw = (int)(t - row * W);
-    const float* rl = dl + row * W;
-    const float* rs = ds + row * W;
+  for (int i = threadIdx.x; i < nr * W; i += BD_THREADS) {
+    const float x = dl[i];
+    dtile[i] = ds[i] - x;
+    l2 = fmaf(x, x, l2);
+  }
+  __syncthreads();
+  float2* yt = Y + (int64_t)b * per + r0 * W;
+  for (int o = threadIdx.x; o < nr * W; o += BD_THREADS) {
+    const int r = o / W, kw = o - r * W;
+    const float* d = dtile + r * W;
     float2 acc = make_float2(0.f, 0.f);
     int m = 0;  // kw * w mod W
     for (int w = 0; w < W; ++w) {
-      const float d = rs[w] - rl[w];
-      acc.x = fmaf(d, tw[m].x, acc.x);
-      acc.y = fmaf(d, tw[m].y, acc.y);
+      acc.x = fmaf(d[w], tw[m].x, acc.x);
+      acc.y = fmaf(d[w], tw[m].y, acc.y);
       m += kw;
       if (m >= W) m -= W;
     }
-    Y[(int64_t)b * per + t] = acc;
-    const float x = dl[t];
-    l2 = x * x;
+    yt[o] = acc;
   }
   const float s = block_sum(l2, red);
   if (threadIdx.x == 0) l2part[(int64_t)b * gridDim.x + blockIdx.x] = s;
 }
 
-// grid (ceil(C*F*H*W / BD_THREADS), B); one thread per (c, f, kh, kw).
+// grid (CF * ceil(W / BD_COLS), B): columns kw0..kw0+31 of one (c, f), all H.
 __global__ void __launch_bounds__(BD_THREADS) k_band_h(const float2* __restrict__ Y1,
                                                        float2* __restrict__ Y2, int CF, int H,
                                                        int W) {
   pdl_wait();
   pdl_release();
   __shared__ float2 tw[BD_MAXN];
+  extern __shared__ float2 ctile[];  // [H][BD_COLS]
   make_twiddles(tw, H);
-  __syncthreads();
-  const int64_t per = (int64_t)CF * H * W;
-  const int64_t t = (int64_t)blockIdx.x * BD_THREADS + threadIdx.x;
-  if (t >= per) return;
-  const int64_t base = (int64_t)blockIdx.y * per;
-  const int kw = (int)(t % W);
-  const int64_t q = t / W;
-  const int kh = (int)(q % H);
-  const int64_t cf = q / H;
-  const float2* col = Y1 + base + cf * H * W + kw;
-  float2 acc = make_float2(0.f, 0.f);
-  int m = 0;
-  for (int h = 0; h < H; ++h) {
-    acc = cmac(acc, col[(int64_t)h * W], tw[m]);
-    m += kh;
-    if (m >= H) m -= H;
+  const int ncb = (W + BD_COLS - 1) / BD_COLS;
+  const int cf = blockIdx.x / ncb, kw0 = (blockIdx.x % ncb) * BD_COLS;
+  const int nc = W - kw0 < BD_COLS ? W - kw0 : BD_COLS;
+  const int64_t base = (int64_t)blockIdx.y * CF * H * W + (int64_t)cf * H * W + kw0;
+  for (int i = threadIdx.x; i < H * BD_COLS; i += BD_THREADS) {
+    const int h = i / BD_COLS, j = i % BD_COLS;
+    if (j < nc) ctile[i] = Y1[base + (int64_t)h * W + j];
   }
-  Y2[base + t] = acc;
+  __syncthreads();
+  for (int o = threadIdx.x; o < H * BD_COLS; o += BD_THREADS) {
+    const int kh = o / BD_COLS, j = o % BD_COLS;
+    if (j >= nc) continue;
+    float2 acc = make_float2(0.f, 0.f);
+    int m = 0;
+    for (int h = 0; h < H; ++h) {
+      acc = cmac(acc, ctile[h * BD_COLS + j], tw[m]);
+      m += kh;
+      if (m >= H) m -= H;
+    }
+    Y2[base + (int64_t)kh * W + j] = acc;
+  }
 }
 
-// grid (ceil(C*F*H*W / BD_THREADS), B); one thread per (c, kf, kh, kw); writes
-// six band partials per block.
+// grid (C * ceil(H*W / BD_COLS), B): positions s0..s0+31 of the (h, w) plane of
+// one channel, all F; six band partials per block.
 __global__ void __launch_bounds__(BD_THREADS) k_band_f(const float2* __restrict__ Y2, int C,
                                                        int F, int H, int W,
                                                        float* __restrict__ bpart) {
@@ -147,35 +159,42 @@ __global__ void __launch_bounds__(BD_THREADS) k_band_f(const float2* __restrict_
   pdl_release();
   __shared__ float2 tw[BD_MAXN];
   __shared__ float red[BD_THREADS / 32];
+  extern __shared__ float2 ctile[];  // [F][BD_COLS]
   make_twiddles(tw, F);
-  __syncthreads();
   const int64_t hw = (int64_t)H * W;
-  const int64_t per = (int64_t)C * F * hw;
-  const int64_t t = (int64_t)blockIdx.x * BD_THREADS + threadIdx.x;
+  const int nsb = (int)((hw + BD_COLS - 1) / BD_COLS);
+  const int c = blockIdx.x / nsb;
+  const int64_t s0 = (int64_t)(blockIdx.x % nsb) * BD_COLS;
+  const int nc = (int)(hw - s0 < BD_COLS ? hw - s0 : BD_COLS);
+  const float2* src = Y2 + (int64_t)blockIdx.y * C * F * hw + (int64_t)c * F * hw + s0;
+  for (int i = threadIdx.x; i < F * BD_COLS; i += BD_THREADS) {
+    const int f = i / BD_COLS, j = i % BD_COLS;
+    if (j < nc) ctile[i] = src[(int64_t)f * hw + j];
+  }
+  __syncthreads();
   float e[6] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-  if (t < per) {
-    const int64_t s2 = t % hw;  // kh * W + kw
-    const int64_t q = t / hw;
-    const int kf = (int)(q % F);
-    const int c = (int)(q / F);
-    const float2* col = Y2 + (int64_t)blockIdx.y * per + (int64_t)c * F * hw + s2;
+  for (int o = threadIdx.x; o < F * BD_COLS; o += BD_THREADS) {
+    const int kf = o / BD_COLS, j = o % BD_COLS;
+    if (j >= nc) continue;
     float2 acc = make_float2(0.f, 0.f);
     int m = 0;
     for (int f = 0; f < F; ++f) {
-      acc = cmac(acc, col[(int64_t)f * hw], tw[m]);
+      acc = cmac(acc, ctile[f * BD_COLS + j], tw[m]);
       m += kf;
       if (m >= F) m -= F;
     }
     const float en = fmaf(acc.x, acc.x, acc.y * acc.y);
-    const int kh = (int)(s2 / W), kw = (int)(s2 % W);
-    e[spatial_band(kh, kw, H, W)] = en;
-    e[3 + temporal_band(kf, F)] = en;
+    const int64_t sp = s0 + j;
+    const int kh = (int)(sp / W), kw = (int)(sp % W);
+    const int bs = spatial_band(kh, kw, H, W), bt = 3 + temporal_band(kf, F);
+#pragma unroll
+    for (int q = 0; q < 6; ++q) e[q] += (q == bs || q == bt) ? en : 0.f;
   }
   float* out = bpart + ((int64_t)blockIdx.y * gridDim.x + blockIdx.x) * 6;
 #pragma unroll
-  for (int j = 0; j < 6; ++j) {
-    const float s = block_sum(e[j], red);
-    if (threadIdx.x == 0) out[j] = s;
+  for (int q = 0; q < 6; ++q) {
+    const float t = block_sum(e[q], red);
+    if (threadIdx.x == 0) out[q] = t;
   }
 }
 
@@ -208,10 +227,18 @@ __global__ void __launch_bounds__(BD_THREADS) k_band_final(const float* __restri
 
 }  // namespace
 
+// Blocks of each pass (the W pass writes one v_L^2 partial per block, the F pass
+// six band partials per block).
+static int64_t blocks_w(int C, int F, int H) {
+  return ((int64_t)C * F * H + BD_ROWS_W - 1) / BD_ROWS_W;
+}
+static int64_t blocks_f(int C, int H, int W) {
+  return (int64_t)C * (((int64_t)H * W + BD_COLS - 1) / BD_COLS);
+}
+
 size_t band_scratch_floats(int B, int C, int F, int H, int W) {
   const int64_t per = (int64_t)C * F * H * W;
-  const int64_t nblk = (per + BD_THREADS - 1) / BD_THREADS;
-  return (size_t)(4 * (int64_t)B * per + (int64_t)B * nblk * 7);
+  return (size_t)(4 * (int64_t)B * per + (int64_t)B * (blocks_w(C, F, H) + 6 * blocks_f(C, H, W)));
 }
 
 cudaError_t band_disagreement(const float* vL, const float* vS, int B, int C, int F, int H, int W,
@@ -219,21 +246,31 @@ cudaError_t band_disagreement(const float* vL, const float* vS, int B, int C, in
   if (B <= 0) return cudaSuccess;
   if (F > BD_MAXN || H > BD_MAXN || W > BD_MAXN) return cudaErrorInvalidValue;
   const int64_t per = (int64_t)C * F * H * W;
-  const int nblk = (int)((per + BD_THREADS - 1) / BD_THREADS);
+  const int64_t nw = blocks_w(C, F, H), nf = blocks_f(C, H, W);
+  const int64_t nh = (int64_t)C * F * ((W + BD_COLS - 1) / BD_COLS);
+  if (nw > INT32_MAX || nf > INT32_MAX || nh > INT32_MAX) return cudaErrorInvalidValue;
+  const size_t smem_hf = (size_t)BD_MAXN * BD_COLS * sizeof(float2);  // up to 128 KB
+  cudaError_t e = cudaFuncSetAttribute(k_band_h, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem_hf);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_band_f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_hf);
+  if (e != cudaSuccess) return e;
   float2* Y1 = reinterpret_cast<float2*>(scratch);
   float2* Y2 = Y1 + (int64_t)B * per;
   float* l2part = reinterpret_cast<float*>(Y2 + (int64_t)B * per);
-  float* bpart = l2part + (int64_t)B * nblk;
-  const dim3 grid(nblk, B);
-  cudaError_t e = launch_pdl(k_band_w, grid, BD_THREADS, 0, s, vL, vS, Y1, (int64_t)C * F * H, W,
-                             l2part);
+  float* bpart = l2part + (int64_t)B * nw;
+  e = launch_pdl(k_band_w, dim3((unsigned)nw, B), BD_THREADS,
+                             (size_t)BD_ROWS_W * W * sizeof(float), s, vL, vS, Y1,
+                             (int64_t)C * F * H, W, l2part);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(k_band_h, grid, BD_THREADS, 0, s, (const float2*)Y1, Y2, C * F, H, W);
+  e = launch_pdl(k_band_h, dim3((unsigned)nh, B), BD_THREADS, (size_t)H * BD_COLS * sizeof(float2),
+                 s, (const float2*)Y1, Y2, C * F, H, W);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(k_band_f, grid, BD_THREADS, 0, s, (const float2*)Y2, C, F, H, W, bpart);
+  e = launch_pdl(k_band_f, dim3((unsigned)nf, B), BD_THREADS, (size_t)F * BD_COLS * sizeof(float2),
+                 s, (const float2*)Y2, C, F, H, W, bpart);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(k_band_final, B, BD_THREADS, 0, s, (const float*)l2part, nblk,
-                 (const float*)bpart, nblk, eps, out);
+  e = launch_pdl(k_band_final, B, BD_THREADS, 0, s, (const float*)l2part, (int)nw,
+                 (const float*)bpart, (int)nf, eps, out);
   if (e != cudaSuccess) return e;
   count_launch(4);
   return cudaGetLastError();
