@@ -223,16 +223,20 @@ class DiT:
         L = y.shape[0]
         return y.reshape(L, self.arch.heads, self.arch.head_dim)
 
-    def self_attention(self, i, h):
+    def self_attention(self, i, h, rows=None):
+        """Self-attention output of the query tokens ``rows`` (all tokens if None); keys
+        and values always come from every token of h."""
         p, eps = f"blk{i}.", self.arch.eps
-        q = rms_norm(linear(h, self.W(p + "q.W"), self.W(p + "q.b")), self.W(p + "qn.g"), eps)
+        rows = np.arange(h.shape[0]) if rows is None else np.asarray(rows)
+        q = rms_norm(linear(h[rows], self.W(p + "q.W"), self.W(p + "q.b")), self.W(p + "qn.g"), eps)
         k = rms_norm(linear(h, self.W(p + "k.W"), self.W(p + "k.b")), self.W(p + "kn.g"), eps)
         v = linear(h, self.W(p + "v.W"), self.W(p + "v.b"))
-        qh, kh, vh = rope(self.heads(q), self.pos), rope(self.heads(k), self.pos), self.heads(v)
+        qh = rope(self.heads(q), self.pos[rows])
+        kh, vh = rope(self.heads(k), self.pos), self.heads(v)
         o = np.empty_like(qh)
         for hh in range(self.arch.heads):
             o[:, hh, :] = attention(qh[:, hh, :], kh[:, hh, :], vh[:, hh, :])
-        return linear(o.reshape(h.shape[0], -1), self.W(p + "o.W"), self.W(p + "o.b"))
+        return linear(o.reshape(len(rows), -1), self.W(p + "o.W"), self.W(p + "o.b"))
 
     def cross_attention(self, i, h, c):
         p, eps = f"blk{i}.", self.arch.eps
@@ -250,13 +254,17 @@ class DiT:
         u = gelu_tanh(linear(h, self.W(p + "ffn.W1"), self.W(p + "ffn.b1")))
         return linear(u, self.W(p + "ffn.W2"), self.W(p + "ffn.b2"))
 
-    def block(self, i, x, e0, c):
-        """One transformer block on the residual stream x [L, d]."""
+    def block(self, i, x, e0, c, rows=None):
+        """One transformer block on the residual stream x [L, d]; with ``rows``, the
+        block's output at those tokens only (self-attention is the one step that
+        mixes tokens, and it reads every token's keys and values)."""
         eps = self.arch.eps
         mod = e0 + self.W(f"blk{i}.mod_bias")
         shift1, scale1, gate1, shift2, scale2, gate2 = mod
         h = layer_norm(x, eps) * (1.0 + scale1) + shift1
-        x = x + gate1 * self.self_attention(i, h)
+        if rows is not None:
+            x = x[np.asarray(rows)]
+        x = x + gate1 * self.self_attention(i, h, rows)
         h = layer_norm(x, eps) * self.W(f"blk{i}.ln3.g") + self.W(f"blk{i}.ln3.b")
         x = x + self.cross_attention(i, h, c)
         h = layer_norm(x, eps) * (1.0 + scale2) + shift2
@@ -267,12 +275,15 @@ class DiT:
         tok = patchify(np.asarray(x, dtype=np.float64), self.arch.patch)
         return linear(tok, self.W("pe.W"), self.W("pe.b"))
 
-    def head(self, x, e):
+    def head_tokens(self, x, e):
+        """The head's per-token output [L, C*pf*ph*pw] (patchified prediction)."""
         hb = self.W("head_bias")
         shift, scale = e + hb[0], e + hb[1]
         h = layer_norm(x, self.arch.eps) * (1.0 + scale) + shift
-        out = linear(h, self.W("head.W"), self.W("head.b"))
-        return unpatchify(out, self.arch.latent_shape, self.arch.patch)
+        return linear(h, self.W("head.W"), self.W("head.b"))
+
+    def head(self, x, e):
+        return unpatchify(self.head_tokens(x, e), self.arch.latent_shape, self.arch.patch)
 
     # -- whole forward -------------------------------------------------------
     def forward(self, x, t, ctx):
@@ -283,3 +294,18 @@ class DiT:
         for i in range(self.arch.layers):
             h = self.block(i, h, e0, c)
         return self.head(h, e)
+
+    def forward_at_tokens(self, x, t, ctx, rows):
+        """Rows ``rows`` of patchify(f_m(x_t, t, c)): [len(rows), C*pf*ph*pw].
+
+        Every block but the last runs on all tokens; the last block, whose
+        self-attention still reads all tokens' keys and values, and the head
+        (per token) run only at ``rows``.  Equal to the same rows of forward()."""
+        e, e0 = self.time_embedding(t)
+        c = self.text_projection(ctx)
+        h = self.embed(x)
+        last = self.arch.layers - 1
+        for i in range(last):
+            h = self.block(i, h, e0, c)
+        h = self.block(last, h, e0, c, rows)
+        return self.head_tokens(h, e)

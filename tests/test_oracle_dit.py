@@ -283,6 +283,24 @@ CHECKS = [check_gates_and_identity, check_self_attention_branch, check_ffn_branc
           check_whole_forward_reduces_to_embed_and_head]
 
 
+@pytest.mark.parametrize("layers", [1, 2])
+def test_forward_at_tokens_is_rows_of_forward(layers):
+    # Only self-attention mixes tokens, so the sampled-token forward must give
+    # the same rows as the whole forward, in the order asked, for any depth.
+    arch = synth.Arch(dim=32, layers=layers, heads=2, ffn=64, text_dim=24, text_len=5,
+                      frames=2, height=4, width=6)
+    m = _model(arch)
+    rng = np.random.default_rng(layers)
+    x = rng.normal(size=arch.latent_shape)
+    ctx = rng.normal(size=(arch.text_len, arch.text_dim))
+    t = np.float32(433.0)
+    full = dit.patchify(m.forward(x, t, ctx), arch.patch)
+    for rows in (np.arange(arch.tokens), np.array([arch.tokens - 1, 0, 5, 3]), np.array([7])):
+        got = m.forward_at_tokens(x, t, ctx, rows)
+        assert got.shape == (len(rows), full.shape[1])
+        assert np.allclose(got, full[rows], rtol=1e-12, atol=1e-12)
+
+
 @pytest.mark.parametrize("check", CHECKS, ids=lambda f: f.__name__)
 def test_structural_pin(check):
     assert check()
@@ -316,11 +334,11 @@ class HeadDropsShift(dit.DiT):
 
 
 class TransposedRope(dit.DiT):
-    def self_attention(self, i, h):
+    def self_attention(self, i, h, rows=None):
         saved = dit.rope
         dit.rope = lambda xh, pos: saved(xh, pos[:, ::-1].copy())
         try:
-            return dit.DiT.self_attention(self, i, h)
+            return dit.DiT.self_attention(self, i, h, rows)
         finally:
             dit.rope = saved
 
