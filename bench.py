@@ -339,8 +339,8 @@ def run_ours(args):
     x_init = xh.to(dev)
 
     # One trajectory (text projection included) replayed from a CUDA graph recorded
-    # per policy; step_eager is the same work launched kernel by kernel (used for the
-    # event-bracketed kernel timing, which cannot see inside a graph).
+    # per policy; step_eager is the same work launched kernel by kernel (the fallback of
+    # the event-bracketed kernel timing).
     def step_device(pol):
         xd.copy_(x_init)                          # on-device reset of the latent
         T.track_sample_graph(L, S, pol, sig, xd, cd, ud, w, stream=sid)
@@ -363,11 +363,10 @@ def run_ours(args):
         step_device(pol)
         step_device(pol)
 
-    def timed(fn, pol, steps, profile=False):
+    def timed(fn, pol, steps):
         if world > 1:
             tdist.barrier()
         torch.cuda.synchronize()
-        T.track_profile_enable(profile)
         n0 = T.track_launch_count()
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
@@ -375,11 +374,51 @@ def run_ours(args):
             fn(pol)
         b.record(stream)
         torch.cuda.synchronize()
-        T.track_profile_enable(False)
         T.track_sync(sid)
         ms = a.elapsed_time(b)
         launches = T.track_launch_count() - n0
         return max_over_ranks(ms, world, dev), launches
+
+    def profiled_pass(pol, steps):
+        # Replays a copy of the trajectory's graph recorded with timing on (an event-
+        # record node before and after each bracketed kernel), reading the brackets after
+        # every replay.  Falls back to kernel-by-kernel launches if that fails.
+        keys = ("gemm", "attention", "norm")
+        tot = {k: [0.0, 0.0, 0] for k in keys}
+        ms_tot = 0.0
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        T.track_profile_enable(True)
+        try:
+            try:
+                mode = "graph"
+                prime(pol)                            # eager run, then the bracketed recording
+                torch.cuda.synchronize()
+                T.track_profile_read()
+                for _ in range(steps):
+                    a.record(stream)
+                    step_device(pol)
+                    b.record(stream)
+                    torch.cuda.synchronize()
+                    ms_tot += a.elapsed_time(b)
+                    for k, v in T.track_profile_read().items():
+                        tot[k] = [tot[k][0] + v[0], tot[k][1] + v[1], tot[k][2] + v[2]]
+            except T.TrackError:
+                mode = "eager"
+                tot = {k: [0.0, 0.0, 0] for k in keys}
+                ms_tot = 0.0
+                torch.cuda.synchronize()
+                T.track_profile_read()
+                for _ in range(steps):
+                    a.record(stream)
+                    step_eager(pol)
+                    b.record(stream)
+                    torch.cuda.synchronize()
+                    ms_tot += a.elapsed_time(b)
+                    for k, v in T.track_profile_read().items():
+                        tot[k] = [tot[k][0] + v[0], tot[k][1] + v[1], tot[k][2] + v[2]]
+        finally:
+            T.track_profile_enable(False)
+        return max_over_ranks(ms_tot, world, dev), {k: tuple(v) for k, v in tot.items()}, mode
 
     for _ in range(args.warmup):                   # the first two record the graph
         step_device(policy)
@@ -394,10 +433,9 @@ def run_ours(args):
         ms, launches = timed(step_device, policy, args.steps)
         e1 = energy.read_mj()
     clocks = clk.summary()
-    # Same steps again with every GEMM / attention launch bracketed by CUDA events on its
-    # stream (the events cost a few percent, so `value` comes from the pass above).
-    ms_prof, _ = timed(step_eager, policy, args.steps, profile=True)
-    prof = T.track_profile_read()
+    # Same steps again with every GEMM / attention / norm launch bracketed by CUDA events
+    # on its stream (the brackets cost a few percent, so `value` comes from the pass above).
+    ms_prof, prof, prof_mode = profiled_pass(policy, args.steps)
 
     all_l = np.zeros(wl.steps, np.uint8)
     prime(all_l)
@@ -482,9 +520,12 @@ def run_ours(args):
             "peak_source": f"{src} bf16 burst (sustained {peaks.get('bf16_tflops_sustained')})",
             "launches": int(dn), "avg_launch_ms": dm / dn if dn else None,
             "share_of_step": dm / ms_prof if ms_prof else None,
-            "measured_in": "a second pass of the timed steps launched kernel by kernel "
-                           "(no graph) with per-launch CUDA events "
-                           f"({ms_prof / args.steps:.3f} ms/step)",
+            "measured_in": ("a second pass of the timed steps replaying the trajectory's graph "
+                            "recorded with a CUDA event-record node before and after each GEMM, "
+                            "attention and norm kernel" if prof_mode == "graph" else
+                            "a second pass of the timed steps launched kernel by kernel "
+                            "(no graph) with per-launch CUDA events")
+                           + f" ({ms_prof / args.steps:.3f} ms/step)",
             "other": {("attention" if dominant == "gemm" else "gemm"):
                       {"ms": am if dominant == "gemm" else gm,
                        "tflops": ((af / (am / 1e3)) if dominant == "gemm" and am
@@ -556,7 +597,7 @@ def run_kernel(args):
     torch.cuda.set_device(0)
     T.track_gemm_schedule(GEMM_SCHEDULES[args.gemm_schedule])
     T.track_attention_schedule(GEMM_SCHEDULES[args.attn_schedule])
-    wl = synth.WORKLOADS[WORKLOAD]
+    wl = synth.WORKLOADS[args.workload]
     a = wl.large
     M = args.batch * a.tokens
     d, F, H, hd = a.dim, a.ffn, a.heads, a.head_dim
@@ -650,12 +691,16 @@ def main():
     ap.add_argument("--kernel", choices=["gemm", "attention", "hbm"], default=None,
                     help="time one kernel class alone at the workload's shapes")
     ap.add_argument("--batch", type=int, default=1, help="sequences for --kernel")
+    ap.add_argument("--workload", choices=sorted(synth.WORKLOADS), default=WORKLOAD,
+                    help="shapes for --kernel (the full benchmark always runs the mid pair)")
     ap.add_argument("--gemm-schedule", choices=["auto", "dp", "sk"], default="auto",
                     help="bf16 GEMM schedule: makespan model, data-parallel or stream-K")
     ap.add_argument("--attn-schedule", choices=["auto", "dp", "sk"], default="auto",
                     help="bf16 attention schedule: makespan model, data-parallel or stream-K")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)     # at least three untimed warm-up steps
+    if args.workload != WORKLOAD and not args.kernel:
+        ap.error("--workload applies to --kernel only")
     if args.impl == "reference":
         return run_reference(args)
     if args.kernel:

@@ -101,7 +101,9 @@ int64_t track_launch_count(void);
  * 2 = LayerNorm-modulate and RMSNorm/RoPE/head split), the summed event time in
  * ms, the summed algorithmic work (FLOPs for classes 0 and 1, bytes moved for
  * class 2) and the number of launches, then clears the records.  Arrays are
- * host, length 3. */
+ * host, length 3.  In a graph recorded by track_sample_graph while timing is
+ * enabled, the brackets are event-record nodes of the graph: each replay
+ * re-records the same events, so read after every replay. */
 int track_profile_enable(int enable);
 int track_profile_read(double* ms, double* flops, int64_t* launches);
 
@@ -285,9 +287,12 @@ int track_sample_multistep(track_model* large, track_model* small, const uint8_t
  * read the current contents of x, cond and uncond.  A graph is dropped when
  * a model it uses is destroyed or a buffer it addresses is reallocated.
  * s must be a created stream: EINVAL for the legacy default stream (it cannot
- * be recorded).  Kernel timing (track_profile_enable) sees none of the
- * replayed kernels.  This is a host-side mechanism; the paper has no
- * counterpart. */
+ * be recorded).  Whether kernel timing (track_profile_enable) is on is part
+ * of the key: a graph recorded with timing on carries an event-record node
+ * before and after each GEMM, attention and normalization kernel (it runs the
+ * same kernels, without the launch overlap that PDL gives between them), and
+ * one recorded with timing off carries none.  This is a host-side mechanism;
+ * the paper has no counterpart. */
 int track_sample_graph(track_model* large, track_model* small, const uint8_t* policy,
                        const float* sigmas, int n_steps, float* x, int B, const float* cond,
                        const float* uncond, float cfg_scale, track_stream s);

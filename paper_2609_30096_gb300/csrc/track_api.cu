@@ -10,6 +10,7 @@
 #include <algorithm>
 #include <atomic>
 #include <map>
+#include <unordered_set>
 #include <mutex>
 #include <string>
 #include <utility>
@@ -84,21 +85,42 @@ struct ProfRec {
   cudaEvent_t a, b;
   int cls;
   double flops;
+  bool owned_by_graph = false;  // recorded by a graph's event nodes; never pooled
 };
 static std::mutex g_prof_mu;
 static std::atomic<bool> g_prof_on{false};
 static std::vector<ProfRec> g_prof;
 static std::vector<std::pair<cudaEvent_t, cudaEvent_t>> g_prof_pool;
 
-// True on a thread while it records a CUDA graph (no event brackets then).
+// True on a thread while it records a CUDA graph.  With profiling on, the
+// brackets of a recorded launch become event-record nodes of the graph; their
+// events belong to the graph and are collected in g_capture_recs.
 static thread_local bool g_capturing = false;
+static thread_local std::vector<ProfRec>* g_capture_recs = nullptr;
 
 struct ProfScope {
   bool on = false;
   ProfRec r;
   cudaStream_t s;
   ProfScope(int cls, double flops, cudaStream_t st) : s(st) {
-    if (g_capturing || !g_prof_on.load(std::memory_order_relaxed)) return;
+    if (!g_prof_on.load(std::memory_order_relaxed)) return;
+    r.cls = cls;
+    r.flops = flops;
+    if (g_capturing) {
+      if (g_capture_recs == nullptr) return;
+      if (cudaEventCreate(&r.a) != cudaSuccess) return;
+      if (cudaEventCreate(&r.b) != cudaSuccess) {
+        cudaEventDestroy(r.a);
+        return;
+      }
+      r.owned_by_graph = true;
+      on = cudaEventRecordWithFlags(r.a, s, cudaEventRecordExternal) == cudaSuccess;
+      if (!on) {
+        cudaEventDestroy(r.a);
+        cudaEventDestroy(r.b);
+      }
+      return;
+    }
     std::lock_guard<std::mutex> lk(g_prof_mu);
     if (!g_prof_pool.empty()) {
       r.a = g_prof_pool.back().first;
@@ -108,12 +130,15 @@ struct ProfScope {
       if (cudaEventCreate(&r.a) != cudaSuccess) return;
       if (cudaEventCreate(&r.b) != cudaSuccess) return;
     }
-    r.cls = cls;
-    r.flops = flops;
     on = cudaEventRecord(r.a, s) == cudaSuccess;
   }
   ~ProfScope() {
     if (!on) return;
+    if (r.owned_by_graph) {
+      cudaEventRecordWithFlags(r.b, s, cudaEventRecordExternal);
+      g_capture_recs->push_back(r);
+      return;
+    }
     cudaEventRecord(r.b, s);
     std::lock_guard<std::mutex> lk(g_prof_mu);
     g_prof.push_back(r);
@@ -780,7 +805,7 @@ int track_profile_read(double* ms, double* flops, int64_t* launches) {
       flops[r.cls] += r.flops;
       launches[r.cls] += 1;
     }
-    g_prof_pool.emplace_back(r.a, r.b);
+    if (!r.owned_by_graph) g_prof_pool.emplace_back(r.a, r.b);
   }
   g_prof.clear();
   return rc;
@@ -1094,8 +1119,10 @@ struct GraphEntry {
   cudaStream_t s;
   int dev;
   uint64_t gen_L, gen_S, gen_sk;  // allocations the graph's addresses come from
+  bool prof = false;                 // recorded with profiling on: bracketed launches
   cudaGraphExec_t exec = nullptr;
-  int64_t launches = 0;  // kernels recorded in the graph
+  int64_t launches = 0;              // kernels recorded in the graph
+  std::vector<ProfRec> recs;         // the brackets' events (prof graphs only)
 };
 std::mutex g_graph_mu;
 std::vector<GraphEntry> g_graphs;
@@ -1104,12 +1131,28 @@ constexpr size_t kMaxGraphs = 32;
 bool same_call(const GraphEntry& e, const GraphEntry& k) {
   return e.L == k.L && e.S == k.S && e.policy == k.policy && e.sigmas == k.sigmas && e.x == k.x &&
          e.B == k.B && e.cond == k.cond && e.uncond == k.uncond && e.w == k.w && e.s == k.s &&
-         e.dev == k.dev;
+         e.dev == k.dev && e.prof == k.prof;
 }
 
+// Destroys the executable graph and the events of its brackets; brackets of
+// its replays that were not read yet are discarded.
 void drop_graph(GraphEntry& e) {
   if (e.exec) cudaGraphExecDestroy(e.exec);
   e.exec = nullptr;
+  if (e.recs.empty()) return;
+  {
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    std::unordered_set<cudaEvent_t> mine;
+    for (const ProfRec& r : e.recs) mine.insert(r.a);
+    g_prof.erase(std::remove_if(g_prof.begin(), g_prof.end(),
+                                [&mine](const ProfRec& q) { return mine.count(q.a) != 0; }),
+                 g_prof.end());
+  }
+  for (const ProfRec& r : e.recs) {
+    cudaEventDestroy(r.a);
+    cudaEventDestroy(r.b);
+  }
+  e.recs.clear();
 }
 
 // The routed loop of Eq. 3 with the text projection always recomputed.
@@ -1202,9 +1245,11 @@ int track_sample_graph(track_model* large, track_model* small, const uint8_t* po
   key.sigmas.assign(sigmas, sigmas + n_steps + 1);
   key.x = x; key.B = B; key.cond = cond; key.uncond = cfg_scale == 1.f ? nullptr : uncond;
   key.w = cfg_scale; key.s = st; key.dev = large->dev;
+  key.prof = g_prof_on.load(std::memory_order_relaxed);
   cudaGraphExec_t exec = nullptr;
   int64_t nlaunch = 0;
   bool warm = false;
+  std::vector<ProfRec> recs;
   {
     std::lock_guard<std::mutex> lk(g_graph_mu);
     for (size_t i = 0; i < g_graphs.size(); ++i) {
@@ -1219,6 +1264,7 @@ int track_sample_graph(track_model* large, track_model* small, const uint8_t* po
       warm = true;
       exec = e.exec;
       nlaunch = e.launches;
+      recs = e.recs;
       break;
     }
   }
@@ -1242,31 +1288,72 @@ int track_sample_graph(track_model* large, track_model* small, const uint8_t* po
     cudaGraph_t graph = nullptr;
     TRACK_CUDA(cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal));
     g_capturing = true;
+    g_capture_recs = key.prof ? &recs : nullptr;
     const int64_t n0 = track_launch_count();
     const int rc =
         sample_loop(large, small, policy, sigmas, n_steps, x, B, cond, uncond, cfg_scale, st);
     nlaunch = track_launch_count() - n0;
     g_capturing = false;
+    g_capture_recs = nullptr;
     const cudaError_t ce = cudaStreamEndCapture(st, &graph);
     large->c_valid = small->c_valid = false;  // the recorded projection has not run yet
+    auto free_recs = [&recs]() {
+      for (const ProfRec& r : recs) {
+        cudaEventDestroy(r.a);
+        cudaEventDestroy(r.b);
+      }
+      recs.clear();
+    };
     if (rc != TRACK_OK) {
       if (graph) cudaGraphDestroy(graph);
+      free_recs();
       return rc;
     }
-    if (ce != cudaSuccess) return fail(TRACK_ECUDA, std::string("graph capture: ") + cudaGetErrorString(ce));
+    if (ce != cudaSuccess) {
+      free_recs();
+      return fail(TRACK_ECUDA, std::string("graph capture: ") + cudaGetErrorString(ce));
+    }
     const cudaError_t ie = cudaGraphInstantiate(&exec, graph, 0);
     cudaGraphDestroy(graph);
-    if (ie != cudaSuccess) return fail(TRACK_ECUDA, std::string("graph instantiate: ") + cudaGetErrorString(ie));
+    if (ie != cudaSuccess) {
+      free_recs();
+      return fail(TRACK_ECUDA, std::string("graph instantiate: ") + cudaGetErrorString(ie));
+    }
     g_launches.fetch_sub(nlaunch, std::memory_order_relaxed);  // recorded, not launched
     std::lock_guard<std::mutex> lk(g_graph_mu);
+    bool stored = false;
     for (GraphEntry& e : g_graphs)
-      if (same_call(e, key)) {
+      if (!stored && same_call(e, key)) {
         e.exec = exec;
         e.launches = nlaunch;
+        e.recs = recs;
+        stored = true;
       }
+    if (!stored) {  // evicted meanwhile: keep the recording under a fresh entry
+      key.gen_L = large->ws_gen;
+      key.gen_S = small->ws_gen;
+      key.gen_sk = sk_scratch_generation();
+      key.exec = exec;
+      key.launches = nlaunch;
+      key.recs = recs;
+      if (g_graphs.size() >= kMaxGraphs) {
+        drop_graph(g_graphs.front());
+        g_graphs.erase(g_graphs.begin());
+      }
+      g_graphs.push_back(key);
+    }
   }
   TRACK_CUDA(cudaGraphLaunch(exec, st));
   count_launch((int)nlaunch);
+  if (!recs.empty()) {
+    // Every replay re-records the same events: the brackets hold the latest
+    // replay until read.
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    std::unordered_set<cudaEvent_t> pending;
+    for (const ProfRec& q : g_prof) pending.insert(q.a);
+    for (const ProfRec& r : recs)
+      if (pending.count(r.a) == 0) g_prof.push_back(r);
+  }
   return TRACK_OK;
 }
 

@@ -248,6 +248,41 @@ def test_graph_replay_matches_eager(T, tiny):
     assert e.value.code == T.TRACK_EINVAL
 
 
+def test_timed_graph_brackets_every_kernel(T, tiny):
+    # With kernel timing on, the recorded graph carries the brackets as event
+    # nodes: a replay computes the same values and reports the same launches,
+    # classes and work as an eager bracketed run, with positive times.
+    prec, P = tiny
+    pol = np.array([1, 0, 0, 1, 0, 1, 1, 0][:WL.steps], np.uint8)
+    x, c, u = synth.evaluation_inputs(WL.large, 5, 1, with_uncond=True)
+    sig = track.schedule(WL.steps, WL.shift)
+    s = torch.cuda.Stream()
+    try:
+        with torch.cuda.stream(s):
+            cd, ud, xg = dev(c), dev(u), dev(x)
+            T.track_profile_enable(True)
+            T.track_profile_read()
+            xe = dev(x)
+            T.track_invalidate_ctx(P.L)
+            T.track_invalidate_ctx(P.S)
+            T.track_sample(P.L, P.S, pol, sig, xe, cd, ud, WL.cfg, stream=s.cuda_stream)
+            T.track_sync(s.cuda_stream)
+            eager = T.track_profile_read()
+            for call in range(4):   # eager, record + replay, replay, replay
+                xg.copy_(dev(x))
+                T.track_sample_graph(P.L, P.S, pol, sig, xg, cd, ud, WL.cfg, stream=s.cuda_stream)
+                T.track_sync(s.cuda_stream)
+                got = T.track_profile_read()
+                assert torch.equal(xg, xe), call
+                for k in ("gemm", "attention", "norm"):
+                    assert got[k][2] == eager[k][2] > 0, (call, k)
+                    assert got[k][1] == eager[k][1], (call, k)
+                    assert got[k][0] > 0, (call, k)
+    finally:
+        T.track_profile_enable(False)
+        T.track_profile_read()
+
+
 def test_argument_errors(T, tiny, calib_inputs):
     prec, P = tiny
     x, c, u = calib_inputs
