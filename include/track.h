@@ -328,15 +328,19 @@ int track_linear(int dtype, const void* X, const void* W, const float* bias, int
 int track_gemm_schedule(int mode);
 
 /* Schedule of the TRACK_BF16 attention kernel (process-wide), with the mode
- * values of track_gemm_schedule (no multicast).  The kernel is persistent, at
- * most one CTA per SM.  TRACK_GEMM_DATA_PARALLEL gives each CTA whole
- * 128-query tiles of one (sequence, head); TRACK_GEMM_STREAM_K shares the
- * tiles' 128-key blocks out evenly over one CTA per SM.  It is used wherever
- * no query tile would span more than 4 CTAs.  A split query tile is finished
- * by the last of its CTAs, which combines the parts' row maxima, row sums and
- * unnormalized outputs in key order.  TRACK_GEMM_AUTO (the default) picks per
- * launch by a makespan model.  Each schedule is deterministic; the two differ
- * in fp32 rounding only.  EINVAL for any other mode. */
+ * values of track_gemm_schedule (no multicast), optionally or-ed with
+ * TRACK_ATTN_ONE_TILE.  The kernel is persistent, at most one CTA per SM, and
+ * its work item is a pair of 128-query tiles of one (sequence, head) sharing
+ * every K and V tile it loads; with TRACK_ATTN_ONE_TILE it is the earlier
+ * kernel whose item is a single 128-query tile.  TRACK_GEMM_DATA_PARALLEL
+ * gives each CTA whole items; TRACK_GEMM_STREAM_K shares the items' 128-key
+ * blocks out evenly over one CTA per SM.  It is used wherever no item would
+ * span more than 4 CTAs.  A split item is finished by the last of its CTAs,
+ * which combines the parts' row maxima, row sums and unnormalized outputs in
+ * key order.  TRACK_GEMM_AUTO (the default) picks per launch by a makespan
+ * model.  Each schedule is deterministic; they differ in fp32 rounding only.
+ * EINVAL for any other mode. */
+#define TRACK_ATTN_ONE_TILE 4
 int track_attention_schedule(int mode);
 
 /* O = softmax(Q K^T / sqrt(hd)) V per (sequence, head), no mask.  Q: [S, H, Lq,

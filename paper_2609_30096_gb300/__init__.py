@@ -22,6 +22,7 @@ FP32, BF16 = 0, 1
 EPI_STORE, EPI_GELU, EPI_RESID_GATE, EPI_RESID = range(4)
 GEMM_AUTO, GEMM_DATA_PARALLEL, GEMM_STREAM_K = range(3)
 GEMM_MULTICAST = 4  # OR-ed into a schedule: two-CTA clusters sharing W tiles
+ATTN_ONE_TILE = 4   # OR-ed into an attention schedule: one query tile per work item
 
 
 class TrackError(RuntimeError):
@@ -154,7 +155,8 @@ def track_gemm_schedule(mode: int):
 
 
 def track_attention_schedule(mode: int):
-    """GEMM_AUTO, GEMM_DATA_PARALLEL or GEMM_STREAM_K for every later bf16 attention."""
+    """GEMM_AUTO, GEMM_DATA_PARALLEL or GEMM_STREAM_K (optionally | ATTN_ONE_TILE) for
+    every later bf16 attention."""
     _check(lib().track_attention_schedule(int(mode)))
 
 

@@ -585,6 +585,497 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   }
 }
 
+// ---------------------------------------------------------------- two query tiles per item
+// The default kernel.  An item is a pair of query tiles (256 query rows) of one
+// (sequence, head); both tiles share every K and V tile the CTA loads.  Each
+// tile has its own softmax warpgroup, one thread per query row holding the
+// whole 128-key row of S, so no row statistics cross warpgroups.  The MMA
+// warp interleaves the two tiles,
+//   S0(j) S1(j) | PV0(j) S0(j+1) | PV1(j) S1(j+1) | PV0(j+1) ...
+// so the tensor cores compute one tile's P V and next S while the other
+// tile's softmax runs; P overwrites the first 64 columns of its tile's S
+// buffer, and S(j+1) of a tile is issued after P V(j) of the same tile has
+// been issued (tensor-core operations of one thread run in order).  With one
+// S buffer and one O accumulator per tile TMEM holds 2 x (HD + 128) columns.
+// Schedules, the stream-K combine and the bounded waits are those of the
+// one-tile kernel above, with items of 256 rows.
+constexpr int PP_THREADS = 320;  // warp 0 TMA, warp 1 MMA, warps 2-5 / 6-9 softmax of tile 0 / 1
+
+template <int HD>
+struct PpShape {
+  static constexpr uint32_t QT_BYTES = AT_BM * HD * 2;  // one query tile
+  static constexpr uint32_t KV_BYTES = AT_BN * HD * 2;  // one K or V tile
+  static constexpr int KST = 3, VST = 2;                // K and V ring stages
+  static constexpr size_t SMEM = 2 * QT_BYTES + (KST + VST) * (size_t)KV_BYTES + 256;
+  // TMEM columns: O of tile t at t * HD, S (then P) of tile t at TM_S0 + 128 t
+  static constexpr uint32_t TM_S0 = 2 * HD;
+  static constexpr uint32_t TMEM_COLS = 512;
+  static_assert(TM_S0 + 2 * AT_BN <= TMEM_COLS, "TMEM budget");
+  // Stream-K slot: per softmax warp wi its 32 rows x HD columns of O (float4
+  // index (wi * HD / 4 + c) * 32 + lane), then per warp m[32] and l[32].
+  static constexpr int SLOT = 2 * AT_BM * HD + 8 * 2 * 32;
+};
+
+// Output of one query tile of a segment by one softmax warp (its 32 rows, all
+// HD columns); see segment_output for the stream-K publish / combine.
+template <int HD>
+__device__ __forceinline__ bool segment_output_pp(uint32_t tO, float m, float lt, int item, int kt0,
+                                                  int kt1, int KT, int QP, int H, int Lq,
+                                                  int64_t U, bf16* __restrict__ O, int t, int row,
+                                                  int lane, int wi, const AtSk& sk, int* err,
+                                                  volatile int* abort_flag) {
+  using S = PpShape<HD>;
+  auto store32 = [&](bf16* dst, const float (&v)[32], float inv) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      uint4 u;
+      u.x = pack_bf16x2(v[8 * j] * inv, v[8 * j + 1] * inv);
+      u.y = pack_bf16x2(v[8 * j + 2] * inv, v[8 * j + 3] * inv);
+      u.z = pack_bf16x2(v[8 * j + 4] * inv, v[8 * j + 5] * inv);
+      u.w = pack_bf16x2(v[8 * j + 6] * inv, v[8 * j + 7] * inv);
+      *reinterpret_cast<uint4*>(dst + 8 * j) = u;
+    }
+  };
+  const int bh = item / QP, sq = bh / H, hq = bh % H;
+  const int qrow = (item % QP) * (2 * AT_BM) + t * AT_BM + row;
+  bf16* orow = O + (((int64_t)sq * Lq + qrow) * H + hq) * HD;
+  if (kt0 == 0 && kt1 == KT) {
+    const float inv = 1.f / lt;
+#pragma unroll 1
+    for (int cc = 0; cc < HD / 32; ++cc) {
+      uint32_t r[32];
+      tmem_ld32(tO + cc * 32, r);
+      float v[32];
+#pragma unroll
+      for (int x = 0; x < 32; ++x) v[x] = __uint_as_float(r[x]);
+      if (qrow < Lq) store32(orow + cc * 32, v, inv);
+    }
+    return true;
+  }
+  const int64_t iu = (int64_t)item * KT;
+  const int w_first = sk_worker_of(iu, U, gridDim.x);
+  const int nparts = sk_worker_of(iu + KT - 1, U, gridDim.x) - w_first + 1;
+  const int part = (int)blockIdx.x - w_first;
+  if (nparts > AT_MAX_PARTS) {  // excluded by the host's choice of schedule
+    if (lane == 0) {
+      *abort_flag = 1;
+      atomicExch(err, 24);
+    }
+    return false;
+  }
+  auto slot_of = [&](int i) -> float* {
+    const int wk = w_first + i;
+    const int first_item = (int)(((int64_t)wk * U / gridDim.x) / KT);
+    return sk.ws + (size_t)(2 * wk + (first_item == item ? 0 : 1)) * S::SLOT;
+  };
+  int* cnt = sk.cnt + 8 * item + wi;
+  int last = 0;
+  if (lane == 0) last = ld_acquire(cnt) == nparts - 1 ? 1 : 0;
+  last = __shfl_sync(0xffffffffu, last, 0);
+  if (!last) {
+    float* mine = slot_of(part);
+    float4* o4 = reinterpret_cast<float4*>(mine) + (size_t)wi * (HD / 4) * 32 + lane;
+#pragma unroll 1
+    for (int cc = 0; cc < HD / 32; ++cc) {
+      uint32_t r[32];
+      tmem_ld32(tO + cc * 32, r);
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        o4[(cc * 8 + j) * 32] =
+            make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                        __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+    }
+    float* ml = mine + 2 * AT_BM * HD + wi * 64;
+    ml[lane] = m;
+    ml[32 + lane] = lt;
+    __threadfence();
+    __syncwarp();
+    if (lane == 0) last = atomicAdd(cnt, 1) == nparts - 1 ? 1 : 0;
+    last = __shfl_sync(0xffffffffu, last, 0);
+  }
+  if (last) {
+    __threadfence();
+    if (lane == 0) *cnt = 0;
+    float wp[AT_MAX_PARTS], lp[AT_MAX_PARTS];
+    float M = m;
+#pragma unroll
+    for (int i = 0; i < AT_MAX_PARTS; ++i) {
+      wp[i] = -INFINITY;
+      lp[i] = 0.f;
+      if (i < nparts) {
+        if (i == part) {
+          wp[i] = m;
+          lp[i] = lt;
+        } else {
+          const float* ml = slot_of(i) + 2 * AT_BM * HD + wi * 64;
+          wp[i] = __ldcg(ml + lane);
+          lp[i] = __ldcg(ml + 32 + lane);
+        }
+        M = fmaxf(M, wp[i]);
+      }
+    }
+    float den = 0.f;
+#pragma unroll
+    for (int i = 0; i < AT_MAX_PARTS; ++i) {
+      wp[i] = i < nparts ? exp2_approx(wp[i] - M) : 0.f;
+      den = fmaf(wp[i], lp[i], den);
+    }
+    const float inv = 1.f / den;
+#pragma unroll 1
+    for (int cc = 0; cc < HD / 32; ++cc) {
+      uint32_t r[32];
+      tmem_ld32(tO + cc * 32, r);
+      float acc[32];
+#pragma unroll
+      for (int x = 0; x < 32; ++x) acc[x] = 0.f;
+#pragma unroll
+      for (int i = 0; i < AT_MAX_PARTS; ++i) {
+        if (i >= nparts) break;
+        float xv[32];
+        if (i == part) {
+#pragma unroll
+          for (int x = 0; x < 32; ++x) xv[x] = __uint_as_float(r[x]);
+        } else {
+          const float4* src =
+              reinterpret_cast<const float4*>(slot_of(i)) + (size_t)wi * (HD / 4) * 32 + lane;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float4 q = __ldcg(src + (cc * 8 + j) * 32);
+            xv[4 * j] = q.x; xv[4 * j + 1] = q.y; xv[4 * j + 2] = q.z; xv[4 * j + 3] = q.w;
+          }
+        }
+#pragma unroll
+        for (int x = 0; x < 32; ++x) acc[x] = fmaf(wp[i], xv[x], acc[x]);
+      }
+      if (qrow < Lq) store32(orow + cc * 32, acc, inv);
+    }
+  }
+  return true;
+}
+
+template <int HD>
+__global__ void __launch_bounds__(PP_THREADS, 1)
+    k_attn_pp(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+              const __grid_constant__ CUtensorMap tmV, bf16* __restrict__ O, int H, int Lq, int Lk,
+              float scale_log2, int q_tok, int kv_tok, int* err, int items, const AtSk sk) {
+  using S = PpShape<HD>;
+  constexpr int NB = HD / 64;  // 64-column boxes per row of Q/K/V
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = smem_raw;
+  uint8_t* sQ = smem;                         // [2] query tiles of the item
+  uint8_t* sK = sQ + 2 * S::QT_BYTES;         // [KST] K stages
+  uint8_t* sV = sK + S::KST * S::KV_BYTES;    // [VST] V stages
+  uint64_t* bars = (uint64_t*)(sV + S::VST * S::KV_BYTES);
+  uint64_t* q_full = bars;        // both query tiles of the segment landed
+  uint64_t* q_empty = bars + 1;   // the segment's last S MMAs completed
+  uint64_t* k_full = bars + 2;    // [KST]
+  uint64_t* k_empty = bars + 5;   // [KST] both S MMAs of the key tile completed
+  uint64_t* v_full = bars + 8;    // [VST]
+  uint64_t* v_empty = bars + 10;  // [VST] both P V MMAs of the key tile completed
+  uint64_t* s_full = bars + 12;   // [2] per query tile: S of its current key tile
+  uint64_t* p_full = bars + 14;   // [2] per query tile: P written (4 warps)
+  uint64_t* o_full = bars + 16;   // [2] per query tile: every P V of the segment completed
+  uint64_t* o_empty = bars + 18;  // [2] per query tile: the segment's O read out (4 warps)
+  uint64_t* done = bars + 20;     // every MMA of the CTA has completed
+  uint32_t* tmem_slot = (uint32_t*)(bars + 21);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int QT = (Lq + AT_BM - 1) / AT_BM, KT = (Lk + AT_BN - 1) / AT_BN;
+  const int QP = (QT + 1) / 2;  // query tile pairs per (sequence, head)
+  const bool use_sk = sk.cnt != nullptr;
+  const int64_t U = use_sk ? sk.units : (int64_t)items * KT;
+
+  if (threadIdx.x == 0) {
+    mbar_init(su32(q_full), 1);
+    mbar_init(su32(q_empty), 1);
+    for (int i = 0; i < S::KST; ++i) {
+      mbar_init(su32(&k_full[i]), 1);
+      mbar_init(su32(&k_empty[i]), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(su32(&v_full[i]), 1);
+      mbar_init(su32(&v_empty[i]), 1);
+      mbar_init(su32(&s_full[i]), 1);
+      mbar_init(su32(&p_full[i]), 4);
+      mbar_init(su32(&o_full[i]), 1);
+      mbar_init(su32(&o_empty[i]), 4);
+    }
+    mbar_init(su32(done), 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(su32(tmem_slot), S::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  pdl_wait();
+  pdl_release();
+  if ((su32(smem) & 1023u) != 0) {  // the 128-byte-swizzled tiles need 1024-byte alignment
+    if (threadIdx.x == 0) atomicExch(err, 25);
+    __syncthreads();
+    if (warp == 1) tmem_dealloc(tmem_base, S::TMEM_COLS);
+    return;
+  }
+
+  if (warp == 0) {
+    // lane 0 streams the query tile pairs and the K tiles, lane 1 the V tiles
+    if (lane < 2) {
+      const bool kside = lane == 0;
+      const CUtensorMap* tm = kside ? &tmK : &tmV;
+      uint8_t* ring = kside ? sK : sV;
+      uint64_t* full = kside ? k_full : v_full;
+      uint64_t* empty = kside ? k_empty : v_empty;
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)tm) : "memory");
+      if (kside) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmQ) : "memory");
+      const int nst = kside ? S::KST : S::VST;
+      uint32_t armed[S::KST] = {}, q_armed = 0;
+      SegIter it(use_sk, U, items, KT, blockIdx.x, gridDim.x);
+      int item, kt0, kt1;
+      int g = 0, si = 0;
+      bool ok = true;
+      while (ok && it.next(item, kt0, kt1)) {
+        const int bh = item / QP, sq = bh / H, hq = bh % H;
+        if (kside) {
+          if (!mbar_wait(su32(q_empty), (si & 1) ^ 1, abort_flag, err, 10)) break;
+          mbar_expect_tx(su32(q_full), 2 * S::QT_BYTES);
+          const int q0 = (item % QP) * (2 * AT_BM);
+          for (int t = 0; t < 2; ++t)
+            for (int b = 0; b < NB; ++b)
+              tma_load_rows(su32(sQ + t * S::QT_BYTES + b * AT_BM * 128), &tmQ, q_tok, b * 64,
+                            q0 + t * AT_BM, hq, sq, su32(q_full));
+          ++q_armed;
+        }
+        for (int kt = kt0; kt < kt1; ++kt, ++g) {
+          const int st = g % nst;
+          if (!mbar_wait(su32(&empty[st]), ((g / nst) & 1) ^ 1, abort_flag, err, 11)) {
+            ok = false;
+            break;
+          }
+          mbar_expect_tx(su32(&full[st]), S::KV_BYTES);
+          for (int b = 0; b < NB; ++b)
+            tma_load_rows(su32(ring + st * S::KV_BYTES + b * AT_BN * 128), tm, kv_tok, b * 64,
+                          kt * AT_BN, hq, sq, su32(&full[st]));
+          ++armed[st];
+        }
+        ++si;
+      }
+      for (int i = 0; i < nst; ++i)
+        if (armed[i] != 0) mbar_drain(su32(&full[i]), (armed[i] - 1) & 1, err, 15);
+      if (q_armed != 0) mbar_drain(su32(q_full), (q_armed - 1) & 1, err, 15);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idS = idesc_bf16(AT_BM, AT_BN);
+      constexpr uint32_t idO = idesc_bf16_bmn(AT_BM, HD);
+      // S_t = Q_t K(g)^T into tile t's S buffer (K stage already waited for).
+      auto issue_s = [&](int t, int g) {
+        const int st = g % S::KST;
+        const uint32_t qa = su32(sQ + t * S::QT_BYTES), ka = su32(sK + st * S::KV_BYTES);
+        const uint32_t d = tmem_base + S::TM_S0 + (uint32_t)(t * AT_BN);
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk)
+          mma_bf16(d, sdesc_sw128(qa + (kk >> 2) * (AT_BM * 128) + (kk & 3) * 32),
+                   sdesc_sw128(ka + (kk >> 2) * (AT_BN * 128) + (kk & 3) * 32), idS,
+                   kk > 0 ? 1u : 0u);
+        mma_commit(su32(&s_full[t]));
+      };
+      // O_t (+)= P_t(g) V(g); P keys 16kk..16kk+15 sit in S columns 8kk..8kk+7.
+      auto issue_pv = [&](int t, int g, bool first) {
+        const uint32_t va = su32(sV + (g % S::VST) * S::KV_BYTES);
+        const uint32_t pt = tmem_base + S::TM_S0 + (uint32_t)(t * AT_BN);
+#pragma unroll
+        for (int kk = 0; kk < AT_BN / 16; ++kk)
+          mma_bf16_ts(tmem_base + (uint32_t)(t * HD), pt + (uint32_t)(kk * 8),
+                      sdesc_sw128_mn(va + kk * 16 * 128, AT_BN * 128), idO,
+                      (!first || kk > 0) ? 1u : 0u);
+      };
+      SegIter it(use_sk, U, items, KT, blockIdx.x, gridDim.x);
+      int item, c0, c1;
+      int g = 0, si = 0;  // key tiles and segments so far
+      bool ok = true;
+      while (ok && it.next(item, c0, c1)) {
+        const int n = c1 - c0;
+        if (!mbar_wait(su32(q_full), si & 1, abort_flag, err, 13)) break;
+        {
+          const int st = g % S::KST;
+          if (!mbar_wait(su32(&k_full[st]), (g / S::KST) & 1, abort_flag, err, 12)) break;
+          tc_fence_after();
+          issue_s(0, g);
+          issue_s(1, g);
+          mma_commit(su32(&k_empty[st]));
+          if (n == 1) mma_commit(su32(q_empty));
+        }
+        for (int j = 1; j <= n; ++j) {
+          const int gp = g + j - 1;  // the key tile whose P V is issued now
+          const int gn = g + j;      // the key tile whose S is issued now (j < n)
+          const int vst = gp % S::VST;
+          if (!mbar_wait(su32(&v_full[vst]), (gp / S::VST) & 1, abort_flag, err, 21)) {
+            ok = false;
+            break;
+          }
+          // query tile 0: P V of tile gp, then S of tile gn
+          if (j == 1 && !mbar_wait(su32(&o_empty[0]), (si & 1) ^ 1, abort_flag, err, 20)) {
+            ok = false;
+            break;
+          }
+          if (!mbar_wait(su32(&p_full[0]), gp & 1, abort_flag, err, 14)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          issue_pv(0, gp, j == 1);
+          if (j == n) mma_commit(su32(&o_full[0]));
+          if (j < n) {
+            const int kst = gn % S::KST;
+            if (!mbar_wait(su32(&k_full[kst]), (gn / S::KST) & 1, abort_flag, err, 12)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            issue_s(0, gn);
+          }
+          // query tile 1
+          if (j == 1 && !mbar_wait(su32(&o_empty[1]), (si & 1) ^ 1, abort_flag, err, 20)) {
+            ok = false;
+            break;
+          }
+          if (!mbar_wait(su32(&p_full[1]), gp & 1, abort_flag, err, 14)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          issue_pv(1, gp, j == 1);
+          mma_commit(su32(&v_empty[vst]));
+          if (j == n) mma_commit(su32(&o_full[1]));
+          if (j < n) {
+            issue_s(1, gn);
+            mma_commit(su32(&k_empty[gn % S::KST]));
+            if (j == n - 1) mma_commit(su32(q_empty));
+          }
+        }
+        g += n;
+        ++si;
+      }
+      mma_commit(su32(done));
+      mbar_drain(su32(done), 0, err, 16);
+    }
+  } else {
+    // Softmax of query tile t: one thread per row (TMEM lane), all 128 keys.
+    const int t = (warp - 2) >> 2;
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;
+    const int wi = warp - 2;
+    const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
+    const uint32_t tO = tmem_base + lane_off + (uint32_t)(t * HD);
+    const uint32_t tS = tmem_base + lane_off + S::TM_S0 + (uint32_t)(t * AT_BN);
+    SegIter it(use_sk, U, items, KT, blockIdx.x, gridDim.x);
+    int item, kt0, kt1;
+    int g = 0, si = 0;
+    bool ok = true;
+    while (ok && it.next(item, kt0, kt1)) {
+      float m = -INFINITY, l = 0.f;
+      for (int kt = kt0; kt < kt1; ++kt, ++g) {
+        if (!warp_wait(su32(&s_full[t]), g & 1, abort_flag, err, 17)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        uint32_t sv[AT_BN];
+        tmem_ld32_nowait(tS, sv);
+        tmem_ld32_nowait(tS + 32, sv + 32);
+        tmem_ld32_nowait(tS + 64, sv + 64);
+        tmem_ld32_nowait(tS + 96, sv + 96);
+        tmem_ld_wait();
+        const int kbase = kt * AT_BN;
+        if (kbase + AT_BN > Lk) {
+#pragma unroll
+          for (int i = 0; i < AT_BN; ++i)
+            if (kbase + i >= Lk) sv[i] = __float_as_uint(-INFINITY);
+        }
+        float pm[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) pm[j] = __uint_as_float(sv[j]);
+#pragma unroll
+        for (int i = 8; i < AT_BN; ++i) pm[i & 7] = fmaxf(pm[i & 7], __uint_as_float(sv[i]));
+        const float rmax = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                                 fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+        // finite: the first key of every key tile is valid
+        const float mt = rmax * scale_log2;
+        // Lazy rescaling: the running maximum moves only when it grows by more
+        // than 2^8; O is then rescaled below, after S is consumed.
+        float alpha = 1.f;
+        bool rescale = false;
+        if (kt > kt0) {
+          const bool need = mt > m + 8.f;
+          rescale = __any_sync(0xffffffffu, need);
+          if (need) {
+            alpha = exp2_approx(m - mt);
+            m = mt;
+            l *= alpha;
+          }
+        } else {
+          m = mt;
+        }
+        // P = exp2(S * scale - m), keys 16c..16c+15 packed into S columns 8c..8c+7
+        float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        const float nm = -m;
+#pragma unroll
+        for (int c = 0; c < AT_BN / 16; ++c) {
+          uint32_t pk[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const float p0 = exp2_approx(fmaf(__uint_as_float(sv[16 * c + 2 * i]), scale_log2, nm));
+            const float p1 =
+                exp2_approx(fmaf(__uint_as_float(sv[16 * c + 2 * i + 1]), scale_log2, nm));
+            ps[(2 * i) & 7] += p0;
+            ps[(2 * i + 1) & 7] += p1;
+            pk[i] = pack_bf16x2(p0, p1);
+          }
+          tmem_st8(tS + 8 * c, pk);
+        }
+        l += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+        if (rescale) {
+          // O_t is idle: S_t of this key tile was issued after P V of the
+          // previous one, whose completion the s_full wait observed; P V of
+          // this tile waits for p_full below.
+          uint32_t r[32];
+#pragma unroll 1
+          for (int cc = 0; cc < HD / 32; ++cc) {
+            tmem_ld32(tO + cc * 32, r);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+            tmem_st32(tO + cc * 32, r);
+          }
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(su32(&p_full[t]));
+      }
+      if (!ok) break;
+      if (!warp_wait(su32(&o_full[t]), si & 1, abort_flag, err, 19)) break;
+      tc_fence_after();
+      if (!segment_output_pp<HD>(tO, m, l, item, kt0, kt1, KT, QP, H, Lq, U, O, t, row, lane, wi,
+                                 sk, err, abort_flag))
+        break;
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(su32(&o_empty[t]));
+      ++si;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem_base, S::TMEM_COLS);
+  }
+}
+
 // 4-D tensor map of one operand, dimensions ordered by increasing stride:
 // (hd, H, L, S) when token-major (hs < ls), (hd, L, H, S) when head-major;
 // the box covers 64 columns of `rows` consecutive positions of one head.
@@ -647,7 +1138,7 @@ cudaError_t launch_attn_tc(const AttnOperand& Q, const AttnOperand& K, const Att
   const int G = num_sms();
   int grid = items < G ? (int)items : G;
   AtSk sk = {nullptr, nullptr, 0};
-  const int mode = g_attn_schedule.load();
+  const int mode = g_attn_schedule.load() & 3;
   if (mode != 1) {
     const int64_t U = items * KT, per = U / G;
     const bool spans_ok = per > 0 && 1 + (KT - 1 + per - 1) / per <= AT_MAX_PARTS;
@@ -666,6 +1157,52 @@ cudaError_t launch_attn_tc(const AttnOperand& Q, const AttnOperand& K, const Att
                     scale_log2, q_tok, k_tok, err, (int)items, sk);
 }
 
+// The same model for the two-tile kernel, in units of one key tile for both
+// query tiles of an item.
+constexpr double PP_OV = 1.5, PP_FIX = 4.0;
+
+template <int HD>
+cudaError_t launch_attn_pp(const AttnOperand& Q, const AttnOperand& K, const AttnOperand& V,
+                           void* O, int S_, int H, int Lq, int Lk, cudaStream_t s) {
+  using S1 = PpShape<HD>;
+  static_assert(S1::SMEM <= 232448, "shared memory budget");
+  CUtensorMap tq, tk, tv;
+  int q_tok = 0, k_tok = 0, v_tok = 0;
+  if (!make_tmap_op(&tq, Q, HD, Lq, H, S_, AT_BM, &q_tok) ||
+      !make_tmap_op(&tk, K, HD, Lk, H, S_, AT_BN, &k_tok) ||
+      !make_tmap_op(&tv, V, HD, Lk, H, S_, AT_BN, &v_tok) || k_tok != v_tok)
+    return cudaErrorInvalidValue;
+  int* err = device_error_word();
+  if (err == nullptr) return cudaErrorMemoryAllocation;
+  const float scale_log2 = (float)(1.4426950408889634 / sqrt((double)HD));
+  cudaError_t e = cudaFuncSetAttribute(k_attn_pp<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)S1::SMEM);
+  if (e != cudaSuccess) return e;
+  const int QT = (Lq + AT_BM - 1) / AT_BM, KT = (Lk + AT_BN - 1) / AT_BN;
+  const int64_t items = (int64_t)S_ * H * ((QT + 1) / 2);
+  if (items > (1 << 26)) return cudaErrorInvalidValue;
+  const int G = num_sms();
+  int grid = items < G ? (int)items : G;
+  AtSk sk = {nullptr, nullptr, 0};
+  const int mode = g_attn_schedule.load() & 3;
+  if (mode != 1) {
+    const int64_t U = items * KT, per = U / G;
+    const bool spans_ok = per > 0 && 1 + (KT - 1 + per - 1) / per <= AT_MAX_PARTS;
+    const double dp_cost = (double)((items + G - 1) / G) * (KT + PP_OV);
+    const double sk_cost = (double)U / G + (double)items / G * PP_OV + PP_FIX;
+    if (spans_ok && (mode == 2 || sk_cost < 0.97 * dp_cost) &&
+        sk_scratch(s, (size_t)8 * items, (size_t)2 * G * S1::SLOT, &sk.cnt, &sk.ws)) {
+      sk.units = U;
+      grid = G;
+    } else {
+      sk = {nullptr, nullptr, 0};
+    }
+  }
+  count_launch();
+  return launch_pdl(k_attn_pp<HD>, grid, PP_THREADS, S1::SMEM, s, tq, tk, tv, (bf16*)O, H, Lq, Lk,
+                    scale_log2, q_tok, k_tok, err, (int)items, sk);
+}
+
 }  // namespace
 
 void set_attention_schedule(int mode) { g_attn_schedule.store(mode); }
@@ -676,8 +1213,13 @@ cudaError_t attention_bf16(const AttnOperand& Q, const AttnOperand& K, const Att
   if (Lk <= 0) return cudaErrorInvalidValue;
   if ((((uintptr_t)Q.ptr) | ((uintptr_t)K.ptr) | ((uintptr_t)V.ptr) | ((uintptr_t)O)) & 15)
     return cudaErrorMisalignedAddress;
-  if (hd == 128) return launch_attn_tc<128>(Q, K, V, O, S, H, Lq, Lk, s);
-  if (hd == 64) return launch_attn_tc<64>(Q, K, V, O, S, H, Lq, Lk, s);
+  const bool one_tile = (g_attn_schedule.load() & 4) != 0;
+  if (hd == 128)
+    return one_tile ? launch_attn_tc<128>(Q, K, V, O, S, H, Lq, Lk, s)
+                    : launch_attn_pp<128>(Q, K, V, O, S, H, Lq, Lk, s);
+  if (hd == 64)
+    return one_tile ? launch_attn_tc<64>(Q, K, V, O, S, H, Lq, Lk, s)
+                    : launch_attn_pp<64>(Q, K, V, O, S, H, Lq, Lk, s);
   return cudaErrorInvalidValue;
 }
 

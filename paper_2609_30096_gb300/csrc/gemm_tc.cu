@@ -86,6 +86,25 @@ constexpr int SK_MAX_PARTS = 4;     // the host only picks stream-K when no tile
 // of one 64-deep k-block of a 256-wide tile = 406 (about 0.33 us).
 constexpr double SK_FIXUP = 10000.0;
 
+// Work tile -> (row unit, column tile).  Tiles are numbered in groups of
+// RASTER_GROUP row units: inside a group the row unit varies fastest, then the
+// column tile.  The ~152 tiles in flight at a time then span about 32 row units
+// and 152/32 column tiles, whose A and W blocks stay in L2 while they are
+// reused, instead of one column of up to all row units, which streams all of A
+// from DRAM once per column tile when A is larger than L2.  With at most
+// RASTER_GROUP row units (3510 tokens: 28) this is the plain column order.
+constexpr int RASTER_GROUP = 32;
+
+__device__ __forceinline__ void tile_coords(int tile, int m_units, int n_tiles, int& mu, int& nt) {
+  const int per_group = RASTER_GROUP * n_tiles;
+  const int g = tile / per_group;
+  const int first = g * RASTER_GROUP;
+  const int rows = m_units - first < RASTER_GROUP ? m_units - first : RASTER_GROUP;
+  const int local = tile - g * per_group;
+  mu = first + local % rows;
+  nt = local / rows;
+}
+
 template <int BN, int STAGES>
 struct TcShape {
   static constexpr uint32_t A_BYTES = BM * BK * 2;
@@ -166,7 +185,9 @@ __global__ void __launch_bounds__(192, 1)
       SegIter it(use_sk, sk.units, num_tiles, nk, worker, workers);
       int tile, kb0, kb1;
       while (it.next(tile, kb0, kb1)) {
-        const int mt = (tile % m_units) * CL + rank, nt = tile / m_units;
+        int mu, nt;
+        tile_coords(tile, m_units, n_tiles, mu, nt);
+        const int mt = mu * CL + rank;
         bool ok = true;
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(su32(&empty[stage]), phase ^ 1, abort_flag, g.err, 1)) {
@@ -253,7 +274,9 @@ __global__ void __launch_bounds__(192, 1)
     SegIter it(use_sk, U, num_tiles, nk, worker, workers);
     int tile, kb0, kb1;
     while (it.next(tile, kb0, kb1)) {
-      const int mt = (tile % m_units) * CL + rank, nt = tile / m_units;
+      int mu, nt;
+        tile_coords(tile, m_units, n_tiles, mu, nt);
+        const int mt = mu * CL + rank;
       const bool final_seg = it.done();
       // Bias and gate of this tile's columns are pulled into L1 while the MMAs run
       // (lane l: columns 8l..8l+7); the column loop below reads them with

@@ -776,7 +776,8 @@ int track_gemm_schedule(int mode) {
 }
 
 int track_attention_schedule(int mode) {
-  if (mode < TRACK_GEMM_AUTO || mode > TRACK_GEMM_STREAM_K)
+  if ((mode & ~TRACK_ATTN_ONE_TILE) < TRACK_GEMM_AUTO ||
+      (mode & ~TRACK_ATTN_ONE_TILE) > TRACK_GEMM_STREAM_K)
     return fail(TRACK_EINVAL, "unknown attention schedule");
   set_attention_schedule(mode);
   return TRACK_OK;

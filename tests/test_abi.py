@@ -115,9 +115,10 @@ def test_gemm_schedule_modes(T):
 
 
 def test_attention_schedule_modes(T):
-    for mode in (T.GEMM_DATA_PARALLEL, T.GEMM_STREAM_K, T.GEMM_AUTO):
+    for mode in (T.GEMM_DATA_PARALLEL, T.GEMM_STREAM_K, T.GEMM_DATA_PARALLEL | T.ATTN_ONE_TILE,
+                 T.GEMM_STREAM_K | T.ATTN_ONE_TILE, T.ATTN_ONE_TILE, T.GEMM_AUTO):
         T.track_attention_schedule(mode)
-    for bad in (-1, 3, T.GEMM_STREAM_K | T.GEMM_MULTICAST):
+    for bad in (-1, 3, 7, 8, 12):
         with pytest.raises(T.TrackError) as e:
             T.track_attention_schedule(bad)
         assert e.value.code == T.TRACK_EINVAL

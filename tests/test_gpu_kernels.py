@@ -256,8 +256,9 @@ def test_attention_growing_logits(T, hd):
     assert rel_l2(O.float().cpu().numpy(), _attn_ref(Q, K, V)) < 1e-2
 
 
-# Both attention schedules at shapes where stream-K splits query tiles over 2
-# (bench shape, ragged keys, hd 64), 3 and 4 CTAs; each run twice for bits.
+# Both attention schedules of both kernels (a pair of query tiles per work
+# item, and one) at shapes where stream-K splits items over 2 (bench shape,
+# ragged keys, hd 64), 3 and 4 CTAs; each run twice for bits.
 ATTN_SCHED_CASES = [
     (1, 12, 3510, 3510, 128),
     (4, 16, 1000, 700, 128),
@@ -267,9 +268,10 @@ ATTN_SCHED_CASES = [
 ]
 
 
-@pytest.fixture(params=["dp", "sk"])
+@pytest.fixture(params=["dp", "sk", "one-tile dp", "one-tile sk"])
 def attn_schedule(T, request):
-    T.track_attention_schedule(T.GEMM_DATA_PARALLEL if request.param == "dp" else T.GEMM_STREAM_K)
+    mode = T.GEMM_DATA_PARALLEL if request.param.endswith("dp") else T.GEMM_STREAM_K
+    T.track_attention_schedule(mode | (T.ATTN_ONE_TILE if "one-tile" in request.param else 0))
     yield request.param
     T.track_attention_schedule(T.GEMM_AUTO)
 
