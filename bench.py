@@ -295,6 +295,7 @@ def run_ours(args):
         tdist.init_process_group("nccl")
     _build.build()
     T.track_gemm_schedule(GEMM_SCHEDULES[args.gemm_schedule])
+    T.track_gemm_raster(args.gemm_raster)
     T.track_attention_schedule(GEMM_SCHEDULES[args.attn_schedule]
                                 | (T.ATTN_ONE_TILE if args.attn_one_tile else 0))
 
@@ -597,6 +598,7 @@ def run_kernel(args):
     _build.build()
     torch.cuda.set_device(0)
     T.track_gemm_schedule(GEMM_SCHEDULES[args.gemm_schedule])
+    T.track_gemm_raster(args.gemm_raster)
     T.track_attention_schedule(GEMM_SCHEDULES[args.attn_schedule]
                                 | (T.ATTN_ONE_TILE if args.attn_one_tile else 0))
     wl = synth.WORKLOADS[args.workload]
@@ -699,6 +701,8 @@ def main():
                     help="bf16 GEMM schedule: makespan model, data-parallel or stream-K")
     ap.add_argument("--attn-schedule", choices=["auto", "dp", "sk"], default="auto",
                     help="bf16 attention schedule: makespan model, data-parallel or stream-K")
+    ap.add_argument("--gemm-raster", type=int, default=0,
+                    help="bf16 GEMM raster group in 128-row units (0: the default)")
     ap.add_argument("--attn-one-tile", action="store_true",
                     help="attention work items of one query tile instead of a pair")
     args = ap.parse_args()

@@ -327,6 +327,17 @@ int track_linear(int dtype, const void* X, const void* W, const float* bias, int
 #define TRACK_GEMM_MULTICAST 4
 int track_gemm_schedule(int mode);
 
+/* Tile order of the TRACK_BF16 GEMM (process-wide): output tiles are taken in
+ * groups of `group` 128-row units (256 with TRACK_GEMM_MULTICAST), the row unit
+ * varying fastest inside a group, then the 128-to-256-column tile.  The tiles
+ * running at one time then share few A and W blocks, which stay in L2 while
+ * they are reused.  A group at least as large as the row-unit count is plain
+ * column order.  0 restores the default: column order for outputs of at most
+ * 32 column tiles, groups of 32 above.  Data-parallel results do not depend
+ * on the order; under stream-K it moves the split points between tiles (fp32
+ * rounding only).  EINVAL outside 0..65536. */
+int track_gemm_raster(int group);
+
 /* Schedule of the TRACK_BF16 attention kernel (process-wide), with the mode
  * values of track_gemm_schedule (no multicast), optionally or-ed with
  * TRACK_ATTN_ONE_TILE.  The kernel is persistent, at most one CTA per SM, and

@@ -61,6 +61,7 @@ def lib():
         "track_profile_enable": (_I, [_I]),
         "track_gemm_schedule": (_I, [_I]),
         "track_attention_schedule": (_I, [_I]),
+        "track_gemm_raster": (_I, [_I]),
         "track_profile_read": (_I, [_P, _P, _P]),
         "track_weight_count": (_I, [_P]),
         "track_weight_shape": (_I, [_P, _I, _P, _P]),
@@ -152,6 +153,11 @@ def track_gemm_schedule(mode: int):
     """GEMM_AUTO, GEMM_DATA_PARALLEL or GEMM_STREAM_K (optionally | GEMM_MULTICAST)
     for every later bf16 GEMM."""
     _check(lib().track_gemm_schedule(int(mode)))
+
+
+def track_gemm_raster(group: int):
+    """Row units per raster group of every later bf16 GEMM (0: the default)."""
+    _check(lib().track_gemm_raster(int(group)))
 
 
 def track_attention_schedule(mode: int):

@@ -87,19 +87,26 @@ constexpr int SK_MAX_PARTS = 4;     // the host only picks stream-K when no tile
 constexpr double SK_FIXUP = 10000.0;
 
 // Work tile -> (row unit, column tile).  Tiles are numbered in groups of
-// RASTER_GROUP row units: inside a group the row unit varies fastest, then the
-// column tile.  The ~152 tiles in flight at a time then span about 32 row units
-// and 152/32 column tiles, whose A and W blocks stay in L2 while they are
+// `group` row units: inside a group the row unit varies fastest, then the
+// column tile.  The ~152 tiles in flight at a time then span `group` row units
+// and 152/group column tiles, whose A and W blocks stay in L2 while they are
 // reused, instead of one column of up to all row units, which streams all of A
 // from DRAM once per column tile when A is larger than L2.  With at most
-// RASTER_GROUP row units (3510 tokens: 28) this is the plain column order.
-constexpr int RASTER_GROUP = 32;
+// `group` row units (3510 tokens: 28) this is the plain column order.
+// Measured at 32760 rows and K 5120 (14B shapes): groups of 32 made the FFN
+// up-projection (54 column tiles) 21 % faster than column order, but the 20-
+// column-tile projections 20-30 % slower; the default therefore keeps column
+// order up to RASTER_NARROW column tiles and groups of 32 above.
+constexpr int RASTER_DEFAULT = 32;
+constexpr int RASTER_NARROW = 32;
 
-__device__ __forceinline__ void tile_coords(int tile, int m_units, int n_tiles, int& mu, int& nt) {
-  const int per_group = RASTER_GROUP * n_tiles;
+__device__ __forceinline__ void tile_coords(int tile, int m_units, int n_tiles, int group, int& mu,
+                                            int& nt) {
+  if (group > m_units) group = m_units;  // per_group <= the tile count: no overflow
+  const int per_group = group * n_tiles;
   const int g = tile / per_group;
-  const int first = g * RASTER_GROUP;
-  const int rows = m_units - first < RASTER_GROUP ? m_units - first : RASTER_GROUP;
+  const int first = g * group;
+  const int rows = m_units - first < group ? m_units - first : group;
   const int local = tile - g * per_group;
   mu = first + local % rows;
   nt = local / rows;
@@ -186,7 +193,7 @@ __global__ void __launch_bounds__(192, 1)
       int tile, kb0, kb1;
       while (it.next(tile, kb0, kb1)) {
         int mu, nt;
-        tile_coords(tile, m_units, n_tiles, mu, nt);
+        tile_coords(tile, m_units, n_tiles, g.raster, mu, nt);
         const int mt = mu * CL + rank;
         bool ok = true;
         for (int kb = kb0; kb < kb1; ++kb) {
@@ -275,7 +282,7 @@ __global__ void __launch_bounds__(192, 1)
     int tile, kb0, kb1;
     while (it.next(tile, kb0, kb1)) {
       int mu, nt;
-        tile_coords(tile, m_units, n_tiles, mu, nt);
+        tile_coords(tile, m_units, n_tiles, g.raster, mu, nt);
         const int mt = mu * CL + rank;
       const bool final_seg = it.done();
       // Bias and gate of this tile's columns are pulled into L1 while the MMAs run
@@ -589,10 +596,15 @@ int max_workers() {
   return n;
 }
 
+std::atomic<int> g_gemm_raster{0};  // 0: the default rule above
+
 template <int BN, int STAGES, int CL>
-cudaError_t launch_tc(const void* A, const void* W, const GemmArgs& g, bool stream_k,
+cudaError_t launch_tc(const void* A, const void* W, const GemmArgs& g_in, bool stream_k,
                       cudaStream_t s) {
   using S = TcShape<BN, STAGES>;
+  GemmArgs g = g_in;
+  g.raster = g_gemm_raster.load();
+  if (g.raster <= 0) g.raster = (g.N + BN - 1) / BN <= RASTER_NARROW ? (1 << 30) : RASTER_DEFAULT;
   static_assert(S::SMEM <= 232448, "shared memory budget");
   CUtensorMap ta, tb, tc;
   const CUtensorMapDataType BF = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
@@ -739,6 +751,7 @@ std::atomic<int> g_schedule{0};
 }
 
 void set_gemm_schedule(int mode) { g_schedule.store(mode); }
+void set_gemm_raster(int group) { g_gemm_raster.store(group > 0 ? group : 0); }
 
 cudaError_t gemm_bf16_tc(const void* A, const void* W, const GemmArgs& g, cudaStream_t s) {
   if (g.M <= 0 || g.N <= 0) return cudaSuccess;

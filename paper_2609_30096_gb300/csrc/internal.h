@@ -77,10 +77,13 @@ struct GemmArgs {
   void* out;           // T [M, ldo] (STORE/GELU) or fp32 [M, ldo] (RESID*)
   int ldo;
   int* err;            // device error word
+  int raster;          // bf16 tensor-core GEMM: row units per raster group (set by its launcher)
 };
 
 // fp32 FFMA GEMM: out = A[M,K] . W[N,K]^T (+ epilogue), all fp32.
 cudaError_t gemm_f32(const float* A, const float* W, const GemmArgs& g, cudaStream_t s);
+// Row units per raster group of the bf16 tensor-core GEMM (0: the default).
+void set_gemm_raster(int group);
 
 // bf16 tcgen05 GEMM: A bf16 [M,K] and W bf16 [N,K], fp32 accumulation in TMEM.
 // Requires K % 64 == 0, N % 32 == 0 and 16-byte aligned A, W and out.

@@ -775,6 +775,12 @@ int track_gemm_schedule(int mode) {
   return TRACK_OK;
 }
 
+int track_gemm_raster(int group) {
+  if (group < 0 || group > 65536) return fail(TRACK_EINVAL, "raster group out of range");
+  set_gemm_raster(group);
+  return TRACK_OK;
+}
+
 int track_attention_schedule(int mode) {
   if ((mode & ~TRACK_ATTN_ONE_TILE) < TRACK_GEMM_AUTO ||
       (mode & ~TRACK_ATTN_ONE_TILE) > TRACK_GEMM_STREAM_K)

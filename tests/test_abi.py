@@ -114,6 +114,15 @@ def test_gemm_schedule_modes(T):
         assert e.value.code == T.TRACK_EINVAL
 
 
+def test_gemm_raster_groups(T):
+    for group in (1, 8, 32, 65536, 0):
+        T.track_gemm_raster(group)
+    for bad in (-1, 65537):
+        with pytest.raises(T.TrackError) as e:
+            T.track_gemm_raster(bad)
+        assert e.value.code == T.TRACK_EINVAL
+
+
 def test_attention_schedule_modes(T):
     for mode in (T.GEMM_DATA_PARALLEL, T.GEMM_STREAM_K, T.GEMM_DATA_PARALLEL | T.ATTN_ONE_TILE,
                  T.GEMM_STREAM_K | T.ATTN_ONE_TILE, T.ATTN_ONE_TILE, T.GEMM_AUTO):

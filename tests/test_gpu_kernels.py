@@ -157,6 +157,42 @@ def test_linear_bf16_schedules_agree(T):
     assert rel_l2(res[1], res[0]) < 2e-5
 
 
+@pytest.mark.parametrize("mode", ["dp", "sk", "dp+multicast"])
+def test_linear_bf16_raster_groups_agree(T, mode):
+    # The tile order changes which CTA computes a tile, never a data-parallel
+    # tile's arithmetic: every raster group gives the same bits (65 row units,
+    # ragged).  Under stream-K the order also moves the split points between
+    # tiles, so split tiles may round differently (fp32 sums in another order,
+    # then bf16): about one bf16 step apart.
+    rng = np.random.default_rng(12)
+    M, N, K = 8250, 1024, 1536
+    X = dev_bf16(rng.normal(size=(M, K)).astype(np.float32))
+    W = dev_bf16((rng.normal(size=(N, K)) / np.sqrt(K)).astype(np.float32))
+    b = dev_f32(rng.normal(size=N).astype(np.float32))
+    T.track_gemm_schedule({"dp": T.GEMM_DATA_PARALLEL, "sk": T.GEMM_STREAM_K,
+                           "dp+multicast": T.GEMM_DATA_PARALLEL | T.GEMM_MULTICAST}[mode])
+    res = []
+    try:
+        for group in (0, 1, 5, 32, 65536):
+            T.track_gemm_raster(group)
+            out = torch.zeros((M, N), dtype=torch.bfloat16, device=DEV)
+            T.track_linear(T.BF16, X, W, b, T.EPI_STORE, out)
+            T.track_sync()
+            res.append(out.float().cpu().numpy())
+    finally:
+        T.track_gemm_raster(0)
+        T.track_gemm_schedule(T.GEMM_AUTO)
+    for r in res[1:]:
+        if mode == "sk":
+            scale = np.sqrt(np.mean(res[0] ** 2))
+            assert np.all(np.abs(r - res[0]) <= 2.0 ** -7 * np.abs(res[0]) + 1e-3 * scale)
+        else:
+            assert np.array_equal(r, res[0])
+    ref = dit.linear(dit.round_bf16(X.float().cpu().numpy()[::97]), W.float().cpu().numpy(),
+                     b.cpu().numpy())
+    assert rel_l2(res[0][::97], ref) < 4e-3
+
+
 @pytest.mark.parametrize("M,N,K", [(1, 32, 64), (100, 96, 80), (513, 700, 256)])
 @pytest.mark.parametrize("epi", [0, 1, 2, 3])
 def test_linear_fp32(T, M, N, K, epi):
