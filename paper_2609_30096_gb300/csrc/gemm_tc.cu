@@ -176,9 +176,14 @@ __global__ void __launch_bounds__(192, 1)
   if (CL > 1) cluster_sync();  // the peer's barriers exist before any multicast reaches them
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  // The prologue above overlaps the previous kernel; inputs and outputs are touched only now.
-  pdl_wait();
-  pdl_release();
+  // The prologue above overlaps the previous kernel; inputs and outputs are touched only
+  // after the grid dependency wait.  The producer thread first requests the W tiles of
+  // its first stages: weights are never written by an earlier kernel.
+  const bool producer = warp == 0 && lane == 0;
+  if (!producer) {
+    pdl_wait();
+    pdl_release();
+  }
 
   if (warp == 0) {
     if (lane == 0) {
@@ -190,6 +195,23 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
       for (int i = 0; i < STAGES; ++i) armed[i] = 0;
       SegIter it(use_sk, sk.units, num_tiles, nk, worker, workers);
+      int pre = 0;  // k-blocks of the first segment whose W tile is already requested
+      if (CL == 1) {
+        SegIter first = it;
+        int t0, a0, a1;
+        if (first.next(t0, a0, a1)) {
+          int mu0, nt0;
+          tile_coords(t0, m_units, n_tiles, g.raster, mu0, nt0);
+          pre = a1 - a0 < STAGES ? a1 - a0 : STAGES;
+          for (int i = 0; i < pre; ++i) {  // fresh stages: no empty wait
+            const uint32_t fb = su32(&full[i]);
+            mbar_expect_tx(fb, S::A_BYTES + S::B_BYTES);
+            tma_load_2d(su32(sB + i * S::B_BYTES), &tmB, (a0 + i) * BK, nt0 * BN, fb);
+          }
+        }
+      }
+      pdl_wait();
+      pdl_release();
       int tile, kb0, kb1;
       while (it.next(tile, kb0, kb1)) {
         int mu, nt;
@@ -197,11 +219,21 @@ __global__ void __launch_bounds__(192, 1)
         const int mt = mu * CL + rank;
         bool ok = true;
         for (int kb = kb0; kb < kb1; ++kb) {
+          const uint32_t fb = su32(&full[stage]);
+          if (pre > 0) {  // W of this stage requested before the dependency wait
+            --pre;
+            tma_load_2d(su32(sA + stage * S::A_BYTES), &tmA, kb * BK, mt * BM, fb);
+            ++armed[stage];
+            if (++stage == STAGES) {
+              stage = 0;
+              phase ^= 1;
+            }
+            continue;
+          }
           if (!mbar_wait(su32(&empty[stage]), phase ^ 1, abort_flag, g.err, 1)) {
             ok = false;
             break;
           }
-          const uint32_t fb = su32(&full[stage]);
           mbar_expect_tx(fb, S::A_BYTES + S::B_BYTES);
           tma_load_2d(su32(sA + stage * S::A_BYTES), &tmA, kb * BK, mt * BM, fb);
           if (CL == 1) {
