@@ -512,7 +512,7 @@ def run_ours(args):
     dm, dflops, dn = prof[dominant]
     achieved = (dflops / dn) / (dm / dn / 1e3) / 1e12 if dn else None
     peak = peaks["bf16_tflops"]
-    traffic, traffic_src = measured_traffic("k_gemm_tc" if dominant == "gemm" else "k_attn_tc",
+    traffic, traffic_src = measured_traffic("k_gemm_tc" if dominant == "gemm" else "k_attn_pp",
                                             dflops / dn if dn else 0.0)
     roof = {"bound": "tensor", "kernel": "bf16 GEMM (tcgen05)" if dominant == "gemm"
             else "flash attention (tcgen05)",
