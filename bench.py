@@ -583,6 +583,79 @@ def run_ours(args):
     return 0
 
 
+# ---------------------------------------------------------------- 14B/1.3B configurations
+def run_workload(args):
+    """One guided denoiser evaluation of each model of a 14B/1.3B configuration at its
+    full size (its batch and CFG), timed with CUDA events after warm-up.  A trajectory
+    evaluates one denoiser per step (Eq. 3), so its latency is the per-step costs summed
+    over the policy: all-large N C_L, routed (N - K) C_L + K C_S.  The mid workload
+    measures that sum directly (`cost_model`, within 1 %); at these sizes a trajectory
+    of 30-50 full-size steps would take minutes, and calibrating one longer."""
+    import torch
+
+    import paper_2609_30096_gb300 as T
+    from paper_2609_30096_gb300 import _build
+
+    _build.build()
+    torch.cuda.set_device(0)
+    T.track_gemm_schedule(GEMM_SCHEDULES[args.gemm_schedule])
+    T.track_gemm_raster(args.gemm_raster)
+    T.track_attention_schedule(GEMM_SCHEDULES[args.attn_schedule]
+                               | (T.ATTN_ONE_TILE if args.attn_one_tile else 0))
+    wl = synth.WORKLOADS[args.workload]
+    B, w = wl.batch, wl.cfg
+    guided = 2 if w != 1.0 else 1
+    sig = T.track_schedule(wl.steps, wl.shift)
+    x0, c0, u0 = synth.evaluation_inputs(wl.large, 0, B, w != 1.0)
+    stream = torch.cuda.Stream()
+    torch.cuda.set_stream(stream)
+    sid = stream.cuda_stream
+    x = torch.from_numpy(x0).cuda()
+    c = torch.from_numpy(c0).cuda()
+    u = torch.from_numpy(u0).cuda() if u0 is not None else None
+    v = torch.empty_like(x)
+    t = float(np.float32(np.float32(1000.0) * np.float32(sig[wl.steps // 2])))
+    peaks, src = load_peaks()
+    res, clocks = {}, None
+    for which, arch, seed in (("large", wl.large, synth.SEED_LARGE),
+                              ("small", wl.small, synth.SEED_SMALL)):
+        m = T.track_model_create_seeded(arch, seed, T.BF16)
+        for _ in range(args.warmup):
+            T.track_denoise(m, x, t, c, u, w, v, stream=sid)
+        T.track_sync(sid)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with ClockSampler(0) as clk:
+            a.record(stream)
+            for _ in range(args.steps):
+                T.track_denoise(m, x, t, c, u, w, v, stream=sid)
+            b.record(stream)
+            T.track_sync(sid)
+        if which == "large":
+            clocks = clk.summary()
+        ms = a.elapsed_time(b) / args.steps
+        tf = forward_flops(arch, guided * B) / (ms / 1e3) / 1e12
+        res[which] = {"ms": ms, "tflops": tf, "frac_of_bf16_peak": tf / peaks["bf16_tflops"],
+                      "params": synth.param_count(arch)}
+        m.close()
+        del m
+        torch.cuda.empty_cache()
+    cl, cs = res["large"]["ms"], res["small"]["ms"]
+    n, k = wl.steps, wl.k
+    line = {
+        "workload_bench": args.workload, "workload": wl.description, "dtype": "bf16",
+        "data": "synthetic", "sequences_per_forward": guided * B,
+        "tokens_per_sequence": wl.large.tokens, "steps": args.steps, "warmup": args.warmup,
+        "forward_large": res["large"], "forward_small": res["small"],
+        "denoise_steps_per_s_large": 1e3 / cl, "denoise_steps_per_s_small": 1e3 / cs,
+        "trajectory_all_large_s": n * cl / 1e3, "trajectory_routed_s": ((n - k) * cl + k * cs) / 1e3,
+        "routed_speedup": n * cl / ((n - k) * cl + k * cs),
+        "routed": f"K={k} of {n} steps on the small model (sum of measured per-step costs)",
+        "peak_source": src, "clocks": clocks,
+    }
+    print(json.dumps(line))
+    return 0
+
+
 # ---------------------------------------------------------------- single kernels
 GEMM_SCHEDULES = {"auto": 0, "dp": 1, "sk": 2}   # track_gemm/attention_schedule modes
 
@@ -696,7 +769,8 @@ def main():
                     help="time one kernel class alone at the workload's shapes")
     ap.add_argument("--batch", type=int, default=1, help="sequences for --kernel")
     ap.add_argument("--workload", choices=sorted(synth.WORKLOADS), default=WORKLOAD,
-                    help="shapes for --kernel (the full benchmark always runs the mid pair)")
+                    help="shapes for --kernel; without --kernel, a 14B/1.3B configuration "
+                         "times one full-size denoiser evaluation of each model")
     ap.add_argument("--gemm-schedule", choices=["auto", "dp", "sk"], default="auto",
                     help="bf16 GEMM schedule: makespan model, data-parallel or stream-K")
     ap.add_argument("--attn-schedule", choices=["auto", "dp", "sk"], default="auto",
@@ -707,12 +781,14 @@ def main():
                     help="attention work items of one query tile instead of a pair")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)     # at least three untimed warm-up steps
-    if args.workload != WORKLOAD and not args.kernel:
-        ap.error("--workload applies to --kernel only")
     if args.impl == "reference":
         return run_reference(args)
     if args.kernel:
         return run_kernel(args)
+    if args.workload != WORKLOAD:
+        if args.gpus != 1 or int(os.environ.get("WORLD_SIZE", "1")) != 1:
+            ap.error("--workload runs on one GPU")
+        return run_workload(args)
     return run_ours(args)
 
 
