@@ -94,6 +94,26 @@ int track_sync(track_stream s);
 /* Number of kernels this library has launched since load (returns the count). */
 int64_t track_launch_count(void);
 
+/* Failure detection, exercised without a GPU fault.
+ *
+ * track_wait_selftest launches one CTA whose thread waits, through the same
+ * bounded mbarrier wait every tensor-core kernel uses for its pipeline, on a
+ * barrier that nothing completes.  After limit_cycles SM cycles the wait gives
+ * up: the CTA records TRACK_WAIT_SELFTEST_CODE in the device error word and
+ * exits, and the context stays usable.  Returns TRACK_OK once launched on s;
+ * the next track_sync on s then returns TRACK_ETIMEOUT naming that code and
+ * clears the word.  EINVAL unless 1e3 <= limit_cycles <= 2e9 (the kernels'
+ * own limit is 2e9 cycles, about one second).
+ *
+ * track_fail_next_allocations makes the next n device allocations the library
+ * makes for itself (weights, workspaces, scratch) fail as if the device were
+ * out of memory: the call that needed one returns TRACK_ENOMEM, or, where a
+ * fallback exists (stream-K scratch), takes it.  n = 0 clears pending
+ * failures; EINVAL for n < 0. */
+#define TRACK_WAIT_SELFTEST_CODE 99
+int track_wait_selftest(int64_t limit_cycles, track_stream s);
+int track_fail_next_allocations(int n);
+
 /* Kernel timing: while enabled, the GEMM, attention and normalization
  * launches inside track_denoise/track_denoise_step/track_calibrate/track_sample
  * are bracketed by CUDA events on their stream.  track_profile_read

@@ -18,6 +18,7 @@ import numpy as np
 from ._build import LIB as _LIB_PATH
 
 TRACK_OK, TRACK_EINVAL, TRACK_ENOMEM, TRACK_ECUDA, TRACK_EUNSUPPORTED, TRACK_ETIMEOUT = range(6)
+TRACK_WAIT_SELFTEST_CODE = 99  # error-word code of track_wait_selftest
 FP32, BF16 = 0, 1
 EPI_STORE, EPI_GELU, EPI_RESID_GATE, EPI_RESID = range(4)
 GEMM_AUTO, GEMM_DATA_PARALLEL, GEMM_STREAM_K = range(3)
@@ -62,6 +63,8 @@ def lib():
         "track_gemm_schedule": (_I, [_I]),
         "track_attention_schedule": (_I, [_I]),
         "track_gemm_raster": (_I, [_I]),
+        "track_wait_selftest": (_I, [ctypes.c_int64, _P]),
+        "track_fail_next_allocations": (_I, [_I]),
         "track_profile_read": (_I, [_P, _P, _P]),
         "track_weight_count": (_I, [_P]),
         "track_weight_shape": (_I, [_P, _I, _P, _P]),
@@ -153,6 +156,17 @@ def track_gemm_schedule(mode: int):
     """GEMM_AUTO, GEMM_DATA_PARALLEL or GEMM_STREAM_K (optionally | GEMM_MULTICAST)
     for every later bf16 GEMM."""
     _check(lib().track_gemm_schedule(int(mode)))
+
+
+def track_wait_selftest(limit_cycles: int, stream=None):
+    """Launches a bounded pipeline wait that is made to run out; the next track_sync
+    raises TrackError(TRACK_ETIMEOUT) naming TRACK_WAIT_SELFTEST_CODE."""
+    _check(lib().track_wait_selftest(int(limit_cycles), _stream(stream)))
+
+
+def track_fail_next_allocations(n: int):
+    """The next n device allocations of the library fail as out-of-memory (0 clears)."""
+    _check(lib().track_fail_next_allocations(int(n)))
 
 
 def track_gemm_raster(group: int):

@@ -760,8 +760,8 @@ bool sk_scratch(cudaStream_t s, size_t ncnt, size_t nws, int** cnt, float** ws) 
     cudaFree(sc.ws);
     sc = SkScratch();
     const size_t nc = ncnt > 4096 ? ncnt : 4096, nw = nws;
-    if (cudaMalloc(&sc.cnt, nc * sizeof(int)) != cudaSuccess ||
-        cudaMalloc(&sc.ws, nw * sizeof(float)) != cudaSuccess ||
+    if (dev_malloc((void**)&sc.cnt, nc * sizeof(int)) != cudaSuccess ||
+        dev_malloc((void**)&sc.ws, nw * sizeof(float)) != cudaSuccess ||
         cudaMemsetAsync(sc.cnt, 0, nc * sizeof(int), s) != cudaSuccess) {
       cudaGetLastError();
       cudaFree(sc.cnt);
@@ -783,6 +783,27 @@ std::atomic<int> g_schedule{0};
 }
 
 void set_gemm_schedule(int mode) { g_schedule.store(mode); }
+
+namespace {
+__global__ void k_wait_selftest(int* err, long long limit, int code) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(su32(&bar), 1);
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  // Nothing arrives on the barrier: its phase 0 never completes.
+  if (threadIdx.x == 0) mbar_wait(su32(&bar), 0, &abort_flag, err, code, limit);
+}
+}  // namespace
+
+cudaError_t wait_selftest(int* err, long long limit, int code, cudaStream_t s) {
+  k_wait_selftest<<<1, 32, 0, s>>>(err, limit, code);
+  count_launch();
+  return cudaGetLastError();
+}
 void set_gemm_raster(int group) { g_gemm_raster.store(group > 0 ? group : 0); }
 
 cudaError_t gemm_bf16_tc(const void* A, const void* W, const GemmArgs& g, cudaStream_t s) {

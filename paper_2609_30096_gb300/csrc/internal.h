@@ -84,6 +84,15 @@ struct GemmArgs {
 cudaError_t gemm_f32(const float* A, const float* W, const GemmArgs& g, cudaStream_t s);
 // Row units per raster group of the bf16 tensor-core GEMM (0: the default).
 void set_gemm_raster(int group);
+// Device allocation of the library's own buffers (weights, workspaces,
+// scratch); fails like an exhausted device while track_fail_next_allocations
+// has failures pending.
+cudaError_t dev_malloc(void** p, size_t bytes);
+void set_failing_allocations(int n);
+// One CTA waits, through the tensor-core kernels' bounded mbarrier wait, on a
+// barrier nothing completes; after `limit` SM cycles the wait gives up and
+// records `code` in the device error word.
+cudaError_t wait_selftest(int* err, long long limit, int code, cudaStream_t s);
 
 // bf16 tcgen05 GEMM: A bf16 [M,K] and W bf16 [N,K], fp32 accumulation in TMEM.
 // Requires K % 64 == 0, N % 32 == 0 and 16-byte aligned A, W and out.

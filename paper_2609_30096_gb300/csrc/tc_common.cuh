@@ -37,15 +37,16 @@ __device__ __forceinline__ uint32_t mbar_try(uint32_t bar, uint32_t parity) {
   return ok;
 }
 // Waits for the phase with the given parity to complete.  Returns false if the
-// CTA was aborted or the wait ran out (then the abort flag is raised).
+// CTA was aborted or the wait ran out after `limit` SM cycles (then the abort
+// flag is raised and `code` is recorded in the device error word).
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                          int* err, int code) {
+                                          int* err, int code, long long limit = WAIT_LIMIT) {
   if (mbar_try(bar, parity)) return true;
   const long long t0 = clock64();
   while (true) {
     if (mbar_try(bar, parity)) return true;
     if (*abort_flag) return false;
-    if (clock64() - t0 > WAIT_LIMIT) {
+    if (clock64() - t0 > limit) {
       *abort_flag = 1;
       atomicExch(err, code);
       return false;

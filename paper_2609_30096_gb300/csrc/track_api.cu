@@ -68,6 +68,22 @@ int num_sms() {
   return n;
 }
 
+// Pending injected allocation failures (track_fail_next_allocations).
+static std::atomic<int> g_failing_allocs{0};
+
+void set_failing_allocations(int n) { g_failing_allocs.store(n); }
+
+cudaError_t dev_malloc(void** p, size_t bytes) {
+  int pending = g_failing_allocs.load();
+  while (pending > 0) {
+    if (g_failing_allocs.compare_exchange_weak(pending, pending - 1)) {
+      *p = nullptr;
+      return cudaErrorMemoryAllocation;
+    }
+  }
+  return cudaMalloc(p, bytes);
+}
+
 int* device_error_word() {
   const int dev = current_device();
   std::lock_guard<std::mutex> lk(g_dev_mu);
@@ -395,7 +411,11 @@ static int build_rope_table(track_model* m) {
         tab[o++] = make_float2((float)cos(ang), (float)sin(ang));
       }
   }
-  TRACK_CUDA(cudaMalloc(&m->rope_tab, tab.size() * sizeof(float2)));
+  if (dev_malloc((void**)&m->rope_tab, tab.size() * sizeof(float2)) != cudaSuccess) {
+    cudaGetLastError();
+    m->rope_tab = nullptr;
+    return fail(TRACK_ENOMEM, "rope table allocation failed");
+  }
   TRACK_CUDA(cudaMemcpy(m->rope_tab, tab.data(), tab.size() * sizeof(float2),
                         cudaMemcpyHostToDevice));
   return TRACK_OK;
@@ -441,7 +461,7 @@ static int ensure_workspace(track_model* m, int nseq) {
   sz((size_t)a.layers * 6 * d * 4);
   sz(2 * d * 4);
   void* base = nullptr;
-  cudaError_t e = cudaMalloc(&base, need);
+  cudaError_t e = dev_malloc((void**)&base, need);
   if (e != cudaSuccess) {
     cudaGetLastError();
     return fail(TRACK_ENOMEM, std::string("workspace allocation failed: ") + cudaGetErrorString(e));
@@ -479,7 +499,7 @@ static int ensure_calib(track_model* m, int B) {
   w.calib_cap = 0;
   const size_t n = (size_t)B * m->latent_n;
   float* p = nullptr;
-  if (cudaMalloc(&p, 2 * n * sizeof(float)) != cudaSuccess) {
+  if (dev_malloc((void**)&p, 2 * n * sizeof(float)) != cudaSuccess) {
     cudaGetLastError();
     return fail(TRACK_ENOMEM, "calibration buffers");
   }
@@ -705,7 +725,7 @@ static float* stream_scratch(cudaStream_t s, size_t floats) {
   slot.first = nullptr;
   slot.second = 0;
   float* p = nullptr;
-  if (cudaMalloc(&p, floats * sizeof(float)) != cudaSuccess) {
+  if (dev_malloc((void**)&p, floats * sizeof(float)) != cudaSuccess) {
     cudaGetLastError();
     return nullptr;
   }
@@ -775,6 +795,22 @@ int track_gemm_schedule(int mode) {
   return TRACK_OK;
 }
 
+int track_fail_next_allocations(int n) {
+  if (n < 0) return fail(TRACK_EINVAL, "n must be non-negative");
+  set_failing_allocations(n);
+  return TRACK_OK;
+}
+
+int track_wait_selftest(int64_t limit_cycles, track_stream s) {
+  if (limit_cycles < 1000 || limit_cycles > 2000000000LL)
+    return fail(TRACK_EINVAL, "limit_cycles outside 1e3 .. 2e9");
+  int* err = device_error_word();
+  if (err == nullptr) return fail(TRACK_ECUDA, "device error word");
+  cudaError_t e = wait_selftest(err, (long long)limit_cycles, TRACK_WAIT_SELFTEST_CODE, (cudaStream_t)s);
+  if (e != cudaSuccess) return fail(TRACK_ECUDA, std::string("self-test launch: ") + cudaGetErrorString(e));
+  return TRACK_OK;
+}
+
 int track_gemm_raster(int group) {
   if (group < 0 || group > 65536) return fail(TRACK_EINVAL, "raster group out of range");
   set_gemm_raster(group);
@@ -840,7 +876,10 @@ static int model_alloc(const track_arch* arch, track_model** out, track_model** 
   track_model* m = new (std::nothrow) track_model();
   if (!m) return fail(TRACK_ENOMEM, "host allocation");
   m->a = *arch;
-  TRACK_CUDA(cudaGetDevice(&m->dev));
+  if (cudaGetDevice(&m->dev) != cudaSuccess) {
+    delete m;
+    return fail(TRACK_ECUDA, "cudaGetDevice");
+  }
   m->dtype = arch->dtype == TRACK_BF16 ? BF16 : F32;
   m->esz = m->dtype == BF16 ? 2 : 4;
   m->hd = arch->dim / arch->heads;
@@ -850,7 +889,7 @@ static int model_alloc(const track_arch* arch, track_model** out, track_model** 
   m->L_tok = m->Fp * m->Hp * m->Wp;
   m->latent_n = (int64_t)arch->in_ch * arch->frames * arch->height * arch->width;
   const size_t bytes = layout_weights(m, nullptr);
-  if (cudaMalloc(&m->wbuf, bytes) != cudaSuccess) {
+  if (dev_malloc((void**)&m->wbuf, bytes) != cudaSuccess) {
     cudaGetLastError();
     delete m;
     return fail(TRACK_ENOMEM, "weight allocation failed");
@@ -895,7 +934,7 @@ int track_model_create(const track_arch* arch, const float* const* weights, trac
     maxn = std::max(maxn, (size_t)(t.rows * t.cols));
   }
   float* staging = nullptr;
-  if (cudaMalloc(&staging, maxn * sizeof(float)) != cudaSuccess) {
+  if (dev_malloc((void**)&staging, maxn * sizeof(float)) != cudaSuccess) {
     cudaGetLastError();
     track_model_destroy(m);
     return fail(TRACK_ENOMEM, "staging allocation failed");

@@ -114,6 +114,18 @@ def test_gemm_schedule_modes(T):
         assert e.value.code == T.TRACK_EINVAL
 
 
+def test_failure_hooks_check_arguments(T):
+    # Host-side argument checks only: nothing is launched or allocated here.
+    for bad in (-1, 999, 2_000_000_001):
+        with pytest.raises(T.TrackError) as e:
+            T.track_wait_selftest(bad, stream=0)
+        assert e.value.code == T.TRACK_EINVAL
+    with pytest.raises(T.TrackError) as e:
+        T.track_fail_next_allocations(-1)
+    assert e.value.code == T.TRACK_EINVAL
+    T.track_fail_next_allocations(0)
+
+
 def test_gemm_raster_groups(T):
     for group in (1, 8, 32, 65536, 0):
         T.track_gemm_raster(group)

@@ -283,6 +283,53 @@ def test_timed_graph_brackets_every_kernel(T, tiny):
         T.track_profile_read()
 
 
+def test_abandoned_wait_is_reported_and_the_context_survives(T):
+    # The bounded pipeline wait of the tensor-core kernels, made to run out on a
+    # barrier nothing completes (about 0.5 ms of SM cycles): the next sync
+    # reports the timeout with the self-test's code, clears it, and the device
+    # keeps working.
+    s = torch.cuda.Stream()
+    T.track_sync(s.cuda_stream)
+    T.track_wait_selftest(1_000_000, stream=s.cuda_stream)
+    with pytest.raises(T.TrackError) as e:
+        T.track_sync(s.cuda_stream)
+    assert e.value.code == T.TRACK_ETIMEOUT
+    assert f"code {T.TRACK_WAIT_SELFTEST_CODE}" in str(e.value)
+    T.track_sync(s.cuda_stream)                        # cleared
+    X = torch.ones((300, 128), dtype=torch.bfloat16, device="cuda")
+    W = torch.eye(128, dtype=torch.bfloat16, device="cuda")
+    out = torch.zeros((300, 128), dtype=torch.bfloat16, device="cuda")
+    T.track_linear(T.BF16, X, W, None, T.EPI_STORE, out)
+    T.track_sync()
+    assert torch.equal(out, X)
+
+
+def test_injected_allocation_failures(T, calib_inputs):
+    # A model whose weight allocation fails is not created; a denoise whose
+    # workspace allocation fails returns ENOMEM and leaves the model usable.
+    x, c, u = calib_inputs
+    T.track_fail_next_allocations(1000)
+    try:
+        with pytest.raises(T.TrackError) as e:
+            T.track_model_create_seeded(WL.large, synth.SEED_LARGE, T.BF16)
+        assert e.value.code == T.TRACK_ENOMEM
+    finally:
+        T.track_fail_next_allocations(0)
+    m = T.track_model_create_seeded(WL.large, synth.SEED_LARGE, T.BF16)
+    T.track_fail_next_allocations(1000)   # every allocation of the call fails
+    try:
+        with pytest.raises(T.TrackError) as e:
+            T.track_denoise(m, dev(x[:1]), 500.0, dev(c[:1]), dev(u[:1]), WL.cfg)
+        assert e.value.code == T.TRACK_ENOMEM
+    finally:
+        T.track_fail_next_allocations(0)
+    v1 = T.track_denoise(m, dev(x[:1]), 500.0, dev(c[:1]), dev(u[:1]), WL.cfg)
+    v2 = T.track_denoise(m, dev(x[:1]), 500.0, dev(c[:1]), dev(u[:1]), WL.cfg)
+    T.track_sync()
+    assert torch.equal(v1, v2) and bool(torch.isfinite(v1).all())
+    m.close()
+
+
 def test_argument_errors(T, tiny, calib_inputs):
     prec, P = tiny
     x, c, u = calib_inputs
