@@ -221,6 +221,25 @@ int track_disagreement(const float* v_L, const float* v_S, int B, int64_t n_per_
  * order in double and rounded to float. */
 int track_mean_score(const float* r, int M, int N, float* q_out);
 
+/* The offline artifact of calibration (Sec. 3.2.1): the per-sample, per-step
+ * disagreement map r [M, N] (host, row j = calibration sample j) and its mean
+ * q [N] (Eq. 5), in a file, so that the policy can be rebuilt without the
+ * models and calibration resumed sample by sample (rows are independent:
+ * load, calibrate further samples, append their rows, save).  Format, all
+ * little-endian: 8 bytes "TRKSCORE", uint32 version (1), uint32 M, uint32 N,
+ * uint64 config_hash (the caller's identifier of the model pair, schedule and
+ * CFG scale), float32 r[M*N] row-major, float32 q[N] as track_mean_score
+ * computes it.
+ *
+ * track_score_map_save writes (replaces) path; EINVAL for bad arguments, a
+ * negative or NaN score, or a file that cannot be written.  track_score_map_load reads path into r (capacity r_cap floats) and
+ * q (capacity q_cap floats; q may be NULL), and sets *M, *N and *config_hash;
+ * EINVAL if the file is missing, truncated, has another magic or version, or
+ * does not fit the capacities.  Host only. */
+int track_score_map_save(const char* path, const float* r, int M, int N, uint64_t config_hash);
+int track_score_map_load(const char* path, float* r, int64_t r_cap, float* q, int64_t q_cap,
+                         int* M, int* N, uint64_t* config_hash);
+
 /* ---- policy (Eq. 6, Eq. 7, top-K switching of Sec. 3.2.3) ------------------ */
 
 /* policy_out[k] = 1 (small model) for the K steps with the lowest score, else

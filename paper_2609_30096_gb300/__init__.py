@@ -63,6 +63,10 @@ def lib():
         "track_gemm_schedule": (_I, [_I]),
         "track_attention_schedule": (_I, [_I]),
         "track_gemm_raster": (_I, [_I]),
+        "track_score_map_save": (_I, [ctypes.c_char_p, _P, _I, _I, ctypes.c_uint64]),
+        "track_score_map_load": (_I, [ctypes.c_char_p, _P, ctypes.c_int64, _P, ctypes.c_int64,
+                                      ctypes.POINTER(_I), ctypes.POINTER(_I),
+                                      ctypes.POINTER(ctypes.c_uint64)]),
         "track_wait_selftest": (_I, [ctypes.c_int64, _P]),
         "track_fail_next_allocations": (_I, [_I]),
         "track_profile_read": (_I, [_P, _P, _P]),
@@ -340,6 +344,26 @@ def track_mean_score(r) -> np.ndarray:
     q = np.zeros(r.shape[1], dtype=np.float32)
     _check(lib().track_mean_score(r.ctypes.data, r.shape[0], r.shape[1], q.ctypes.data))
     return q
+
+
+def track_score_map_save(path, r, config_hash: int = 0):
+    """Writes the calibration map r [M, N] (and its Eq. 5 mean) to path."""
+    r = np.ascontiguousarray(r, dtype=np.float32)
+    if r.ndim != 2:
+        raise TrackError(TRACK_EINVAL, "r must be [M, N]")
+    _check(lib().track_score_map_save(os.fsencode(path), r.ctypes.data, r.shape[0], r.shape[1],
+                                      int(config_hash)))
+
+
+def track_score_map_load(path):
+    """(r [M, N], q [N], config_hash) read from a score-map file."""
+    cap = max(1, (os.path.getsize(path) - 28) // 4) if os.path.exists(path) else 1
+    r = np.empty(cap, np.float32)
+    q = np.empty(cap, np.float32)
+    M, N, h = _I(), _I(), ctypes.c_uint64()
+    _check(lib().track_score_map_load(os.fsencode(path), r.ctypes.data, cap, q.ctypes.data, cap,
+                                      ctypes.byref(M), ctypes.byref(N), ctypes.byref(h)))
+    return r[:M.value * N.value].reshape(M.value, N.value).copy(), q[:N.value].copy(), h.value
 
 
 def track_policy_topk(score_map, K: int) -> np.ndarray:

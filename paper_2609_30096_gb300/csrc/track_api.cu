@@ -1069,6 +1069,91 @@ int track_mean_score(const float* r, int M, int N, float* q_out) {
   return TRACK_OK;
 }
 
+static const char kScoreMagic[8] = {'T', 'R', 'K', 'S', 'C', 'O', 'R', 'E'};
+
+// Little-endian encoding independent of the host's byte order.
+static void put_u32(std::vector<uint8_t>& b, uint32_t v) {
+  for (int i = 0; i < 4; ++i) b.push_back((uint8_t)(v >> (8 * i)));
+}
+static void put_u64(std::vector<uint8_t>& b, uint64_t v) {
+  for (int i = 0; i < 8; ++i) b.push_back((uint8_t)(v >> (8 * i)));
+}
+static void put_f32(std::vector<uint8_t>& b, float f) {
+  uint32_t u;
+  memcpy(&u, &f, 4);
+  put_u32(b, u);
+}
+static uint32_t get_u32(const uint8_t* p) {
+  uint32_t v = 0;
+  for (int i = 0; i < 4; ++i) v |= (uint32_t)p[i] << (8 * i);
+  return v;
+}
+static uint64_t get_u64(const uint8_t* p) {
+  uint64_t v = 0;
+  for (int i = 0; i < 8; ++i) v |= (uint64_t)p[i] << (8 * i);
+  return v;
+}
+static float get_f32(const uint8_t* p) {
+  const uint32_t u = get_u32(p);
+  float f;
+  memcpy(&f, &u, 4);
+  return f;
+}
+
+int track_score_map_save(const char* path, const float* r, int M, int N, uint64_t config_hash) {
+  if (!path || !r || M < 1 || N < 1) return fail(TRACK_EINVAL, "bad arguments");
+  const size_t n = (size_t)M * N;
+  for (size_t i = 0; i < n; ++i)
+    if (!(r[i] >= 0.f)) return fail(TRACK_EINVAL, "scores must be non-negative numbers");
+  std::vector<float> q((size_t)N);
+  TRACK_TRY(track_mean_score(r, M, N, q.data()));
+  std::vector<uint8_t> b;
+  b.reserve(28 + 4 * (n + N));
+  b.insert(b.end(), kScoreMagic, kScoreMagic + 8);
+  put_u32(b, 1);
+  put_u32(b, (uint32_t)M);
+  put_u32(b, (uint32_t)N);
+  put_u64(b, config_hash);
+  for (size_t i = 0; i < n; ++i) put_f32(b, r[i]);
+  for (int k = 0; k < N; ++k) put_f32(b, q[(size_t)k]);
+  FILE* f = fopen(path, "wb");
+  if (!f) return fail(TRACK_EINVAL, std::string("cannot open for writing: ") + path);
+  const size_t w = fwrite(b.data(), 1, b.size(), f);
+  const int closed = fclose(f);
+  if (w != b.size() || closed != 0) return fail(TRACK_EINVAL, std::string("write failed: ") + path);
+  return TRACK_OK;
+}
+
+int track_score_map_load(const char* path, float* r, int64_t r_cap, float* q, int64_t q_cap,
+                         int* M, int* N, uint64_t* config_hash) {
+  if (!path || !r || !M || !N || !config_hash || r_cap < 1 || (q && q_cap < 1))
+    return fail(TRACK_EINVAL, "bad arguments");
+  FILE* f = fopen(path, "rb");
+  if (!f) return fail(TRACK_EINVAL, std::string("cannot open: ") + path);
+  std::vector<uint8_t> b;
+  uint8_t buf[65536];
+  size_t got;
+  while ((got = fread(buf, 1, sizeof(buf), f)) > 0) b.insert(b.end(), buf, buf + got);
+  fclose(f);
+  if (b.size() < 28 || memcmp(b.data(), kScoreMagic, 8) != 0)
+    return fail(TRACK_EINVAL, "not a score-map file");
+  if (get_u32(b.data() + 8) != 1) return fail(TRACK_EINVAL, "unknown score-map version");
+  const uint32_t m = get_u32(b.data() + 12), n = get_u32(b.data() + 16);
+  if (m < 1 || n < 1 || m > (1u << 30) || n > (1u << 30)) return fail(TRACK_EINVAL, "bad dimensions");
+  const uint64_t need = 28 + 4 * ((uint64_t)m * n + n);
+  if ((uint64_t)b.size() != need) return fail(TRACK_EINVAL, "truncated or oversized score-map file");
+  if ((int64_t)m * n > r_cap || (q && (int64_t)n > q_cap))
+    return fail(TRACK_EINVAL, "score map larger than the given capacity");
+  const uint8_t* p = b.data() + 28;
+  for (uint64_t i = 0; i < (uint64_t)m * n; ++i) r[i] = get_f32(p + 4 * i);
+  if (q)
+    for (uint32_t k = 0; k < n; ++k) q[k] = get_f32(p + 4 * ((uint64_t)m * n + k));
+  *M = (int)m;
+  *N = (int)n;
+  *config_hash = get_u64(b.data() + 20);
+  return TRACK_OK;
+}
+
 int track_policy_topk(const float* score_map, int N, int K, uint8_t* policy_out) {
   if (!score_map || !policy_out || N < 1) return fail(TRACK_EINVAL, "bad arguments");
   if (K < 0 || K > N) return fail(TRACK_EINVAL, "K must satisfy 0 <= K <= N");

@@ -143,3 +143,54 @@ def test_attention_schedule_modes(T):
         with pytest.raises(T.TrackError) as e:
             T.track_attention_schedule(bad)
         assert e.value.code == T.TRACK_EINVAL
+
+
+# ---------------------------------------------------------------- score-map file
+def test_score_map_round_trip_and_resume(T, tmp_path):
+    # The calibration map survives a round trip bit for bit, the stored mean is
+    # Eq. 5 of the oracle, and calibrating in two halves (rows are independent
+    # samples) then appending gives the same file, mean and policy as all at once.
+    rng = np.random.default_rng(3)
+    M, N, K = 8, 50, 25
+    r = rng.uniform(0.0, 2.0, (M, N)).astype(np.float32)
+    whole = tmp_path / "whole.trk"
+    T.track_score_map_save(whole, r, config_hash=0xABCDEF0123456789)
+    r2, q2, h = T.track_score_map_load(whole)
+    assert h == 0xABCDEF0123456789
+    assert np.array_equal(r2, r)
+    assert np.array_equal(q2, otrack.mean_score(r.astype(np.float64)).astype(np.float32))
+    assert np.array_equal(q2, T.track_mean_score(r))
+    half = tmp_path / "half.trk"
+    T.track_score_map_save(half, r[:3], config_hash=7)
+    r_a, _, h_a = T.track_score_map_load(half)
+    resumed = tmp_path / "resumed.trk"
+    T.track_score_map_save(resumed, np.concatenate([r_a, r[3:]]), config_hash=h_a)
+    r3, q3, _ = T.track_score_map_load(resumed)
+    assert np.array_equal(r3, r) and np.array_equal(q3, q2)
+    assert np.array_equal(T.track_policy_topk(q3, K), otrack.topk_policy(q2, K))
+
+
+def test_score_map_rejects_bad_files_and_scores(T, tmp_path):
+    r = np.ones((2, 4), np.float32)
+    good = tmp_path / "good.trk"
+    T.track_score_map_save(good, r)
+    raw = good.read_bytes()
+    assert raw[:8] == b"TRKSCORE" and len(raw) == 28 + 4 * (8 + 4)
+    cases = {"truncated": raw[:-3], "magic": b"X" + raw[1:], "version": raw[:8] + b"\x02" + raw[9:],
+             "empty": b""}
+    for name, data in cases.items():
+        p = tmp_path / f"{name}.trk"
+        p.write_bytes(data)
+        with pytest.raises(T.TrackError) as e:
+            T.track_score_map_load(p)
+        assert e.value.code == T.TRACK_EINVAL, name
+    with pytest.raises(T.TrackError):
+        T.track_score_map_load(tmp_path / "missing.trk")
+    for bad in (np.float32(-1.0), np.float32(np.nan)):
+        rb = r.copy()
+        rb[1, 2] = bad
+        with pytest.raises(T.TrackError) as e:
+            T.track_score_map_save(tmp_path / "bad.trk", rb)
+        assert e.value.code == T.TRACK_EINVAL
+    with pytest.raises(T.TrackError):
+        T.track_score_map_save(tmp_path / "no_such_dir" / "x.trk", r)
