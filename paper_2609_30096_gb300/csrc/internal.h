@@ -169,6 +169,9 @@ cudaError_t qk_norm_rope(const NormRopeArgs& a, cudaStream_t s);
 cudaError_t head_unpatchify(const float* xres, int nseq, int L, int d, const float* head_mod,
                             const void* Whead, int dtype, const float* bhead, float eps, int C,
                             int F, int H, int W, float* out, cudaStream_t s);
+// Token-major [nseq * L, 4C] -> [nseq, C, F, H, W] (exact inverse of patchify).
+cudaError_t unpatchify(const float* tokv, int nseq, int L, int C, int F, int H, int W, float* out,
+                       cudaStream_t s);
 // Eq. 1 and Eq. 2 on n floats.
 cudaError_t cfg_combine(const float* fc, const float* fu, int64_t n, float w, float* p,
                         cudaStream_t s);

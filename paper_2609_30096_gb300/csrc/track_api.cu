@@ -661,8 +661,20 @@ static int forward(track_model* m, const float* x, int B, int nseq, float t, con
     TRACK_TRY(run_gemm(m, w.h, Ly.W1, M, F, d, Ly.b1, EPI_GELU, nullptr, w.ffh, F, s));
     TRACK_TRY(run_gemm(m, w.ffh, Ly.W2, M, d, F, Ly.b2, EPI_RESID_GATE, gate2, w.xres, d, s));
   }
-  LAUNCH(head_unpatchify(w.xres, nseq, L, d, w.head_mod, m->head_W, m->dtype, m->head_b, a.eps,
-                         a.in_ch, a.frames, a.height, a.width, out, s));
+  // Head: LN(x)(1 + scale) + shift (a11), then its Linear(d -> 4C) as a GEMM into
+  // token-major fp32 (the FFN hidden buffer is free after the last block), then
+  // unpatchify.
+  const int P = 4 * a.in_ch;
+  if ((m->dtype == F32 || P % 32 == 0) && (size_t)F * es >= (size_t)P * sizeof(float)) {
+    LAUNCH(run_ln(m, w.xres, M, d, w.head_mod + d, w.head_mod, 0, w.h, s));
+    float* hv = (float*)w.ffh;
+    TRACK_CUDA(cudaMemsetAsync(hv, 0, (size_t)M * P * sizeof(float), s));
+    TRACK_TRY(run_gemm(m, w.h, m->head_W, M, P, d, m->head_b, EPI_RESID, nullptr, hv, P, s));
+    LAUNCH(unpatchify(hv, nseq, L, a.in_ch, a.frames, a.height, a.width, out, s));
+  } else {
+    LAUNCH(head_unpatchify(w.xres, nseq, L, d, w.head_mod, m->head_W, m->dtype, m->head_b, a.eps,
+                           a.in_ch, a.frames, a.height, a.width, out, s));
+  }
   return TRACK_OK;
 }
 
