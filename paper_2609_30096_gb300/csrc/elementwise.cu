@@ -462,6 +462,30 @@ __device__ __forceinline__ void rope8(float (&v)[8], int eh, const NormRopeArgs&
   }
 }
 
+// The (cos, sin) pairs rope8 uses for the 4 pairs of a chunk at head offset eh.
+__device__ __forceinline__ void rope_coeffs(float2 (&cs)[4], int eh, const NormRopeArgs& a, int pf,
+                                            int ph, int pw) {
+  const int s6 = a.hd / 6;
+  const int nf = (a.hd - 4 * s6) / 2, nh = s6;
+#pragma unroll
+  for (int p = 0; p < 4; ++p) {
+    const int j = eh / 2 + p;
+    int idx;
+    if (j < nf) idx = pf * nf + j;
+    else if (j < nf + nh) idx = a.Fp * nf + ph * nh + (j - nf);
+    else idx = a.Fp * nf + a.Hp * nh + pw * nh + (j - nf - nh);
+    cs[p] = a.rope_tab[idx];
+  }
+}
+__device__ __forceinline__ void rope_apply8(float (&v)[8], const float2 (&cs)[4]) {
+#pragma unroll
+  for (int p = 0; p < 4; ++p) {
+    const float x0 = v[2 * p], x1 = v[2 * p + 1];
+    v[2 * p] = x0 * cs[p].x - x1 * cs[p].y;
+    v[2 * p + 1] = x0 * cs[p].y + x1 * cs[p].x;
+  }
+}
+
 __device__ __forceinline__ void scale8(float (&v)[8], float rstd, const float* g) {
   const float4 g0 = reinterpret_cast<const float4*>(g)[0];
   const float4 g1 = reinterpret_cast<const float4*>(g)[1];
@@ -529,11 +553,17 @@ __global__ void __launch_bounds__(256) k_norm_rope_r(NormRopeArgs a) {
   const float ss = ((s8[0] + s8[1]) + (s8[2] + s8[3])) + ((s8[4] + s8[5]) + (s8[6] + s8[7]));
   const float rstd = 1.f / sqrtf(warp_sum(ss) / (float)D + a.eps);
   const int pf = l / (a.Hp * a.Wp), ph = (l / a.Wp) % a.Hp, pw = l % a.Wp;
+  // A lane's chunks lie 256 elements apart, a whole number of heads (hd 64 or
+  // 128), so they share one head offset and one set of rotation coefficients.
+  float2 cs[4];
+  const bool shared_cs = a.rope && 256 % a.hd == 0;
+  if (shared_cs) rope_coeffs(cs, (8 * lane) % a.hd, a, pf, ph, pw);
 #pragma unroll
   for (int c = 0; c < CPL; ++c) {
     const int e0 = 8 * (lane + 32 * c);
     scale8(v[c], rstd, g + e0);
-    if (a.rope) rope8(v[c], e0 % a.hd, a, pf, ph, pw);
+    if (shared_cs) rope_apply8(v[c], cs);
+    else if (a.rope) rope8(v[c], e0 % a.hd, a, pf, ph, pw);
     store8(p + e0, v[c]);
   }
 }
