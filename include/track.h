@@ -388,8 +388,10 @@ int track_gemm_raster(int group);
  * span more than 4 CTAs.  A split item is finished by the last of its CTAs,
  * which combines the parts' row maxima, row sums and unnormalized outputs in
  * key order.  TRACK_GEMM_AUTO (the default) picks per launch by a makespan
- * model.  Each schedule is deterministic; they differ in fp32 rounding only.
- * EINVAL for any other mode. */
+ * model.  Without TRACK_ATTN_ONE_TILE the one-tile kernel is still taken for
+ * key ranges of at most 4 tiles (512 keys) when the pair kernel would have at
+ * most two items per SM.  Each schedule is deterministic; they differ in fp32
+ * rounding only.  EINVAL for any other mode. */
 #define TRACK_ATTN_ONE_TILE 4
 int track_attention_schedule(int mode);
 

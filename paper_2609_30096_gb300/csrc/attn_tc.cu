@@ -1213,7 +1213,15 @@ cudaError_t attention_bf16(const AttnOperand& Q, const AttnOperand& K, const Att
   if (Lk <= 0) return cudaErrorInvalidValue;
   if ((((uintptr_t)Q.ptr) | ((uintptr_t)K.ptr) | ((uintptr_t)V.ptr) | ((uintptr_t)O)) & 15)
     return cudaErrorMisalignedAddress;
-  const bool one_tile = (g_attn_schedule.load() & 4) != 0;
+  // The one-tile kernel double-buffers Q, so it pays less per work item; it is
+  // taken by default for short key ranges (cross-attention to 512 text tokens)
+  // when the pair kernel would have at most two items per SM: there a work item
+  // is a few key tiles and the pair kernel's exposed Q load dominates (measured
+  // at one 3510-token sequence: 26 against 28 us).
+  const int QT = (Lq + AT_BM - 1) / AT_BM, KT = (Lk + AT_BN - 1) / AT_BN;
+  const int64_t pair_items = (int64_t)S * H * ((QT + 1) / 2);
+  const bool one_tile = (g_attn_schedule.load() & 4) != 0 ||
+                        (KT <= 4 && pair_items <= 2 * (int64_t)num_sms());
   if (hd == 128)
     return one_tile ? launch_attn_tc<128>(Q, K, V, O, S, H, Lq, Lk, s)
                     : launch_attn_pp<128>(Q, K, V, O, S, H, Lq, Lk, s);
