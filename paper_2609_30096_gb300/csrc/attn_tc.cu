@@ -1,6 +1,11 @@
 // Flash attention on the sm_103a tensor cores (bf16 in, fp32 accumulate):
 // O = softmax(Q K^T / sqrt(hd)) V per (sequence, head), no mask.
 //
+// Two kernels share the schedules below: k_attn_tc, whose work item is one
+// 128-query tile (described first), and k_attn_pp, whose item is a pair of
+// query tiles sharing every K/V tile (described before it, further down; the
+// default).
+//
 // Work: an item is one 128-query tile of one (sequence, head); its KT key tiles
 // of 128 keys are its units.  The kernel is persistent (at most one CTA per SM)
 // and follows one of two schedules:

@@ -177,8 +177,8 @@ __global__ void __launch_bounds__(192, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   // The prologue above overlaps the previous kernel; inputs and outputs are touched only
-  // after the grid dependency wait.  The producer thread first requests the W tiles of
-  // its first stages: weights are never written by an earlier kernel.
+  // after the grid dependency wait.  For model weights (g.w_static) the producer thread
+  // first requests the W tiles of its first stages: no kernel writes them.
   const bool producer = warp == 0 && lane == 0;
   if (!producer) {
     pdl_wait();
@@ -196,7 +196,7 @@ __global__ void __launch_bounds__(192, 1)
       for (int i = 0; i < STAGES; ++i) armed[i] = 0;
       SegIter it(use_sk, sk.units, num_tiles, nk, worker, workers);
       int pre = 0;  // k-blocks of the first segment whose W tile is already requested
-      if (CL == 1) {
+      if (CL == 1 && g.w_static) {
         SegIter first = it;
         int t0, a0, a1;
         if (first.next(t0, a0, a1)) {

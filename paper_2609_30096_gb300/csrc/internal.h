@@ -78,6 +78,8 @@ struct GemmArgs {
   int ldo;
   int* err;            // device error word
   int raster;          // bf16 tensor-core GEMM: row units per raster group (set by its launcher)
+  int w_static = 0;    // W is never written by a kernel (model weights): it may be
+                       // requested before the grid dependency wait
 };
 
 // fp32 FFMA GEMM: out = A[M,K] . W[N,K]^T (+ epilogue), all fp32.

@@ -515,6 +515,7 @@ static int run_gemm(const track_model* m, const void* A, const void* W, int M, i
                     cudaStream_t s) {
   GemmArgs g;
   g.M = M; g.N = N; g.K = K; g.epi = epi; g.bias = bias; g.gate = gate; g.out = out; g.ldo = ldo;
+  g.w_static = 1;  // W is a weight of the model
   g.err = device_error_word();
   if (g.err == nullptr) return fail(TRACK_ECUDA, "device error word allocation failed");
   ProfScope ps(0, 2.0 * M * N * (double)K, s);
