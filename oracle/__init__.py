@@ -9,10 +9,13 @@ seeded input generator ``synth``, which holds no arithmetic of the method.
 Contents (each function cites the passage of the paper it restates):
 
 * ``oracle.track`` - the method proper: guidance (Eq. 1), the scheduler update
-  (Eq. 2, flow-matching Euler instance), routed sampling (Eq. 3), the relative
-  disagreement (Eq. 4), the mean score (Eq. 5), the box-constrained relaxation
-  and its threshold solution (Eq. 6-7), top-K switching (Sec. 3.2.3) and
-  reference-trajectory calibration (Sec. 3.2.1).
+  (Eq. 2: the flow-matching Euler instance, and a second-order multistep
+  instance whose history h_i carries across model switches), routed sampling
+  (Eq. 3), the relative disagreement (Eq. 4) and its frequency-band split
+  (Sec. 4.4), the mean score (Eq. 5), the box-constrained relaxation and its
+  threshold solution (Eq. 6-7), top-K switching (Sec. 3.2.3), the equal-budget
+  First-K / Last-K / Random-K policies (Sec. 4.5) and reference-trajectory
+  calibration (Sec. 3.2.1).
 * ``oracle.dit`` - the denoiser f_m that Eq. 1 treats as a black box: the
   Wan-style video DiT (patchify, adaLN-modulated self-attention with 3D RoPE,
   cross-attention, GELU MLP, unpatchify).  The paper does not define these
@@ -20,6 +23,8 @@ Contents (each function cites the passage of the paper it restates):
   conditioning interface and prediction target); the definitions written here
   are this library's reading, pinned by component tests (closed forms,
   invariants, brute force) and by structural tests of the composed block.
+  ``DiT.forward_at_tokens`` evaluates the last block and the head at chosen
+  tokens only, for checks at sizes where the whole forward is too slow.
 
 Precision: everything is computed in fp64 from fp32 inputs.  ``precision="bf16"``
 rounds the weight matrices and the text conditioning to bf16 (round to nearest
