@@ -218,6 +218,29 @@ __global__ void __launch_bounds__(256) k_patch_embed(const float* __restrict__ x
 // order as k_patch_embed: the sum over k from 0, then the bias.
 constexpr int PT = 32;
 
+// A 64-element weight row in 16-byte loads (the row starts 128- or 256-byte aligned).
+__device__ __forceinline__ void load_row64(const float* src, float (&w)[64]) {
+  const float4* s4 = reinterpret_cast<const float4*>(src);
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const float4 v = s4[i];
+    w[4 * i] = v.x; w[4 * i + 1] = v.y; w[4 * i + 2] = v.z; w[4 * i + 3] = v.w;
+  }
+}
+__device__ __forceinline__ void load_row64(const bf16* src, float (&w)[64]) {
+  const uint4* s4 = reinterpret_cast<const uint4*>(src);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const uint4 u = s4[i];
+    const uint32_t q[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      w[8 * i + 2 * j] = __uint_as_float(q[j] << 16);
+      w[8 * i + 2 * j + 1] = __uint_as_float(q[j] & 0xFFFF0000u);
+    }
+  }
+}
+
 template <typename T>
 __global__ void __launch_bounds__(256) k_patch_embed64(const float* __restrict__ x, int B, int rows,
                                                        int F, int H, int W,
@@ -227,7 +250,7 @@ __global__ void __launch_bounds__(256) k_patch_embed64(const float* __restrict__
   pdl_wait();
   pdl_release();
   constexpr int C = 16, P = 64;
-  __shared__ float patch[PT][P];
+  __shared__ __align__(16) float patch[PT][P];
   const int Hp = H / 2, Wp = W / 2, L = F * Hp * Wp;
   const int r0 = blockIdx.x * PT;
   for (int i = threadIdx.x; i < PT * P; i += blockDim.x) {
@@ -245,8 +268,7 @@ __global__ void __launch_bounds__(256) k_patch_embed64(const float* __restrict__
   float w[P];
   float bb = 0.f;
   if (n < d) {
-#pragma unroll
-    for (int k = 0; k < P; ++k) w[k] = ldv(Wpe, (int64_t)n * P + k);
+    load_row64(Wpe + (int64_t)n * P, w);
     bb = bpe[n];
   }
   __syncthreads();
@@ -254,9 +276,16 @@ __global__ void __launch_bounds__(256) k_patch_embed64(const float* __restrict__
   const int nt = rows - r0 < PT ? rows - r0 : PT;
 #pragma unroll 1
   for (int t = 0; t < nt; ++t) {
+    const float4* pt = reinterpret_cast<const float4*>(patch[t]);
     float acc = 0.f;
 #pragma unroll
-    for (int k = 0; k < P; ++k) acc = fmaf(w[k], patch[t][k], acc);
+    for (int k4 = 0; k4 < P / 4; ++k4) {
+      const float4 q = pt[k4];  // one shared-memory broadcast for four FMAs
+      acc = fmaf(w[4 * k4], q.x, acc);
+      acc = fmaf(w[4 * k4 + 1], q.y, acc);
+      acc = fmaf(w[4 * k4 + 2], q.z, acc);
+      acc = fmaf(w[4 * k4 + 3], q.w, acc);
+    }
     xres[(int64_t)(r0 + t) * d + n] = acc + bb;
   }
 }
