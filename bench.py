@@ -517,7 +517,10 @@ def run_ours(args):
     roof = {"bound": "tensor", "kernel": "bf16 GEMM (tcgen05)" if dominant == "gemm"
             else "flash attention (tcgen05)",
             "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-            "frac": achieved / peak if achieved else None, "traffic": traffic,
+            "frac": achieved / peak if achieved else None,
+            "frac_of_sustained": (achieved / peaks["bf16_tflops_sustained"]
+                                  if achieved and peaks.get("bf16_tflops_sustained") else None),
+            "traffic": traffic,
             "traffic_unit": "bytes per launch", "traffic_source": traffic_src,
             "peak_source": f"{src} bf16 burst (sustained {peaks.get('bf16_tflops_sustained')})",
             "launches": int(dn), "avg_launch_ms": dm / dn if dn else None,
