@@ -314,8 +314,8 @@ __global__ void __launch_bounds__(192, 1)
     int tile, kb0, kb1;
     while (it.next(tile, kb0, kb1)) {
       int mu, nt;
-        tile_coords(tile, m_units, n_tiles, g.raster, mu, nt);
-        const int mt = mu * CL + rank;
+      tile_coords(tile, m_units, n_tiles, g.raster, mu, nt);
+      const int mt = mu * CL + rank;
       const bool final_seg = it.done();
       // Bias and gate of this tile's columns are pulled into L1 while the MMAs run
       // (lane l: columns 8l..8l+7); the column loop below reads them with
