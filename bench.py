@@ -385,39 +385,32 @@ def run_ours(args):
         # Replays a copy of the trajectory's graph recorded with timing on (an event-
         # record node before and after each bracketed kernel), reading the brackets after
         # every replay.  Falls back to kernel-by-kernel launches if that fails.
-        keys = ("gemm", "attention", "norm")
-        tot = {k: [0.0, 0.0, 0] for k in keys}
-        ms_tot = 0.0
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+        def bracketed(fn):
+            tot = {k: [0.0, 0.0, 0] for k in ("gemm", "attention", "norm")}
+            ms_tot = 0.0
+            torch.cuda.synchronize()
+            T.track_profile_read()                    # drop the priming calls' records
+            for _ in range(steps):
+                a.record(stream)
+                fn(pol)
+                b.record(stream)
+                torch.cuda.synchronize()
+                ms_tot += a.elapsed_time(b)
+                for k, v in T.track_profile_read().items():
+                    tot[k] = [x + y for x, y in zip(tot[k], v)]
+            return ms_tot, tot
+
         T.track_profile_enable(True)
         try:
             try:
-                mode = "graph"
                 prime(pol)                            # eager run, then the bracketed recording
-                torch.cuda.synchronize()
-                T.track_profile_read()
-                for _ in range(steps):
-                    a.record(stream)
-                    step_device(pol)
-                    b.record(stream)
-                    torch.cuda.synchronize()
-                    ms_tot += a.elapsed_time(b)
-                    for k, v in T.track_profile_read().items():
-                        tot[k] = [tot[k][0] + v[0], tot[k][1] + v[1], tot[k][2] + v[2]]
+                mode = "graph"
+                ms_tot, tot = bracketed(step_device)
             except T.TrackError:
                 mode = "eager"
-                tot = {k: [0.0, 0.0, 0] for k in keys}
-                ms_tot = 0.0
-                torch.cuda.synchronize()
-                T.track_profile_read()
-                for _ in range(steps):
-                    a.record(stream)
-                    step_eager(pol)
-                    b.record(stream)
-                    torch.cuda.synchronize()
-                    ms_tot += a.elapsed_time(b)
-                    for k, v in T.track_profile_read().items():
-                        tot[k] = [tot[k][0] + v[0], tot[k][1] + v[1], tot[k][2] + v[2]]
+                ms_tot, tot = bracketed(step_eager)
         finally:
             T.track_profile_enable(False)
         return max_over_ranks(ms_tot, world, dev), {k: tuple(v) for k, v in tot.items()}, mode
