@@ -40,6 +40,11 @@ def test_every_declared_symbol_is_exported(T):
     assert T.track_abi_version() == 1
 
 
+def test_every_declared_symbol_has_a_binding_of_the_same_name(T):
+    missing = [n for n in declared_functions() if not callable(getattr(T, n, None))]
+    assert not missing, missing
+
+
 @pytest.mark.parametrize("n,shift", [(1, 5.0), (4, 5.0), (8, 5.0), (50, 5.0), (30, 3.0), (7, 1.0)])
 def test_schedule_matches_oracle_bitwise(T, n, shift):
     assert np.array_equal(T.track_schedule(n, shift), otrack.schedule(n, shift))
