@@ -353,21 +353,16 @@ int track_linear(int dtype, const void* X, const void* W, const float* bias, int
  * split across CTAs is summed by the last of them in k order).
  * TRACK_GEMM_DATA_PARALLEL always uses whole tiles; TRACK_GEMM_STREAM_K uses
  * stream-K wherever the shape allows it (every CTA gets at least one k-block
- * and no tile spans more than 4 CTAs), else decides as AUTO.  OR-ing in
- * TRACK_GEMM_MULTICAST runs the CTAs in clusters of two that compute vertically
- * adjacent row tiles and share each W tile through TMA multicast (half the W
- * bytes per SM), when the GEMM has more than 128 rows.  Every schedule is
- * deterministic (same inputs, same launch: same bits); two schedules differ in
- * fp32 rounding only (data-parallel gives the same bits with or without
- * multicast).  EINVAL for any other mode. */
+ * and no tile spans more than 4 CTAs), else decides as AUTO.  Every schedule
+ * is deterministic (same inputs, same launch: same bits); two schedules differ
+ * in fp32 rounding only.  EINVAL for any other mode. */
 #define TRACK_GEMM_AUTO 0
 #define TRACK_GEMM_DATA_PARALLEL 1
 #define TRACK_GEMM_STREAM_K 2
-#define TRACK_GEMM_MULTICAST 4
 int track_gemm_schedule(int mode);
 
 /* Tile order of the TRACK_BF16 GEMM (process-wide): output tiles are taken in
- * groups of `group` 128-row units (256 with TRACK_GEMM_MULTICAST), the row unit
+ * groups of `group` 128-row units, the row unit
  * varying fastest inside a group, then the 128-to-256-column tile.  The tiles
  * running at one time then share few A and W blocks, which stay in L2 while
  * they are reused.  A group at least as large as the row-unit count is plain
@@ -378,7 +373,7 @@ int track_gemm_schedule(int mode);
 int track_gemm_raster(int group);
 
 /* Schedule of the TRACK_BF16 attention kernel (process-wide), with the mode
- * values of track_gemm_schedule (no multicast), optionally or-ed with
+ * values of track_gemm_schedule, optionally or-ed with
  * TRACK_ATTN_ONE_TILE.  The kernel is persistent, at most one CTA per SM, and
  * its work item is a pair of 128-query tiles of one (sequence, head) sharing
  * every K and V tile it loads; with TRACK_ATTN_ONE_TILE it is the earlier

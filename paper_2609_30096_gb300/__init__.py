@@ -22,7 +22,6 @@ TRACK_WAIT_SELFTEST_CODE = 99  # error-word code of track_wait_selftest
 FP32, BF16 = 0, 1
 EPI_STORE, EPI_GELU, EPI_RESID_GATE, EPI_RESID = range(4)
 GEMM_AUTO, GEMM_DATA_PARALLEL, GEMM_STREAM_K = range(3)
-GEMM_MULTICAST = 4  # OR-ed into a schedule: two-CTA clusters sharing W tiles
 ATTN_ONE_TILE = 4   # OR-ed into an attention schedule: one query tile per work item
 
 
@@ -157,8 +156,7 @@ def track_launch_count() -> int:
 
 
 def track_gemm_schedule(mode: int):
-    """GEMM_AUTO, GEMM_DATA_PARALLEL or GEMM_STREAM_K (optionally | GEMM_MULTICAST)
-    for every later bf16 GEMM."""
+    """GEMM_AUTO, GEMM_DATA_PARALLEL or GEMM_STREAM_K for every later bf16 GEMM."""
     _check(lib().track_gemm_schedule(int(mode)))
 
 

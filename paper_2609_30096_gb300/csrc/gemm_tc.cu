@@ -1,22 +1,17 @@
 // bf16 GEMM on the sm_103a tensor cores: out = A[M,K] . W[N,K]^T (+ epilogue).
 //
-// Persistent, warp-specialised kernel, one CTA per SM.  When there are at
-// least two row tiles the CTAs run in clusters of two: the pair computes a
-// 256-row work tile (one 128-row tile each) and shares the W tile through TMA
-// multicast, each CTA fetching half of it for both, which cuts the operand
-// bytes an SM pulls from L2 per k-block by a third at BN = 256.  A worker (a
-// CTA, or a cluster) follows one of two schedules:
-//   data-parallel  worker w takes work tiles w, w + workers, ... (whole K loop);
-//   stream-K       the work tiles' k-blocks form one sequence of U units and
-//                  worker w takes the contiguous share [w U / G, (w+1) U / G),
-//                  so every worker does the same number of k-blocks whatever
-//                  the tile count.  A tile split across workers is finished by
-//                  whichever ends its part last: the others write their fp32
-//                  partial sums to a workspace slot and count in on a
-//                  per-(tile, warp) counter; the last one adds the parts in k
-//                  order (a fixed order, so the result does not depend on
-//                  timing), applies the epilogue and resets the counter for
-//                  the next launch.
+// Persistent, warp-specialised kernel, one CTA per SM.  A CTA follows one of
+// two schedules:
+//   data-parallel  CTA w takes output tiles w, w + G, ... (whole K loop);
+//   stream-K       the tiles' k-blocks form one sequence of U units and CTA w
+//                  takes the contiguous share [w U / G, (w+1) U / G), so every
+//                  CTA does the same number of k-blocks whatever the tile
+//                  count.  A tile split across CTAs is finished by whichever
+//                  ends its part last: the others write their fp32 partial
+//                  sums to a workspace slot and count in on a per-(tile, warp)
+//                  counter; the last one adds the parts in k order (a fixed
+//                  order, so the result does not depend on timing), applies
+//                  the epilogue and resets the counter for the next launch.
 //   warp 0      TMA producer: 128x64 A tile and BNx64 W tile per stage into a
 //               STAGES-deep shared-memory ring (128-byte swizzle, zero fill past
 //               the matrix edges), completion counted on an mbarrier.
@@ -122,14 +117,7 @@ struct TcShape {
   static constexpr size_t SMEM = 1024 + (size_t)STAGES * (A_BYTES + B_BYTES) + STG_BYTES + 256;
 };
 
-// CL = CTAs per cluster (1 or 2).  With CL = 2 the two CTAs of a cluster take
-// vertically adjacent 128-row tiles of the same BN columns (a "work tile" of
-// 256 rows): each loads its own A tile and one half of the shared W tile, which
-// TMA multicasts into both CTAs, so each SM pulls 128x64 + (BN/2)x64 elements
-// per k-block instead of 128x64 + BNx64.  A stage is refilled only after the
-// MMAs of both CTAs have read it (its empty barrier counts one multicast
-// commit from each).
-template <int BN, int STAGES, int CL>
+template <int BN, int STAGES>
 __global__ void __launch_bounds__(192, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const __grid_constant__ CUtensorMap tmC, const GemmArgs g, const SkArgs sk) {
@@ -149,10 +137,9 @@ __global__ void __launch_bounds__(192, 1)
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int rank = CL == 1 ? 0 : (int)cluster_ctarank();
-  const int worker = blockIdx.x / CL, workers = gridDim.x / CL;
-  const int m_tiles = (g.M + BM - 1) / BM, n_tiles = (g.N + BN - 1) / BN;
-  const int m_units = (m_tiles + CL - 1) / CL;  // work tiles per column of tiles
+  const int worker = blockIdx.x, workers = gridDim.x;
+  const int n_tiles = (g.N + BN - 1) / BN;
+  const int m_units = (g.M + BM - 1) / BM;  // row tiles
   const int num_tiles = m_units * n_tiles;
   const int nk = g.K / BK;
   const bool use_sk = sk.cnt != nullptr;
@@ -160,7 +147,7 @@ __global__ void __launch_bounds__(192, 1)
   if (threadIdx.x == 0) {
     for (int i = 0; i < STAGES; ++i) {
       mbar_init(su32(&full[i]), 1);
-      mbar_init(su32(&empty[i]), CL);
+      mbar_init(su32(&empty[i]), 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(su32(&accf[i]), 1);
@@ -173,7 +160,6 @@ __global__ void __launch_bounds__(192, 1)
   if (warp == 1) tmem_alloc(su32(tmem_slot), S::TMEM_COLS);
   tc_fence_before();
   __syncthreads();
-  if (CL > 1) cluster_sync();  // the peer's barriers exist before any multicast reaches them
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   // The prologue above overlaps the previous kernel; inputs and outputs are touched only
@@ -196,7 +182,7 @@ __global__ void __launch_bounds__(192, 1)
       for (int i = 0; i < STAGES; ++i) armed[i] = 0;
       SegIter it(use_sk, sk.units, num_tiles, nk, worker, workers);
       int pre = 0;  // k-blocks of the first segment whose W tile is already requested
-      if (CL == 1 && g.w_static) {
+      if (g.w_static) {
         SegIter first = it;
         int t0, a0, a1;
         if (first.next(t0, a0, a1)) {
@@ -216,7 +202,7 @@ __global__ void __launch_bounds__(192, 1)
       while (it.next(tile, kb0, kb1)) {
         int mu, nt;
         tile_coords(tile, m_units, n_tiles, g.raster, mu, nt);
-        const int mt = mu * CL + rank;
+        const int mt = mu;
         bool ok = true;
         for (int kb = kb0; kb < kb1; ++kb) {
           const uint32_t fb = su32(&full[stage]);
@@ -236,13 +222,7 @@ __global__ void __launch_bounds__(192, 1)
           }
           mbar_expect_tx(fb, S::A_BYTES + S::B_BYTES);
           tma_load_2d(su32(sA + stage * S::A_BYTES), &tmA, kb * BK, mt * BM, fb);
-          if (CL == 1) {
-            tma_load_2d(su32(sB + stage * S::B_BYTES), &tmB, kb * BK, nt * BN, fb);
-          } else {
-            constexpr int HB = BN / CL;  // W rows this CTA fetches for the cluster
-            tma_load_2d_mc(su32(sB + stage * S::B_BYTES + rank * HB * 128), &tmB, kb * BK,
-                           nt * BN + rank * HB, fb, (uint16_t)((1u << CL) - 1));
-          }
+          tma_load_2d(su32(sB + stage * S::B_BYTES), &tmB, kb * BK, nt * BN, fb);
           ++armed[stage];
           if (++stage == STAGES) {
             stage = 0;
@@ -251,13 +231,11 @@ __global__ void __launch_bounds__(192, 1)
         }
         if (!ok) break;
       }
-      // Every copy into this CTA has landed, and (in a cluster) both CTAs' MMAs
-      // have released every stage, before the CTA may exit.
+      // Every copy into this CTA has landed before the CTA may exit.
 #pragma unroll
       for (int i = 0; i < STAGES; ++i) {
         if (armed[i] == 0) continue;
         mbar_drain(su32(&full[i]), (armed[i] - 1) & 1, g.err, 5);
-        if (CL > 1) mbar_drain(su32(&empty[i]), (armed[i] - 1) & 1, g.err, 8);
       }
     }
   } else if (warp == 1) {
@@ -284,8 +262,7 @@ __global__ void __launch_bounds__(192, 1)
           for (int k = 0; k < BK / 16; ++k)
             mma_bf16(d_tmem, sdesc_sw128(a0 + k * 32), sdesc_sw128(b0 + k * 32), idesc,
                      (kb > kb0 || k != 0) ? 1u : 0u);
-          if (CL == 1) mma_commit(su32(&empty[stage]));
-          else mma_commit_mc(su32(&empty[stage]), (uint16_t)((1u << CL) - 1));
+          mma_commit(su32(&empty[stage]));
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1;
@@ -315,7 +292,7 @@ __global__ void __launch_bounds__(192, 1)
     while (it.next(tile, kb0, kb1)) {
       int mu, nt;
       tile_coords(tile, m_units, n_tiles, g.raster, mu, nt);
-      const int mt = mu * CL + rank;
+      const int mt = mu;
       const bool final_seg = it.done();
       // Bias and gate of this tile's columns are pulled into L1 while the MMAs run
       // (lane l: columns 8l..8l+7); the column loop below reads them with
@@ -337,13 +314,13 @@ __global__ void __launch_bounds__(192, 1)
       // Stream-K parts of this work tile: workers w_first .. w_first + nparts - 1 in k order.
       int nparts = 1, part = 0, w_first = 0;
       bool finish = true, staged = false;
-      // Partial-sum slot of part i (this CTA's rank): 2w for worker w's first
+      // Partial-sum slot of part i: 2w for worker w's first
       // segment, 2w+1 for its last.
       auto slot_of = [&](int i) -> float4* {
         const int wi = w_first + i;
         const int first_tile = (int)(((int64_t)wi * U / workers) / nk);
         const int s = 2 * wi + (first_tile == tile ? 0 : 1);
-        return reinterpret_cast<float4*>(sk.ws + (size_t)(s * CL + rank) * SLOT);
+        return reinterpret_cast<float4*>(sk.ws + (size_t)s * SLOT);
       };
       const int rowq = quarter * 32 + lane;  // this thread's row within the tile
       if (kb0 != 0 || kb1 != nk) {
@@ -358,7 +335,7 @@ __global__ void __launch_bounds__(192, 1)
           }
           break;
         }
-        int* cnt = sk.cnt + 4 * (tile * CL + rank) + quarter;
+        int* cnt = sk.cnt + 4 * tile + quarter;
         int last = 0;
         if (lane == 0) last = ld_acquire(cnt) == nparts - 1 ? 1 : 0;
         last = __shfl_sync(0xffffffffu, last, 0);
@@ -574,8 +551,6 @@ __global__ void __launch_bounds__(192, 1)
     __syncwarp();
     tmem_dealloc(tmem_base, S::TMEM_COLS);
   }
-  // Neither CTA of a cluster exits while the other may still signal its barriers.
-  if (CL > 1) cluster_sync();
 }
 
 // 2-D tensor map of a row-major [rows, cols] matrix with leading dimension ld
@@ -593,44 +568,13 @@ bool make_tmap(CUtensorMap* tm, CUtensorMapDataType dt, size_t esize, const void
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Concurrently resident workers (CTAs, or clusters of CL CTAs) of one kernel
-// instantiation on the current device, looked up once.
-template <int BN, int STAGES, int CL>
-int max_workers() {
-  static std::mutex mu;
-  static std::map<int, int> cache;
-  int dev = 0;
-  cudaGetDevice(&dev);
-  std::lock_guard<std::mutex> lk(mu);
-  auto it = cache.find(dev);
-  if (it != cache.end()) return it->second;
-  int n = num_sms() / CL;
-  if (CL > 1 &&
-      cudaFuncSetAttribute(k_gemm_tc<BN, STAGES, CL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)TcShape<BN, STAGES>::SMEM) == cudaSuccess) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(num_sms());
-    cfg.blockDim = dim3(192);
-    cfg.dynamicSmemBytes = TcShape<BN, STAGES>::SMEM;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = CL;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    int c = 0;
-    if (cudaOccupancyMaxActiveClusters(&c, k_gemm_tc<BN, STAGES, CL>, &cfg) == cudaSuccess && c > 0)
-      n = c;
-    cudaGetLastError();
-  }
-  cache[dev] = n;
-  return n;
-}
+// CTAs of one kernel instantiation resident at once on the current device
+// (one per SM: the kernel's shared memory admits no second).
+int max_workers() { return num_sms(); }
 
 std::atomic<int> g_gemm_raster{0};  // 0: the default rule above
 
-template <int BN, int STAGES, int CL>
+template <int BN, int STAGES>
 cudaError_t launch_tc(const void* A, const void* W, const GemmArgs& g_in, bool stream_k,
                       cudaStream_t s) {
   using S = TcShape<BN, STAGES>;
@@ -642,36 +586,32 @@ cudaError_t launch_tc(const void* A, const void* W, const GemmArgs& g_in, bool s
   const CUtensorMapDataType BF = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
   if (!make_tmap(&ta, BF, 2, A, (uint64_t)g.M, (uint64_t)g.K, (uint64_t)g.K, BM, BK))
     return cudaErrorInvalidValue;
-  if (!make_tmap(&tb, BF, 2, W, (uint64_t)g.N, (uint64_t)g.K, (uint64_t)g.K, BN / CL, BK))
+  if (!make_tmap(&tb, BF, 2, W, (uint64_t)g.N, (uint64_t)g.K, (uint64_t)g.K, BN, BK))
     return cudaErrorInvalidValue;
   const bool bf16_out = g.epi == EPI_STORE || g.epi == EPI_GELU;
   if (bf16_out ? !make_tmap(&tc, BF, 2, g.out, (uint64_t)g.M, (uint64_t)g.N, (uint64_t)g.ldo, 32, 64)
                : !make_tmap(&tc, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, g.out, (uint64_t)g.M,
                             (uint64_t)g.N, (uint64_t)g.ldo, 32, 32))
     return cudaErrorInvalidValue;
-  cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN, STAGES, CL>,
+  cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN, STAGES>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)S::SMEM);
   if (e != cudaSuccess) return e;
-  const int m_units = ((g.M + BM - 1) / BM + CL - 1) / CL;
+  const int m_units = (g.M + BM - 1) / BM;
   const int tiles = m_units * ((g.N + BN - 1) / BN);
-  const int wmax = max_workers<BN, STAGES, CL>();
+  const int wmax = max_workers();
   int workers = tiles < wmax ? tiles : wmax;
   SkArgs sk = {nullptr, nullptr, 0};
   if (stream_k) {
     sk.units = (int64_t)tiles * (g.K / BK);
-    if (sk_scratch(s, (size_t)4 * tiles * CL, (size_t)2 * wmax * CL * BM * BN, &sk.cnt, &sk.ws))
+    if (sk_scratch(s, (size_t)4 * tiles, (size_t)2 * wmax * BM * BN, &sk.cnt, &sk.ws))
       workers = wmax;
     else
       sk = {nullptr, nullptr, 0};
   }
   count_launch();
-  if (CL == 1)
-    return launch_pdl(k_gemm_tc<BN, STAGES, CL>, workers, 192, S::SMEM, s, ta, tb, tc, g, sk);
-  return launch_pdl_cluster(k_gemm_tc<BN, STAGES, CL>, workers * CL, 192, S::SMEM, s, CL, ta, tb,
-                            tc, g, sk);
+  return launch_pdl(k_gemm_tc<BN, STAGES>, workers, 192, S::SMEM, s, ta, tb, tc, g, sk);
 }
 
-template <int CL>
 cudaError_t gemm_dispatch(const void* A, const void* W, const GemmArgs& g, int sched,
                           cudaStream_t s) {
   // Schedule and tile width by a makespan model: every worker of a wave runs
@@ -682,17 +622,14 @@ cudaError_t gemm_dispatch(const void* A, const void* W, const GemmArgs& g, int s
   // costs the average number of work tiles per worker (fractional) times the
   // same figure, plus SK_FIXUP; it is taken only when no tile spans more than
   // SK_MAX_PARTS workers.
-  const int m_units = ((g.M + BM - 1) / BM + CL - 1) / CL;
+  const int m_units = (g.M + BM - 1) / BM;
   const bool fp32_out = g.epi == EPI_RESID || g.epi == EPI_RESID_GATE;  // 32-column epilogue chunks
   const long nk = g.K / BK;
   int best_bn = 256;
   long best_cost = -1;
   for (int bn : {256, 192, 160, 128}) {
     if (bn == 160 && !fp32_out) continue;  // bf16 epilogue chunks are 64 columns wide
-    const int wk = bn == 256   ? max_workers<256, 4, CL>()
-                   : bn == 192 ? max_workers<192, 4, CL>()
-                   : bn == 160 ? max_workers<160, 5, CL>()
-                               : max_workers<128, 6, CL>();
+    const int wk = max_workers();
     const long tiles = (long)m_units * ((g.N + bn - 1) / bn);
     const long cost = ((tiles + wk - 1) / wk) * nk * (bn + 150);
     if (best_cost < 0 || cost < best_cost) {
@@ -701,19 +638,19 @@ cudaError_t gemm_dispatch(const void* A, const void* W, const GemmArgs& g, int s
     }
   }
   if (sched != 1) {
-    const int wk = max_workers<256, 4, CL>();
+    const int wk = max_workers();
     const long tiles = (long)m_units * ((g.N + 255) / 256);
     const long units = tiles * nk, per_worker = units / wk;
     const bool spans_ok =
         per_worker > 0 && 1 + (nk - 1 + per_worker - 1) / per_worker <= SK_MAX_PARTS;
     const double sk_cost = (double)tiles / wk * nk * (256 + 150) + SK_FIXUP;
     if (spans_ok && (sched == 2 || (tiles > wk / 2 && sk_cost < (double)best_cost)))
-      return launch_tc<256, 4, CL>(A, W, g, true, s);
+      return launch_tc<256, 4>(A, W, g, true, s);
   }
-  if (best_bn == 256) return launch_tc<256, 4, CL>(A, W, g, false, s);
-  if (best_bn == 192) return launch_tc<192, 4, CL>(A, W, g, false, s);
-  if (best_bn == 160) return launch_tc<160, 5, CL>(A, W, g, false, s);
-  return launch_tc<128, 6, CL>(A, W, g, false, s);
+  if (best_bn == 256) return launch_tc<256, 4>(A, W, g, false, s);
+  if (best_bn == 192) return launch_tc<192, 4>(A, W, g, false, s);
+  if (best_bn == 160) return launch_tc<160, 5>(A, W, g, false, s);
+  return launch_tc<128, 6>(A, W, g, false, s);
 }
 
 }  // namespace
@@ -813,10 +750,7 @@ cudaError_t gemm_bf16_tc(const void* A, const void* W, const GemmArgs& g, cudaSt
   if (g.bias != nullptr && (((uintptr_t)g.bias) & 15)) return cudaErrorMisalignedAddress;
   if (g.epi == EPI_RESID_GATE && (g.gate == nullptr || (((uintptr_t)g.gate) & 15)))
     return cudaErrorInvalidValue;
-  // Clusters of two CTAs (shared W tile) on request, when there are two row tiles to pair.
-  const int mode = g_schedule.load();
-  if ((mode & 4) != 0 && g.M > BM) return gemm_dispatch<2>(A, W, g, mode & 3, s);
-  return gemm_dispatch<1>(A, W, g, mode & 3, s);
+  return gemm_dispatch(A, W, g, g_schedule.load(), s);
 }
 
 }  // namespace track

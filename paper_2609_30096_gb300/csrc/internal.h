@@ -34,27 +34,6 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
-// As launch_pdl, for a kernel launched in clusters of `cluster_x` CTAs.
-template <typename... KArgs, typename... Args>
-cudaError_t launch_pdl_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
-                               cudaStream_t s, int cluster_x, Args&&... args) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = grid;
-  cfg.blockDim = block;
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  attr[1].id = cudaLaunchAttributeClusterDimension;
-  attr[1].val.clusterDim.x = (unsigned)cluster_x;
-  attr[1].val.clusterDim.y = 1;
-  attr[1].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
-}
-
 enum Dtype { F32 = 0, BF16 = 1 };
 enum Epi { EPI_STORE = 0, EPI_GELU = 1, EPI_RESID_GATE = 2, EPI_RESID = 3 };
 
@@ -105,8 +84,7 @@ cudaError_t gemm_bf16_tc(const void* A, const void* W, const GemmArgs& g, cudaSt
 bool sk_scratch(cudaStream_t s, size_t ncnt, size_t nws, int** cnt, float** ws);
 // Bumped whenever any stream-K scratch is reallocated (recorded graphs hold its addresses).
 uint64_t sk_scratch_generation();
-// 0 auto, 1 data-parallel, 2 stream-K where the shape allows it; + 4: W tiles
-// shared by two-CTA clusters through TMA multicast.
+// 0 auto, 1 data-parallel, 2 stream-K where the shape allows it.
 void set_gemm_schedule(int mode);
 
 // ---------------------------------------------------------------- attention

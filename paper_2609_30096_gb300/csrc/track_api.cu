@@ -801,8 +801,7 @@ int track_sync(track_stream s) {
 }
 
 int track_gemm_schedule(int mode) {
-  if ((mode & ~TRACK_GEMM_MULTICAST) < TRACK_GEMM_AUTO ||
-      (mode & ~TRACK_GEMM_MULTICAST) > TRACK_GEMM_STREAM_K)
+  if (mode < TRACK_GEMM_AUTO || mode > TRACK_GEMM_STREAM_K)
     return fail(TRACK_EINVAL, "unknown GEMM schedule");
   set_gemm_schedule(mode);
   return TRACK_OK;

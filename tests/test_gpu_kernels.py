@@ -93,11 +93,9 @@ SK_SHAPES = [
 ]
 
 
-@pytest.fixture(params=["sk", "sk+multicast", "dp+multicast"])
+@pytest.fixture(params=["sk", "dp"])
 def schedule(T, request):
-    T.track_gemm_schedule({"sk": T.GEMM_STREAM_K,
-                           "sk+multicast": T.GEMM_STREAM_K | T.GEMM_MULTICAST,
-                           "dp+multicast": T.GEMM_DATA_PARALLEL | T.GEMM_MULTICAST}[request.param])
+    T.track_gemm_schedule({"sk": T.GEMM_STREAM_K, "dp": T.GEMM_DATA_PARALLEL}[request.param])
     yield request.param
     T.track_gemm_schedule(T.GEMM_AUTO)
 
@@ -137,27 +135,25 @@ def test_linear_bf16_schedules(T, schedule, M, N, K, epi):
 
 
 def test_linear_bf16_schedules_agree(T):
-    # Stream-K differs from data-parallel only in the order of fp32 partial sums;
-    # multicast under data-parallel changes no bit.
+    # Stream-K differs from data-parallel only in the order of fp32 partial sums.
     rng = np.random.default_rng(11)
     M, N, K = 3510, 1536, 8960
     X = dev_bf16(rng.normal(size=(M, K)).astype(np.float32))
     W = dev_bf16((rng.normal(size=(N, K)) / np.sqrt(K)).astype(np.float32))
     res = []
-    for mode in (T.GEMM_DATA_PARALLEL, T.GEMM_STREAM_K, T.GEMM_DATA_PARALLEL | T.GEMM_MULTICAST):
+    for mode in (T.GEMM_DATA_PARALLEL, T.GEMM_STREAM_K):
         T.track_gemm_schedule(mode)
         out = torch.zeros((M, N), dtype=torch.float32, device=DEV)
         T.track_linear(T.BF16, X, W, None, T.EPI_RESID, out)
         T.track_sync()
         res.append(out.cpu().numpy().astype(np.float64))
     T.track_gemm_schedule(T.GEMM_AUTO)
-    assert np.array_equal(res[2], res[0])
     # Two fp32 sums of K terms in different association differ by about
     # sqrt(K) * 2^-24 relative (6e-6 at K = 8960); the bound allows 3x that.
     assert rel_l2(res[1], res[0]) < 2e-5
 
 
-@pytest.mark.parametrize("mode", ["dp", "sk", "dp+multicast"])
+@pytest.mark.parametrize("mode", ["dp", "sk"])
 def test_linear_bf16_raster_groups_agree(T, mode):
     # The tile order changes which CTA computes a tile, never a data-parallel
     # tile's arithmetic: every raster group gives the same bits (65 row units,
@@ -169,8 +165,7 @@ def test_linear_bf16_raster_groups_agree(T, mode):
     X = dev_bf16(rng.normal(size=(M, K)).astype(np.float32))
     W = dev_bf16((rng.normal(size=(N, K)) / np.sqrt(K)).astype(np.float32))
     b = dev_f32(rng.normal(size=N).astype(np.float32))
-    T.track_gemm_schedule({"dp": T.GEMM_DATA_PARALLEL, "sk": T.GEMM_STREAM_K,
-                           "dp+multicast": T.GEMM_DATA_PARALLEL | T.GEMM_MULTICAST}[mode])
+    T.track_gemm_schedule({"dp": T.GEMM_DATA_PARALLEL, "sk": T.GEMM_STREAM_K}[mode])
     res = []
     try:
         for group in (0, 1, 5, 32, 65536):
