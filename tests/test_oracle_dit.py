@@ -278,9 +278,101 @@ def check_whole_forward_reduces_to_embed_and_head(cls=dit.DiT):
     return np.allclose(m.forward(x, t, ctx), dit.unpatchify(out, ARCH.latent_shape), atol=1e-11)
 
 
+# Conditioning pins (Eq. 1's t and c enter f_m through these two maps).  The
+# architecture is square (frequency, text and model widths all 32) so that
+# identity, diagonal and permutation weights are well defined.  Every closed
+# form is evaluated element by element with libm's exp and tanh.
+SQ = synth.Arch(dim=32, layers=1, heads=2, ffn=64, text_dim=32, text_len=5,
+                frames=2, height=4, width=6, freq_dim=32)
+_A = np.array([0.5, 1.5, 2.0, -1.0, 0.75, -0.25, 3.0, 1.25] * 4)     # bf16-exact diagonals
+_PERM = np.array([(7 * i + 3) % 32 for i in range(32)])              # a permutation of 0..31
+
+
+def _silu1(u):
+    return u / (1.0 + math.exp(-u))
+
+
+def _gelu1(u):
+    return 0.5 * u * (1.0 + math.tanh(math.sqrt(2.0 / math.pi) * (u + 0.044715 * u ** 3)))
+
+
+def _perm_matrix(p):
+    P = np.zeros((len(p), len(p)))
+    P[np.arange(len(p)), p] = 1.0                       # (P v)[i] = v[p[i]]
+    return P
+
+
+def check_time_embedding_identity(cls=dit.DiT, precision="fp32"):
+    # Identity W1, W2 and stacked identity mod.W, zero biases: e = SiLU(emb) and
+    # every one of the six rows of e0 is SiLU(e).
+    m = cls(SQ, synth.make_weights(SQ, 3), precision)
+    d = SQ.dim
+    m.w["tim.W1"], m.w["tim.W2"] = np.eye(d), np.eye(d)
+    m.w["mod.W"] = np.tile(np.eye(d), (6, 1))
+    _zero(m, "tim.b1", "tim.b2", "mod.b")
+    t = np.float32(421.0)
+    emb = dit.sinusoid(t, d)
+    e, e0 = m.time_embedding(t)
+    want_e = np.array([_silu1(v) for v in emb])
+    want_row = np.array([_silu1(v) for v in want_e])
+    ok = e.shape == (d,) and e0.shape == (6, d) and np.allclose(e, want_e, atol=1e-14)
+    return ok and all(np.allclose(e0[k], want_row, atol=1e-14) for k in range(6))
+
+
+def check_time_embedding_structured(cls=dit.DiT, precision="fp32"):
+    # W1 = diag(a), W2 = a permutation P, mod.W = six stacked diagonals diag(c_k),
+    # random biases:  e[i] = SiLU(a_p(i) emb_p(i) + b1_p(i)) + b2[i] and
+    # e0[k, i] = c_k[i] SiLU(e[i]) + mod.b[k d + i]  (row k of the [6, d] reshape
+    # is the k-th block of d outputs).
+    m = cls(SQ, synth.make_weights(SQ, 4), precision)
+    d = SQ.dim
+    rng = np.random.default_rng(21)
+    c = dit.round_bf16(rng.choice([0.5, -1.0, 2.0, 1.5, -0.75], size=(6, d)).astype(np.float32))
+    m.w["tim.W1"], m.w["tim.W2"] = np.diag(_A), _perm_matrix(_PERM)
+    m.w["mod.W"] = np.concatenate([np.diag(c[k]) for k in range(6)])
+    b1, b2, mb = rng.normal(size=d), rng.normal(size=d), rng.normal(size=6 * d)
+    m.w["tim.b1"], m.w["tim.b2"], m.w["mod.b"] = b1, b2, mb
+    t = np.float32(87.0)
+    emb = dit.sinusoid(t, d)
+    e, e0 = m.time_embedding(t)
+    want_e = np.array([_silu1(_A[_PERM[i]] * emb[_PERM[i]] + b1[_PERM[i]]) + b2[i] for i in range(d)])
+    want_e0 = np.array([[c[k, i] * _silu1(want_e[i]) + mb[k * d + i] for i in range(d)]
+                        for k in range(6)])
+    return np.allclose(e, want_e, atol=1e-13) and np.allclose(e0, want_e0, atol=1e-13)
+
+
+def check_text_projection_structured(cls=dit.DiT, precision="fp32"):
+    # W1 = diag(a), W2 = a permutation P, random biases:
+    # c[l, i] = GELU_tanh(a_p(i) ctx[l, p(i)] + b1_p(i)) + b2[i], with ctx rounded to
+    # bf16 first in bf16 mode (the conditioning is fed to the tensor cores in bf16).
+    m = cls(SQ, synth.make_weights(SQ, 5), precision)
+    d = SQ.dim
+    rng = np.random.default_rng(22)
+    m.w["txt.W1"], m.w["txt.W2"] = np.diag(_A), _perm_matrix(_PERM)
+    b1, b2 = rng.normal(size=d), rng.normal(size=d)
+    m.w["txt.b1"], m.w["txt.b2"] = b1, b2
+    ctx = rng.normal(size=(SQ.text_len, d)).astype(np.float32)
+    ctx[0, :] = np.float32(1.0 + 2.0 ** -10)            # not bf16-representable: rounds to 1
+    cin = dit.round_bf16(ctx) if precision == "bf16" else ctx.astype(np.float64)
+    got = m.text_projection(ctx)
+    want = np.array([[_gelu1(_A[_PERM[i]] * float(cin[l, _PERM[i]]) + b1[_PERM[i]]) + b2[i]
+                      for i in range(d)] for l in range(SQ.text_len)])
+    return got.shape == (SQ.text_len, d) and np.allclose(got, want, atol=1e-13)
+
+
+def check_text_projection_bf16(cls=dit.DiT):
+    return check_text_projection_structured(cls, "bf16")
+
+
+def check_time_embedding_bf16(cls=dit.DiT):
+    return check_time_embedding_structured(cls, "bf16")
+
+
 CHECKS = [check_gates_and_identity, check_self_attention_branch, check_ffn_branch,
           check_cross_attention_branch, check_self_attention_against_torch,
-          check_whole_forward_reduces_to_embed_and_head]
+          check_whole_forward_reduces_to_embed_and_head, check_time_embedding_identity,
+          check_time_embedding_structured, check_time_embedding_bf16,
+          check_text_projection_structured, check_text_projection_bf16]
 
 
 @pytest.mark.parametrize("layers", [1, 2])
@@ -343,7 +435,65 @@ class TransposedRope(dit.DiT):
             dit.rope = saved
 
 
+class TimeNoSiluBeforeModulation(dit.DiT):
+    def time_embedding(self, t):
+        emb = dit.sinusoid(t, self.arch.freq_dim)
+        e = dit.linear(dit.silu(dit.linear(emb, self.W("tim.W1"), self.W("tim.b1"))),
+                       self.W("tim.W2"), self.W("tim.b2"))
+        e0 = dit.linear(e, self.W("mod.W"), self.W("mod.b"))
+        return e, e0.reshape(6, self.arch.dim)
+
+
+class TimeSwappedLayers(dit.DiT):
+    def time_embedding(self, t):
+        emb = dit.sinusoid(t, self.arch.freq_dim)
+        e = dit.linear(dit.silu(dit.linear(emb, self.W("tim.W2"), self.W("tim.b1"))),
+                       self.W("tim.W1"), self.W("tim.b2"))
+        e0 = dit.linear(dit.silu(e), self.W("mod.W"), self.W("mod.b"))
+        return e, e0.reshape(6, self.arch.dim)
+
+
+class TimeModulationTransposed(dit.DiT):
+    def time_embedding(self, t):
+        e, e0 = dit.DiT.time_embedding(self, t)
+        return e, e0.reshape(-1).reshape(self.arch.dim, 6).T
+
+
+class TextGeluAfterSecondLayer(dit.DiT):
+    def text_projection(self, ctx):
+        ctx = np.asarray(ctx, dtype=np.float32)
+        if self.precision == "bf16":
+            ctx = dit.round_bf16(ctx)
+        h = dit.linear(ctx, self.W("txt.W1"), self.W("txt.b1"))
+        return dit.gelu_tanh(dit.linear(h, self.W("txt.W2"), self.W("txt.b2")))
+
+
+class TextSwappedLayers(dit.DiT):
+    def text_projection(self, ctx):
+        ctx = np.asarray(ctx, dtype=np.float32)
+        if self.precision == "bf16":
+            ctx = dit.round_bf16(ctx)
+        h = dit.gelu_tanh(dit.linear(ctx, self.W("txt.W2"), self.W("txt.b1")))
+        return dit.linear(h, self.W("txt.W1"), self.W("txt.b2"))
+
+
+class TextNoBf16Rounding(dit.DiT):
+    def text_projection(self, ctx):
+        h = dit.gelu_tanh(dit.linear(np.asarray(ctx, dtype=np.float64), self.W("txt.W1"),
+                                     self.W("txt.b1")))
+        return dit.linear(h, self.W("txt.W2"), self.W("txt.b2"))
+
+
 @pytest.mark.parametrize("mutant", [SwappedGates, ShiftScaleSwapped, CrossValuesFromLatent,
-                                    HeadDropsShift, TransposedRope], ids=lambda c: c.__name__)
+                                    HeadDropsShift, TransposedRope, TimeNoSiluBeforeModulation,
+                                    TimeSwappedLayers, TimeModulationTransposed,
+                                    TextGeluAfterSecondLayer, TextSwappedLayers,
+                                    TextNoBf16Rounding], ids=lambda c: c.__name__)
 def test_planted_mistakes_are_caught(mutant):
-    assert not all(check(mutant) for check in CHECKS)
+    def passes(check):
+        try:
+            return bool(check(mutant))
+        except ValueError:          # a shape mismatch also exposes the mistake
+            return False
+    failed = [c.__name__ for c in CHECKS if not passes(c)]
+    assert failed
