@@ -213,7 +213,8 @@ int track_cfg_step(float* x, const float* f_c, const float* f_u, int64_t n, floa
  * over the n_per_sample elements of sample b; adds r_b to score_accum[b]
  * (device, B floats).  Deterministic: identical inputs give bitwise-identical
  * results (fixed-order two-level reduction, no floating-point atomics).
- * Uses library-owned device scratch per (device, stream). */
+ * Uses library-owned device scratch per (device, stream); s must be a stream
+ * of the current device. */
 int track_disagreement(const float* v_L, const float* v_S, int B, int64_t n_per_sample,
                        float eps, float* score_accum, track_stream s);
 
@@ -403,12 +404,13 @@ int track_attention(int dtype, const void* Q, const void* K, const void* V, int 
  * fail), or a latency-critical loop that cannot take the device-wide
  * synchronization that cudaMalloc/cudaFree imply.
  *
- * Computes what track_disagreement computes (Eq. 4 per sample, added to
- * score_accum[b]), with the same arguments, but allocates nothing: its partial
+ * Computes the relative disagreement score computed by track_disagreement
+ * (added to score_accum[b]), with the same arguments, but allocates nothing: its partial
  * sums live in one fixed device array of TRACK_STATIC_MAX_SAMPLES x
  * TRACK_STATIC_MAX_BLOCKS x 2 floats (256 KiB) compiled into the library, which
  * every GPU that loads the library holds until the process exits.
  *  - B above TRACK_STATIC_MAX_SAMPLES is rejected with TRACK_EINVAL.
+ *  - s must be a stream of the current device (or NULL): TRACK_EINVAL if not.
  *  - The first call on each device looks up the array's device address
  *    (cudaGetSymbolAddress) with that device current; make that first call
  *    before any stream capture.

@@ -1,5 +1,6 @@
-// track_disagreement_static: the Eq. 4 score reduction with its scratch held in
-// a fixed device array of this library instead of memory the library allocates.
+// track_disagreement_static: the disagreement score of track_disagreement with
+// its scratch held in a fixed device array of this library instead of memory
+// the library allocates.
 //
 // Callers that cannot allocate device memory while they run - a serving process
 // whose device memory is entirely reserved up front by its own pool, so that a
@@ -51,6 +52,16 @@ extern "C" int track_disagreement_static(const float* v_L, const float* v_S, int
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
     return err(TRACK_ECUDA, "no usable current device");
+  // The array's address is per device: a stream of another device would be
+  // handed this device's copy.
+  if (s != nullptr) {
+    int sdev = -1;
+    cudaError_t e = cudaStreamGetDevice((cudaStream_t)s, &sdev);
+    if (e != cudaSuccess) return err(TRACK_EINVAL, std::string("bad stream: ") + cudaGetErrorString(e));
+    if (sdev != dev)
+      return err(TRACK_EINVAL, "the stream belongs to device " + std::to_string(sdev) +
+                                   ", not to the current device " + std::to_string(dev));
+  }
   float* scratch = nullptr;
   int sms = 0;
   {
