@@ -1,25 +1,34 @@
 """Benchmark of TRACK's routed denoising hot path on GB300.
 
-One benchmark step is one routed sampling trajectory (Eq. 3) of one request on
-the mid workload: a 1536-wide 30-block large DiT and a 768-wide 12-block small
-DiT (bf16, weights generated on the device), latent 16x9x30x52 (3510 tokens),
-text 512x4096, 4 flow-matching Euler steps, no CFG, and the policy that top-K
-(K=2) derives from a calibration run (Sec. 3.2.1, Eq. 4-5) on 8 seeds, which is
-executed and timed once before the timed region.  Each step projects its
-request's text, runs the 4 routed denoiser evaluations and the fused guidance +
-Euler updates.
+Default workload: the Wan-2.1-shaped pair of the paper's Table 1 row (a
+14B-shaped large DiT, 5120 wide, 40 blocks, 40 heads, FFN 13824, and a
+1.3B-shaped small DiT, 1536 wide, 30 blocks, 12 heads, FFN 8960; bf16, weights
+generated on the device), one 480p latent 16x21x60x104 (32760 tokens), text
+512x4096, classifier-free guidance 5 (cond and uncond batched: 2 sequences per
+forward), 50 flow-matching Euler steps with shift 5, and the top-K policy
+(K = 25) of a calibration run over 8 seeds (Sec. 3.2.1, Eq. 4-5), read from the
+score map that `bench.py --calibrate` wrote.
 
-Printed metric: routed denoise steps/s (whole job over all ranks), plus the
-all-large latency and the routed speedup, DiT TFLOPS, the roofline of the
-dominant kernel class measured with CUDA events inside the timed region, an
-end-to-end number through the C ABI with host buffers, clocks sampled during
-the timed region, and the oracle's CPU throughput on a bounded sample.
+One benchmark step is one routed denoise step (Eq. 3): the policy's model
+evaluated on the guided pair, with the guidance combine fused into the Euler
+update.  The steps walk the routed trajectory in order: the warm-up steps are
+its first steps, the timed steps the next ones (a trajectory that ends starts
+over from its x_T).  Printed metric: routed denoise steps/s of the timed
+steps, plus the full routed and all-large trajectories measured end to end
+(latency, speedup, energy), per-class kernel rooflines measured with CUDA
+events inside the step, an end-to-end number through the C ABI with host
+buffers, clocks sampled during the timed region, and the oracle's CPU
+throughput on a bounded sample.
 
     python bench.py [--steps K] [--warmup W] [--gpus N] [--impl ours|reference]
+    python bench.py --calibrate [--workload W]        # writes the score map
+    python bench.py --workload mid                    # the mid pair, whole trajectories
+    python bench.py --kernel gemm|attention|hbm|forward [--workload W] [--batch B]
 """
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import math
 import os
@@ -35,10 +44,13 @@ sys.path.insert(0, ROOT)
 
 import synth  # noqa: E402
 
-WORKLOAD = "mid"
+WORKLOAD = "wan480"
+WINDOW_WORKLOADS = ("wan480", "wan720", "serving")   # one denoise step per bench step
 METRIC = "routed denoise steps/s"
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+SCORE_MAPS = os.path.join(ROOT, "paper_2609_30096_gb300", "score_maps")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "ncu_traffic.json")
 
 
 def load_peaks():
@@ -50,21 +62,26 @@ def load_peaks():
         return FALLBACK_PEAKS, "fallback"
 
 
-def measured_traffic(kernel, flops_per_launch):
-    """DRAM bytes per launch from the committed ncu capture of `kernel`, scaled to a launch
-    of `flops_per_launch` by its FLOPs; None if the kernel's source changed since."""
-    import hashlib
+def source_digest(sources):
+    """sha1 over the named files of the package's csrc/ (the kernel's sources)."""
+    m = hashlib.sha1()
+    for src in sources:
+        with open(os.path.join(ROOT, "paper_2609_30096_gb300", "csrc", src), "rb") as f:
+            m.update(f.read())
+    return m.hexdigest()
+
+
+def measured_traffic(kernel, workload, work_per_launch):
+    """DRAM bytes per launch from the committed ncu record of `kernel` on `workload`,
+    scaled to a launch of `work_per_launch` (the record's unit of work); None if the
+    kernel's sources changed since the capture or no record exists."""
     try:
-        with open(os.path.join(ROOT, "profiles", "ncu_traffic.json")) as f:
-            rec = json.load(f)[kernel]
-        m = hashlib.sha1()
-        for src in rec["sources"]:
-            with open(os.path.join(ROOT, "paper_2609_30096_gb300", "csrc", src), "rb") as f:
-                m.update(f.read())
-        if m.hexdigest() != rec["source_sha1"]:
+        with open(TRAFFIC_FILE) as f:
+            rec = json.load(f)[kernel][workload]
+        if source_digest(rec["sources"]) != rec["source_sha1"]:
             return None, "kernel changed since the ncu capture"
-        per_flop = (rec["dram_read_bytes"] + rec["dram_write_bytes"]) / rec["flops"]
-        return per_flop * flops_per_launch, "scaled by FLOPs from " + rec["launch"]
+        per = (rec["dram_read_bytes"] + rec["dram_write_bytes"]) / rec["work"]
+        return per * work_per_launch, f"scaled by {rec['work_unit']} from {rec['launch']}"
     except Exception as e:  # noqa: BLE001
         return None, f"no capture ({type(e).__name__})"
 
@@ -80,6 +97,56 @@ def text_flops(arch, batch):
     """Once per request and model: text projection and the blocks' cross-attention K/V."""
     Lt, d, Dt, l = arch.text_len, arch.dim, arch.text_dim, arch.layers
     return batch * (2 * Lt * Dt * d + 2 * Lt * d * d + l * 2 * Lt * d * 2 * d)
+
+
+def guided_sequences(wl):
+    """Sequences per denoiser evaluation: cond (and uncond with guidance) per sample."""
+    return wl.batch * (1 if wl.cfg == 1.0 else 2)
+
+
+def policy_str(pol):
+    return "".join("S" if p else "L" for p in pol)
+
+
+# ---------------------------------------------------------------- calibration score maps
+def config_hash(wl):
+    """64-bit identifier of everything a score map depends on: the pair's
+    architectures and weight seeds, the schedule, the guidance scale and the
+    calibration seeds."""
+    desc = json.dumps({"large": wl.large.__dict__, "small": wl.small.__dict__,
+                       "seeds": [synth.SEED_LARGE, synth.SEED_SMALL, synth.SEED_LATENT,
+                                 synth.SEED_COND, synth.SEED_UNCOND],
+                       "steps": wl.steps, "shift": wl.shift, "cfg": wl.cfg,
+                       "generator": "splitmix64-irwin-hall-4"}, sort_keys=True, default=str)
+    return int.from_bytes(hashlib.sha1(desc.encode()).digest()[:8], "little")
+
+
+def score_map_path(wl):
+    return os.path.join(SCORE_MAPS, f"{wl.name}.trkscore")
+
+
+def load_policy(T, wl):
+    """(policy, q, M, provenance) from the committed score map of `wl`."""
+    path = score_map_path(wl)
+    if not os.path.exists(path):
+        raise SystemExit(f"no score map for {wl.name}: run `python bench.py --calibrate "
+                         f"--workload {wl.name}` first")
+    r, q, h = T.track_score_map_load(path)
+    if h != config_hash(wl) or r.shape[1] != wl.steps:
+        raise SystemExit(f"{path} was written for another configuration")
+    prov = {}
+    try:
+        with open(path[:-len(".trkscore")] + ".json") as f:
+            prov = json.load(f)
+    except OSError:
+        pass
+    return T.track_policy_topk(q, wl.k), q, r.shape[0], prov
+
+
+def window_steps(n_steps, first, count):
+    """Trajectory step index of bench steps first .. first+count-1: the steps walk
+    the trajectory in order and start over after its last step."""
+    return [(first + s) % n_steps for s in range(count)]
 
 
 # ---------------------------------------------------------------- ranks (replicas)
@@ -208,11 +275,20 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------- CPU oracle sample
-class OracleSample:
-    """The oracle on a bounded sample of the workload: one full-size DiT block of each
-    model (fp64 numpy), timed and extrapolated to one routed trajectory."""
+def block_flops(arch, tokens):
+    """Algorithmic FLOPs of one transformer block over `tokens` tokens of one sequence."""
+    d, F, Lt = arch.dim, arch.ffn, arch.text_len
+    return 2 * tokens * (6 * d * d + 2 * d * F) + 4 * tokens * tokens * d + 4 * tokens * Lt * d
 
-    def __init__(self, wl):
+
+class OracleSample:
+    """The oracle on a bounded sample of the workload: one DiT block of each model
+    (fp64 numpy) over the first `frames` latent frames of the workload's latent
+    (all of them when frames is None), timed and extrapolated to one full-size
+    forward of one sequence by algorithmic FLOPs (block FLOPs at the full token
+    count over those at the sample's) times the model's depth."""
+
+    def __init__(self, wl, frames=None):
         from oracle import dit
 
         self.wl = wl
@@ -220,86 +296,433 @@ class OracleSample:
         self.parts = {}
         for which, arch, seed in (("large", wl.large, synth.SEED_LARGE),
                                   ("small", wl.small, synth.SEED_SMALL)):
+            f = arch.frames if frames is None else min(frames, arch.frames)
+            sample = synth.Arch(**{**arch.__dict__, "layers": 1, "frames": f})
             specs = [s for s in synth.weight_specs(arch)
                      if not s.name.startswith("blk") or s.name.startswith("blk0.")]
             w = {s.name: synth.make_tensor(s, seed) for s in specs}
-            m = dit.DiT(synth.Arch(**{**arch.__dict__, "layers": 1}), w, "bf16")
-            x = rng.normal(size=(arch.tokens, arch.dim))
+            m = dit.DiT(sample, w, "bf16")
+            x = rng.normal(size=(sample.tokens, arch.dim))
             _, e0 = m.time_embedding(np.float32(500.0))
             c = m.text_projection(synth.draw(1, 0, (arch.text_len, arch.text_dim), 1.0))
-            self.parts[which] = (m, x, e0, c, arch.layers)
+            scale = block_flops(arch, arch.tokens) / block_flops(arch, sample.tokens)
+            self.parts[which] = (m, x, e0, c, arch.layers * scale)
+        tok = self.parts["large"][0].arch.tokens
         self.description = (
-            f"one full-size DiT block of each model (oracle, fp64 numpy, {wl.large.tokens} tokens) "
-            f"per step, extrapolated x layers x routed evaluations ({wl.steps - wl.k} large + "
-            f"{wl.k} small); embedding, head and text work not included")
+            f"one DiT block of each model (oracle, fp64 numpy) over {tok} of the "
+            f"{wl.large.tokens} tokens, extrapolated by block FLOPs to the full latent and "
+            f"x layers x sequences per evaluation ({guided_sequences(wl)}); embedding, head "
+            f"and text work not included")
 
-    def seconds_per_trajectory(self):
+    def forward_seconds(self):
+        """Extrapolated seconds of one full-size forward of one sequence, per model."""
         t = {}
-        for which, (m, x, e0, c, layers) in self.parts.items():
+        for which, (m, x, e0, c, factor) in self.parts.items():
             t0 = time.perf_counter()
             m.block(0, x, e0, c)
-            t[which] = (time.perf_counter() - t0) * layers
-        guided = 1 if self.wl.cfg == 1.0 else 2
-        return guided * ((self.wl.steps - self.wl.k) * t["large"] + self.wl.k * t["small"])
+            t[which] = (time.perf_counter() - t0) * factor
+        return t
+
+    def step_seconds(self, n_large, n_small):
+        """Extrapolated seconds per denoise step over a mix of large and small steps."""
+        t = self.forward_seconds()
+        n = n_large + n_small
+        return guided_sequences(self.wl) * (n_large * t["large"] + n_small * t["small"]) / n
 
 
-def cpu_threads():
+def cpu_cores():
+    """(threads the oracle's BLAS uses, os.cpu_count())."""
+    n = None
     try:
         from threadpoolctl import threadpool_info
-        n = [i.get("num_threads") for i in threadpool_info() if i.get("user_api") == "blas"]
-        if n:
-            return int(max(n))
+        b = [i.get("num_threads") for i in threadpool_info() if i.get("user_api") == "blas"]
+        if b:
+            n = int(max(b))
     except Exception:
         pass
-    return os.cpu_count()
+    return (n or os.cpu_count()), os.cpu_count()
+
+
+def read_score_map(path):
+    """(r [M, N], q [N], config_hash) of a score-map file, parsed on the host (the
+    little-endian layout of track_score_map_save)."""
+    with open(path, "rb") as f:
+        b = f.read()
+    if b[:8] != b"TRKSCORE" or int.from_bytes(b[8:12], "little") != 1:
+        raise SystemExit(f"{path}: not a score map")
+    M, N = int.from_bytes(b[12:16], "little"), int.from_bytes(b[16:20], "little")
+    h = int.from_bytes(b[20:28], "little")
+    v = np.frombuffer(b[28:28 + 4 * (M * N + N)], dtype="<f4")
+    return v[:M * N].reshape(M, N).copy(), v[M * N:].copy(), h
 
 
 # ---------------------------------------------------------------- reference arm
 def run_reference(args):
+    """The oracle, as it stands, on the host cores: each bench step times a bounded
+    sample of the same workload and converts it to the metric's unit."""
+    from oracle import track as otrack
+
     rank, _, _ = rank_env()
     if rank != 0:
         return 0  # the oracle baseline runs once, on rank 0
-    wl = synth.WORKLOADS[WORKLOAD]
-    sampler = OracleSample(wl)
+    wl = synth.WORKLOADS[args.workload]
+    if wl.name in WINDOW_WORKLOADS:
+        _, q, h = read_score_map(score_map_path(wl))
+        if h != config_hash(wl):
+            raise SystemExit("score map written for another configuration")
+        pol = otrack.topk_policy(q, wl.k)
+        idx = window_steps(wl.steps, args.warmup, args.steps)
+        n_small = int(sum(int(pol[i]) for i in idx))
+        mix = (args.steps - n_small, n_small)
+        sampler = OracleSample(wl, frames=1)
+    else:
+        pol = None
+        n_small = wl.k
+        mix = (wl.steps - wl.k, wl.k)
+        sampler = OracleSample(wl)
     for _ in range(args.warmup):
-        sampler.seconds_per_trajectory()
-    times = [sampler.seconds_per_trajectory() for _ in range(args.steps)]
-    desc = sampler.description
+        sampler.step_seconds(*mix)
+    times = [sampler.step_seconds(*mix) for _ in range(args.steps)]
     sec = float(np.mean(times))
-    value = wl.steps / sec
+    value = wl.batch / sec
+    threads, ncpu = cpu_cores()
+    cpu = {"value": value, "unit": "steps/s", "cores": threads, "host_cpus": ncpu,
+           "kind": "oracle", "sample": sampler.description}
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "steps/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": sec * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": wl.description, "global_batch": 1, "seq_len": wl.large.tokens},
-        "cpu_baseline": {"value": value, "unit": "steps/s", "cores": cpu_threads(),
-                         "kind": "oracle", "sample": desc},
+        "config": {"workload": wl.description, "global_batch": wl.batch,
+                   "seq_len": wl.large.tokens,
+                   "steps_large_small": list(mix)},
+        "cpu_baseline": cpu,
         "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line))
     return 0
 
 
-# ---------------------------------------------------------------- our arm
-def run_ours(args):
-    import torch
-    import torch.distributed as tdist
-
+# ---------------------------------------------------------------- calibration command
+def setup_library(args):
+    """Builds and loads the library and applies the schedule flags."""
     import paper_2609_30096_gb300 as T
     from paper_2609_30096_gb300 import _build
+
+    _build.build()
+    T.track_gemm_schedule(GEMM_SCHEDULES[args.gemm_schedule])
+    T.track_gemm_raster(args.gemm_raster)
+    T.track_attention_schedule(GEMM_SCHEDULES[args.attn_schedule]
+                               | (T.ATTN_ONE_TILE if args.attn_one_tile else 0))
+    return T
+
+
+def run_calibrate(args):
+    """Calibration of Sec. 3.2.1 (Eq. 4-5) for the workload on its calibration
+    seeds, written to the package's score map of that workload.  Samples are
+    calibrated `--calib-batch` at a time and the map is saved after every batch,
+    so an interrupted run resumes from the rows already saved."""
+    import torch
+
+    wl = synth.WORKLOADS[args.workload]
+    torch.cuda.set_device(0)
+    T = setup_library(args)
+    M = args.seeds or wl.calib_seeds
+    batch = args.calib_batch or (2 if wl.large.dim >= 5120 else M)
+    sig = T.track_schedule(wl.steps, wl.shift)
+    L = T.track_model_create_seeded(wl.large, synth.SEED_LARGE, T.BF16)
+    S = T.track_model_create_seeded(wl.small, synth.SEED_SMALL, T.BF16)
+    uses_uncond = wl.cfg != 1.0
+    path = score_map_path(wl)
+    meta_path = path[:-len(".trkscore")] + ".json"
+    os.makedirs(SCORE_MAPS, exist_ok=True)
+    rows, meta = [], {"workload": wl.description, "config_hash": f"{config_hash(wl):016x}",
+                      "seeds": f"calibration samples 0..{M - 1} (latent {synth.SEED_LATENT}+j, "
+                               f"cond {synth.SEED_COND}+j, uncond {synth.SEED_UNCOND}+j)",
+                      "batches": []}
+    if os.path.exists(path) and not args.fresh:
+        r0, _, h = T.track_score_map_load(path)
+        if h == config_hash(wl) and r0.shape[1] == wl.steps:
+            rows = list(r0[:M])
+            try:
+                with open(meta_path) as f:
+                    meta["batches"] = json.load(f).get("batches", [])
+            except OSError:
+                pass
+    stream = torch.cuda.Stream()
+    torch.cuda.set_stream(stream)
+    while len(rows) < M:
+        first = len(rows)
+        b = min(batch, M - first)
+        x, c, u = synth.calibration_inputs(wl.large, first, b, uses_uncond)
+        xd, cd = torch.from_numpy(x).cuda(), torch.from_numpy(c).cuda()
+        ud = torch.from_numpy(u).cuda() if uses_uncond else None
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record(stream)
+        r = T.track_calibrate(L, S, xd, cd, ud, wl.cfg, sig, stream=stream.cuda_stream)
+        ev1.record(stream)
+        T.track_sync(stream.cuda_stream)
+        rows.extend(r.cpu().numpy().T)
+        meta["batches"].append({"samples": [first, first + b], "seconds": ev0.elapsed_time(ev1) / 1e3})
+        meta["M"] = len(rows)
+        T.track_score_map_save(path, np.stack(rows), config_hash(wl))
+        with open(meta_path, "w") as f:
+            json.dump(meta, f, indent=1)
+        print(json.dumps({"calibrated": [first, first + b], "of": M,
+                          "seconds": meta["batches"][-1]["seconds"]}), flush=True)
+        del xd, cd, ud, r
+    _, q, _ = T.track_score_map_load(path)
+    print(json.dumps({"score_map": path, "q": [float(v) for v in q],
+                      "policy": policy_str(T.track_policy_topk(q, wl.k))}))
+    return 0
+
+
+# ---------------------------------------------------------------- the default: routed steps
+def class_summary(prof, peaks):
+    """Per-class kernel time and rate from track_profile_read's sums."""
+    out = {}
+    for k, (ms, work, n) in prof.items():
+        if not n:
+            continue
+        rec = {"ms": ms, "launches": int(n), "avg_launch_ms": ms / n}
+        if k in ("gemm", "attention"):
+            rec["tflops"] = work / (ms / 1e3) / 1e12 if ms else None
+            rec["frac_of_sustained"] = rec["tflops"] / peaks["bf16_tflops_sustained"] if ms else None
+        else:
+            rec["gb_per_s"] = work / (ms / 1e3) / 1e9 if ms else None
+            rec["frac_of_hbm"] = rec["gb_per_s"] / peaks["hbm_gbs"] if ms else None
+            rec["bytes_per_launch"] = work / n
+        out[k] = rec
+    return out
+
+
+def run_window(args):
+    """Routed denoise steps of a 14B/1.3B workload (module docstring)."""
+    import torch
+    import torch.distributed as tdist
 
     rank, local, world = rank_env()
     torch.cuda.set_device(local)
     if world > 1:
         tdist.init_process_group("nccl")
-    _build.build()
-    T.track_gemm_schedule(GEMM_SCHEDULES[args.gemm_schedule])
-    T.track_gemm_raster(args.gemm_raster)
-    T.track_attention_schedule(GEMM_SCHEDULES[args.attn_schedule]
-                                | (T.ATTN_ONE_TILE if args.attn_one_tile else 0))
+    T = setup_library(args)
+    wl = synth.WORKLOADS[args.workload]
+    B, w, N = wl.batch, wl.cfg, wl.steps
+    uses_uncond = w != 1.0
+    nseq = guided_sequences(wl)
+    sig = T.track_schedule(N, wl.shift)
+    L = T.track_model_create_seeded(wl.large, synth.SEED_LARGE, T.BF16)
+    S = T.track_model_create_seeded(wl.small, synth.SEED_SMALL, T.BF16)
+    policy, q, M, prov = load_policy(T, wl)
+    all_l = np.zeros(N, np.uint8)
 
-    wl = synth.WORKLOADS[WORKLOAD]
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.Stream(device=dev)
+    torch.cuda.set_stream(stream)
+    sid = stream.cuda_stream
+    x0, c0, u0 = synth.evaluation_inputs(wl.large, rank_first_sample(rank, B), B, uses_uncond)
+    xh = torch.from_numpy(x0).pin_memory()            # x_T of this rank's request(s)
+    ch = torch.from_numpy(c0).pin_memory()
+    uh = torch.from_numpy(u0).pin_memory() if uses_uncond else None
+    x_init = xh.to(dev)
+    xd = x_init.clone()
+    cd = ch.to(dev)
+    ud = uh.to(dev) if uses_uncond else None
+    x_host = torch.empty_like(xh).pin_memory()         # the host-driven loop's latent
+
+    def event():
+        return torch.cuda.Event(enable_timing=True)
+
+    def step(i, pol, x):
+        if i == 0:
+            x.copy_(x_init)                            # a trajectory starts from x_T
+        T.track_sample(L, S, pol[i:i + 1], sig[i:i + 2], x, cd, ud, w, stream=sid)
+
+    def step_e2e(i, pol):
+        # The latent lives on the host between steps: copy it and the request's
+        # conditioning in, run the step, read the new latent back.
+        xd.copy_(xh if i == 0 else x_host, non_blocking=True)
+        cd.copy_(ch, non_blocking=True)
+        if uses_uncond:
+            ud.copy_(uh, non_blocking=True)
+        T.track_sample(L, S, pol[i:i + 1], sig[i:i + 2], xd, cd, ud, w, stream=sid)
+        x_host.copy_(xd, non_blocking=True)
+
+    def run(indices, fn):
+        """Runs the steps back to back, bracketed by a barrier and a device sync on both
+        sides, with an event between steps: (total ms over ranks, per-step ms, launches)."""
+        if world > 1:
+            tdist.barrier()
+        torch.cuda.synchronize()
+        n0 = T.track_launch_count()
+        marks = [event() for _ in range(len(indices) + 1)]
+        marks[0].record(stream)
+        for s, i in enumerate(indices):
+            fn(i)
+            marks[s + 1].record(stream)
+        torch.cuda.synchronize()
+        T.track_sync(sid)
+        per = [marks[s].elapsed_time(marks[s + 1]) for s in range(len(indices))]
+        total = marks[0].elapsed_time(marks[-1])
+        return max_over_ranks(total, world, dev), per, T.track_launch_count() - n0
+
+    # warm-up: the routed trajectory's first W steps
+    for i in window_steps(N, 0, args.warmup):
+        step(i, policy, xd)
+    torch.cuda.synchronize()
+    x_at_window = xd.clone()
+    idx = window_steps(N, args.warmup, args.steps)
+    n_small = int(sum(int(policy[i]) for i in idx))
+    n_large = args.steps - n_small
+
+    energy = EnergyMeter(local)
+    with ClockSampler(local) as clk:
+        ms, per_step, launches = run(idx, lambda i: step(i, policy, xd))
+    clocks = clk.summary()
+    value = world * B * args.steps / (ms / 1e3)
+    fl = n_large * forward_flops(wl.large, nseq) + n_small * forward_flops(wl.small, nseq)
+    tflops = fl / (ms / 1e3) / 1e12
+
+    # kernel classes: the window's first steps again, every launch bracketed by events
+    peaks, src = load_peaks()
+    xp = x_at_window.clone()
+    T.track_profile_read()
+    T.track_profile_enable(True)
+    try:
+        n_prof = min(args.steps, args.profile_steps)
+        run(idx[:n_prof], lambda i: step(i, policy, xp))
+        prof = T.track_profile_read()
+        # one calibration step (Sec. 3.2.1: both models on the same latent, Eq. 4, the
+        # large model's update) at the middle of the schedule, for its cost and Eq. 4's rate
+        k = N // 2
+        xc = x_at_window.clone()
+        ca, cb = event(), event()
+        ca.record(stream)
+        T.track_calibrate(L, S, xc, cd, ud, w, sig[k:k + 2], stream=sid)
+        cb.record(stream)
+        T.track_sync(sid)
+        calib_step_ms = ca.elapsed_time(cb)
+        prof_calib = T.track_profile_read()
+    finally:
+        T.track_profile_enable(False)
+    del xp, xc
+    classes = class_summary(prof, peaks)
+    if "disagreement" in class_summary(prof_calib, peaks):
+        classes["disagreement"] = class_summary(prof_calib, peaks)["disagreement"]
+    dominant = max(("gemm", "attention"), key=lambda c: classes.get(c, {}).get("ms", 0.0))
+    dm, dwork, dn = prof[dominant]
+    kname = "k_gemm_tc" if dominant == "gemm" else "k_attn_pp"
+    achieved = dwork / (dm / 1e3) / 1e12
+    peak = peaks["bf16_tflops_sustained"]
+    traffic, traffic_src = measured_traffic(kname, wl.name, dwork / dn)
+    roof = {"bound": "tensor", "kernel": kname, "achieved": achieved, "peak": peak,
+            "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
+            "peak_source": f"{src} bf16 sustained (a step lasts seconds under the power cap; "
+                           f"burst {peaks['bf16_tflops']})",
+            "frac_of_burst": achieved / peaks["bf16_tflops"],
+            "traffic_unit": "bytes per launch", "traffic_source": traffic_src,
+            "launches": int(dn), "avg_launch_ms": dm / dn,
+            "share_of_timed_kernels": dm / sum(v[0] for v in prof.values()),
+            "measured_in": f"the first {n_prof} timed steps run again with a CUDA event "
+                           "before and after every kernel of the classes below"}
+
+    # e2e: the same steps through the C ABI with the latent on the host between steps
+    x_host.copy_(x_at_window)
+    ms_e2e, _, _ = run(idx, lambda i: step_e2e(i, policy))
+    e2e_value = world * B * args.steps / (ms_e2e / 1e3)
+
+    # whole trajectories, end to end (text projection included): routed and all-large
+    traj = {}
+    if not args.no_trajectories:
+        for name, pol in (("routed", policy), ("all_large", all_l)):
+            T.track_invalidate_ctx(L)
+            T.track_invalidate_ctx(S)
+            e0 = energy.read_mj()
+            t_ms, per, _ = run(list(range(N)), lambda i, pol=pol: step(i, pol, xd))
+            e1 = energy.read_mj()
+            traj[name] = {"s": t_ms / 1e3, "per_step_ms": per,
+                          "joules": (e1 - e0) / 1e3 if None not in (e0, e1) else None}
+        cl = float(np.mean(traj["all_large"]["per_step_ms"][1:]))
+        cs = float(np.mean([t for t, p in zip(traj["routed"]["per_step_ms"], policy) if p])) \
+            if policy.any() else None
+        model_s = ((N - wl.k) * cl + wl.k * (cs or 0.0)) / 1e3
+        for name in traj:
+            traj[name].pop("per_step_ms")
+        ja, jr = traj["all_large"]["joules"], traj["routed"]["joules"]
+        traj.update({
+            "speedup": traj["all_large"]["s"] / traj["routed"]["s"],
+            "ideal_flop_speedup": N / ((N - wl.k) + wl.k * forward_flops(wl.small, 1)
+                                       / forward_flops(wl.large, 1)),
+            "C_large_ms": cl, "C_small_ms": cs,
+            "cost_model": {"routed_s": model_s,
+                           "rel_err": abs(model_s - traj["routed"]["s"]) / traj["routed"]["s"],
+                           "note": "Eq. 3 cost model: (N - K) C_L + K C_S from the measured "
+                                   "per-step costs against the measured routed trajectory"},
+            "energy_savings": (1.0 - jr / ja) if ja and jr else None})
+
+    cpu = None
+    if rank == 0 and not args.skip_cpu:
+        sampler = OracleSample(wl, frames=1)
+        sec = sampler.step_seconds(n_large, n_small)
+        threads, ncpu = cpu_cores()
+        cpu = {"value": B / sec, "unit": "steps/s", "cores": threads, "host_cpus": ncpu,
+               "kind": "oracle", "sample": sampler.description}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic",
+            "config": {"workload": wl.description, "global_batch": world * B,
+                       "seq_len": wl.large.tokens, "sequences_per_forward": nseq,
+                       "parallelism": f"replicas x{world}",
+                       "timed_steps": f"trajectory steps {idx[0]}..{idx[-1]} of the {N}-step "
+                                      f"routed trajectory (warm-up: steps 0..{args.warmup - 1})",
+                       "steps_large_small": [n_large, n_small],
+                       "policy": policy_str(policy),
+                       "l2": "inputs larger than L2: every large step streams the 28.6 GB of "
+                             "bf16 weights and GB-sized activations through the 126 MB L2",
+                       "launch": "eager, one track_sample call per step"},
+            "dit_tflops": tflops, "dit_frac_of_sustained": tflops / peaks["bf16_tflops_sustained"],
+            "trajectory": traj or None,
+            "calibration": {"score_map": os.path.relpath(score_map_path(wl), ROOT), "seeds": M,
+                            "seconds": sum(b["seconds"] for b in prov.get("batches", [])) or None,
+                            "q": [float(v) for v in q], "step_ms": calib_step_ms},
+            "kernels": classes,
+            "roofline": roof,
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_value, "unit": "steps/s",
+                    "h2d_bytes_per_step": int(xh.numel() * 4 + ch.numel() * 4 +
+                                              (uh.numel() * 4 if uses_uncond else 0)),
+                    "d2h_bytes_per_step": int(xh.numel() * 4)},
+            "gpu_launches": int(launches),
+            "clocks": clocks,
+        }
+        print(json.dumps(line))
+    L.close()
+    S.close()
+    if world > 1:
+        tdist.destroy_process_group()
+    return 0
+# ---------------------------------------------------------------- whole trajectories (tiny, mid)
+def run_trajectories(args):
+    """Whole routed trajectories of a small workload (tiny, mid): each timed unit is
+    one trajectory of the request (text projection, the policy's N denoiser
+    evaluations, fused guidance + Euler updates) replayed from a CUDA graph;
+    `--steps` counts trajectories here and the line reports per denoise step.
+    The policy comes from a calibration run on the workload's seeds, executed and
+    timed before the timed region."""
+    import torch
+    import torch.distributed as tdist
+
+    rank, local, world = rank_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        tdist.init_process_group("nccl")
+    T = setup_library(args)
+
+    wl = synth.WORKLOADS[args.workload]
     B = wl.batch
     w = wl.cfg
     sig = T.track_schedule(wl.steps, wl.shift)
@@ -388,7 +811,7 @@ def run_ours(args):
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
 
         def bracketed(fn):
-            tot = {k: [0.0, 0.0, 0] for k in ("gemm", "attention", "norm")}
+            tot = {k: [0.0, 0.0, 0] for k in T.PROFILE_CLASSES}
             ms_tot = 0.0
             torch.cuda.synchronize()
             T.track_profile_read()                    # drop the priming calls' records
@@ -486,7 +909,8 @@ def run_ours(args):
         step_e2e(policy)
     ms_e2e, _ = timed(step_e2e, policy, args.steps)
 
-    per_step_ms = ms / args.steps
+    per_traj_ms = ms / args.steps
+    per_step_ms = per_traj_ms / wl.steps
     value = job_throughput(world, wl.steps, B, args.steps, ms)
     e2e_value = job_throughput(world, wl.steps, B, args.steps, ms_e2e)
     n_small = int(policy.sum())
@@ -495,18 +919,20 @@ def run_ours(args):
     fl = (n_large * forward_flops(wl.large, guided * B) + n_small * forward_flops(wl.small, guided * B)
           + (text_flops(wl.large, guided * B) if n_large else 0)
           + (text_flops(wl.small, guided * B) if n_small else 0))
-    tflops = fl / (per_step_ms / 1e3) / 1e12
+    tflops = fl / (per_traj_ms / 1e3) / 1e12
 
     peaks, src = load_peaks()
     gm, gf, gn = prof["gemm"]
     am, af, an = prof["attention"]
-    nm, nb, nn = prof["norm"]
+    nm = prof["layernorm"][0] + prof["norm_rope"][0]
+    nb = prof["layernorm"][1] + prof["norm_rope"][1]
+    nn = prof["layernorm"][2] + prof["norm_rope"][2]
     dominant = "gemm" if gm >= am else "attention"
     dm, dflops, dn = prof[dominant]
     achieved = (dflops / dn) / (dm / dn / 1e3) / 1e12 if dn else None
     peak = peaks["bf16_tflops"]
     traffic, traffic_src = measured_traffic("k_gemm_tc" if dominant == "gemm" else "k_attn_pp",
-                                            dflops / dn if dn else 0.0)
+                                            wl.name, dflops / dn if dn else 0.0)
     roof = {"bound": "tensor", "kernel": "bf16 GEMM (tcgen05)" if dominant == "gemm"
             else "flash attention (tcgen05)",
             "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
@@ -523,7 +949,7 @@ def run_ours(args):
                             "attention and norm kernel" if prof_mode == "graph" else
                             "a second pass of the timed steps launched kernel by kernel "
                             "(no graph) with per-launch CUDA events")
-                           + f" ({ms_prof / args.steps:.3f} ms/step)",
+                           + f" ({ms_prof / args.steps:.3f} ms/trajectory)",
             "other": {("attention" if dominant == "gemm" else "gemm"):
                       {"ms": am if dominant == "gemm" else gm,
                        "tflops": ((af / (am / 1e3)) if dominant == "gemm" and am
@@ -536,9 +962,10 @@ def run_ours(args):
     cpu = None
     if rank == 0 and not args.skip_cpu:
         sampler = OracleSample(wl)
-        sec = sampler.seconds_per_trajectory()
-        cpu = {"value": wl.steps / sec, "unit": "steps/s", "cores": cpu_threads(), "kind": "oracle",
-               "sample": sampler.description}
+        sec = sampler.step_seconds(wl.steps - wl.k, wl.k)
+        threads, ncpu = cpu_cores()
+        cpu = {"value": B / sec, "unit": "steps/s", "cores": threads, "host_cpus": ncpu,
+               "kind": "oracle", "sample": sampler.description}
 
     if rank == 0:
         line = {
@@ -548,11 +975,12 @@ def run_ours(args):
             "data": "synthetic",
             "config": {"workload": wl.description, "global_batch": world * B,
                        "seq_len": wl.large.tokens, "parallelism": f"replicas x{world}",
-                       "l2": "inputs larger than L2: every step streams 2.8 GB of large-model "
-                             "and 0.24 GB of small-model bf16 weights through the 126 MB L2",
+                       "l2": "inputs larger than L2: every trajectory streams the large model's "
+                             "bf16 weights (2.8 GB for the mid pair) through the 126 MB L2",
                        "policy": "".join("S" if p else "L" for p in policy),
-                       "launch": "CUDA graph replay of each trajectory (recorded once per policy)"},
-            "routed_ms": per_step_ms, "all_large_ms": ms_all_large / args.steps,
+                       "launch": "CUDA graph replay of each trajectory (recorded once per policy)",
+                       "timed_unit": f"{args.steps} whole {wl.steps}-step trajectories"},
+            "routed_trajectory_ms": per_traj_ms, "all_large_trajectory_ms": ms_all_large / args.steps,
             "speedup_vs_all_large": (ms_all_large / ms) if ms else None,
             "ideal_flop_speedup": wl.steps / (n_large + n_small *
                                               forward_flops(wl.small, 1) / forward_flops(wl.large, 1)),
@@ -579,25 +1007,16 @@ def run_ours(args):
     return 0
 
 
-# ---------------------------------------------------------------- 14B/1.3B configurations
-def run_workload(args):
-    """One guided denoiser evaluation of each model of a 14B/1.3B configuration at its
-    full size (its batch and CFG), timed with CUDA events after warm-up.  A trajectory
-    evaluates one denoiser per step (Eq. 3), so its latency is the per-step costs summed
-    over the policy: all-large N C_L, routed (N - K) C_L + K C_S.  The mid workload
-    measures that sum directly (`cost_model`, within 1 %); at these sizes a trajectory
-    of 30-50 full-size steps would take minutes, and calibrating one longer."""
+
+
+# ---------------------------------------------------------------- one forward of each model
+def run_forward(args):
+    """One guided denoiser evaluation of each model of a workload at its full size
+    (its batch and CFG), timed with CUDA events after warm-up (`--kernel forward`)."""
     import torch
 
-    import paper_2609_30096_gb300 as T
-    from paper_2609_30096_gb300 import _build
-
-    _build.build()
     torch.cuda.set_device(0)
-    T.track_gemm_schedule(GEMM_SCHEDULES[args.gemm_schedule])
-    T.track_gemm_raster(args.gemm_raster)
-    T.track_attention_schedule(GEMM_SCHEDULES[args.attn_schedule]
-                               | (T.ATTN_ONE_TILE if args.attn_one_tile else 0))
+    T = setup_library(args)
     wl = synth.WORKLOADS[args.workload]
     B, w = wl.batch, wl.cfg
     guided = 2 if w != 1.0 else 1
@@ -630,22 +1049,17 @@ def run_workload(args):
             clocks = clk.summary()
         ms = a.elapsed_time(b) / args.steps
         tf = forward_flops(arch, guided * B) / (ms / 1e3) / 1e12
-        res[which] = {"ms": ms, "tflops": tf, "frac_of_bf16_peak": tf / peaks["bf16_tflops"],
+        res[which] = {"ms": ms, "tflops": tf, "frac_of_burst": tf / peaks["bf16_tflops"],
+                      "frac_of_sustained": tf / peaks["bf16_tflops_sustained"],
                       "params": synth.param_count(arch)}
         m.close()
         del m
         torch.cuda.empty_cache()
-    cl, cs = res["large"]["ms"], res["small"]["ms"]
-    n, k = wl.steps, wl.k
     line = {
-        "workload_bench": args.workload, "workload": wl.description, "dtype": "bf16",
+        "forward_bench": args.workload, "workload": wl.description, "dtype": "bf16",
         "data": "synthetic", "sequences_per_forward": guided * B,
         "tokens_per_sequence": wl.large.tokens, "steps": args.steps, "warmup": args.warmup,
         "forward_large": res["large"], "forward_small": res["small"],
-        "denoise_steps_per_s_large": 1e3 / cl, "denoise_steps_per_s_small": 1e3 / cs,
-        "trajectory_all_large_s": n * cl / 1e3, "trajectory_routed_s": ((n - k) * cl + k * cs) / 1e3,
-        "routed_speedup": n * cl / ((n - k) * cl + k * cs),
-        "routed": f"K={k} of {n} steps on the small model (sum of measured per-step costs)",
         "peak_source": src, "clocks": clocks,
     }
     print(json.dumps(line))
@@ -661,15 +1075,8 @@ def run_kernel(args):
     sequences): the GEMMs of one block, or self- and cross-attention."""
     import torch
 
-    import paper_2609_30096_gb300 as T
-    from paper_2609_30096_gb300 import _build
-
-    _build.build()
     torch.cuda.set_device(0)
-    T.track_gemm_schedule(GEMM_SCHEDULES[args.gemm_schedule])
-    T.track_gemm_raster(args.gemm_raster)
-    T.track_attention_schedule(GEMM_SCHEDULES[args.attn_schedule]
-                                | (T.ATTN_ONE_TILE if args.attn_one_tile else 0))
+    T = setup_library(args)
     wl = synth.WORKLOADS[args.workload]
     a = wl.large
     M = args.batch * a.tokens
@@ -760,13 +1167,21 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--skip-cpu", action="store_true", help="omit the oracle CPU baseline")
-    ap.add_argument("--kernel", choices=["gemm", "attention", "hbm"], default=None,
-                    help="time one kernel class alone at the workload's shapes")
-    ap.add_argument("--batch", type=int, default=1, help="sequences for --kernel")
     ap.add_argument("--workload", choices=sorted(synth.WORKLOADS), default=WORKLOAD,
-                    help="shapes for --kernel; without --kernel, a 14B/1.3B configuration "
-                         "times one full-size denoiser evaluation of each model")
+                    help="the configuration (default: the Wan-2.1-shaped 480p pair)")
+    ap.add_argument("--skip-cpu", action="store_true", help="omit the oracle CPU baseline")
+    ap.add_argument("--no-trajectories", action="store_true",
+                    help="omit the whole routed and all-large trajectories")
+    ap.add_argument("--profile-steps", type=int, default=6,
+                    help="timed steps run again with per-kernel events")
+    ap.add_argument("--calibrate", action="store_true",
+                    help="run the workload's calibration and write its score map")
+    ap.add_argument("--seeds", type=int, default=0, help="calibration samples (default: the workload's)")
+    ap.add_argument("--calib-batch", type=int, default=0, help="calibration samples per call")
+    ap.add_argument("--fresh", action="store_true", help="recalibrate from the first sample")
+    ap.add_argument("--kernel", choices=["gemm", "attention", "hbm", "forward"], default=None,
+                    help="time one kernel class (or one forward of each model) alone")
+    ap.add_argument("--batch", type=int, default=1, help="sequences for --kernel")
     ap.add_argument("--gemm-schedule", choices=["auto", "dp", "sk"], default="auto",
                     help="bf16 GEMM schedule: makespan model, data-parallel or stream-K")
     ap.add_argument("--attn-schedule", choices=["auto", "dp", "sk"], default="auto",
@@ -779,13 +1194,15 @@ def main():
     args.warmup = max(3, args.warmup)     # at least three untimed warm-up steps
     if args.impl == "reference":
         return run_reference(args)
+    if args.calibrate:
+        return run_calibrate(args)
+    if args.kernel == "forward":
+        return run_forward(args)
     if args.kernel:
         return run_kernel(args)
-    if args.workload != WORKLOAD:
-        if args.gpus != 1 or int(os.environ.get("WORLD_SIZE", "1")) != 1:
-            ap.error("--workload runs on one GPU")
-        return run_workload(args)
-    return run_ours(args)
+    if args.workload in WINDOW_WORKLOADS:
+        return run_window(args)
+    return run_trajectories(args)
 
 
 if __name__ == "__main__":

@@ -186,15 +186,18 @@ def track_profile_enable(enable: bool):
     _check(lib().track_profile_enable(int(bool(enable))))
 
 
+PROFILE_CLASSES = ("gemm", "attention", "layernorm", "norm_rope", "update", "disagreement")
+
+
 def track_profile_read():
-    """{'gemm': (ms, flops, launches), 'attention': (ms, flops, launches),
-    'norm': (ms, bytes, launches)} since the last read."""
-    ms = (ctypes.c_double * 3)()
-    fl = (ctypes.c_double * 3)()
-    n = (ctypes.c_int64 * 3)()
+    """{class: (ms, work, launches)} since the last read, for the classes of
+    PROFILE_CLASSES; work is FLOPs for gemm and attention, bytes for the rest."""
+    k = len(PROFILE_CLASSES)
+    ms = (ctypes.c_double * k)()
+    fl = (ctypes.c_double * k)()
+    n = (ctypes.c_int64 * k)()
     _check(lib().track_profile_read(ms, fl, n))
-    return {"gemm": (ms[0], fl[0], n[0]), "attention": (ms[1], fl[1], n[1]),
-            "norm": (ms[2], fl[2], n[2])}
+    return {c: (ms[i], fl[i], n[i]) for i, c in enumerate(PROFILE_CLASSES)}
 
 
 # ---------------------------------------------------------------- models

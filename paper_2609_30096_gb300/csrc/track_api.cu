@@ -97,6 +97,17 @@ int* device_error_word() {
 }
 
 // ---------------------------------------------------------------- profiling
+// Timed classes (track_profile_read): work is FLOPs for GEMM and attention,
+// algorithmic bytes for the others.
+enum ProfClass {
+  PROF_GEMM = 0,
+  PROF_ATTN = 1,
+  PROF_LN = 2,      // LayerNorm-modulate (and the cross-attention LayerNorm)
+  PROF_NORM = 3,    // RMSNorm of q/k with 3-D RoPE, in place
+  PROF_UPDATE = 4,  // guidance combine and scheduler updates (Eq. 1, Eq. 2)
+  PROF_DIS = 5,     // Eq. 4 reduction
+  PROF_NCLASS = TRACK_PROFILE_CLASSES
+};
 struct ProfRec {
   cudaEvent_t a, b;
   int cls;
@@ -518,7 +529,7 @@ static int run_gemm(const track_model* m, const void* A, const void* W, int M, i
   g.w_static = 1;  // W is a weight of the model
   g.err = device_error_word();
   if (g.err == nullptr) return fail(TRACK_ECUDA, "device error word allocation failed");
-  ProfScope ps(0, 2.0 * M * N * (double)K, s);
+  ProfScope ps(PROF_GEMM, 2.0 * M * N * (double)K, s);
   cudaError_t e = m->dtype == BF16 ? gemm_bf16_tc(A, W, g, s)
                                    : gemm_f32((const float*)A, (const float*)W, g, s);
   if (e != cudaSuccess)
@@ -529,7 +540,7 @@ static int run_gemm(const track_model* m, const void* A, const void* W, int M, i
 static int run_attention(const track_model* m, const AttnOperand& Q, const AttnOperand& K,
                          const AttnOperand& V, void* O, int S, int Lq, int Lk, cudaStream_t s) {
   const int H = m->a.heads, hd = m->hd;
-  ProfScope ps(1, 4.0 * S * H * (double)Lq * Lk * hd, s);
+  ProfScope ps(PROF_ATTN, 4.0 * S * H * (double)Lq * Lk * hd, s);
   cudaError_t e = m->dtype == BF16 ? attention_bf16(Q, K, V, O, S, H, Lq, Lk, hd, s)
                                    : attention_f32(Q, K, V, (float*)O, S, H, Lq, Lk, hd, s);
   if (e != cudaSuccess)
@@ -537,15 +548,16 @@ static int run_attention(const track_model* m, const AttnOperand& Q, const AttnO
   return TRACK_OK;
 }
 
-// LayerNorm-modulate and in-place RMSNorm/RoPE launches, timed as class 2 with
-// their algorithmic bytes (fp32 row in + activation row out; activation in + out).
+// LayerNorm-modulate (class 2) and in-place RMSNorm/RoPE (class 3) launches,
+// timed with their algorithmic bytes (fp32 row in + activation row out;
+// activation in + out).
 static cudaError_t run_ln(const track_model* m, const float* x, int M, int d, const float* a,
                           const float* b, int mode, void* out, cudaStream_t s) {
-  ProfScope ps(2, (double)M * d * (4.0 + m->esz), s);
+  ProfScope ps(PROF_LN, (double)M * d * (4.0 + m->esz), s);
   return ln_modulate(x, M, d, a, b, mode, m->a.eps, out, m->dtype, s);
 }
 static cudaError_t run_norm(const track_model* m, const NormRopeArgs& p, cudaStream_t s) {
-  ProfScope ps(2, (double)p.rows * p.d * p.nsec * 2.0 * m->esz, s);
+  ProfScope ps(PROF_NORM, (double)p.rows * p.d * p.nsec * 2.0 * m->esz, s);
   return qk_norm_rope(p, s);
 }
 
@@ -706,6 +718,7 @@ static int denoise_impl(track_model* m, const float* x, int B, float t, const fl
   TRACK_TRY(ensure_workspace(m, nseq));  // ws.fout is read below: allocate first
   TRACK_TRY(forward(m, x, B, nseq, t, cond, uncond, m->ws.fout, s));
   const int64_t n = (int64_t)B * m->latent_n;
+  ProfScope ps(PROF_UPDATE, 12.0 * n, s);  // read f_c, f_u; write p
   LAUNCH(cfg_combine(m->ws.fout, m->ws.fout + n, n, w, v_out, s));
   return TRACK_OK;
 }
@@ -717,6 +730,7 @@ static int denoise_step_impl(track_model* m, float* x, int B, float sigma_t, flo
   TRACK_TRY(ensure_workspace(m, nseq));  // ws.fout is read below: allocate first
   TRACK_TRY(forward(m, x, B, nseq, t, cond, w == 1.f ? nullptr : uncond, m->ws.fout, s));
   const int64_t n = (int64_t)B * m->latent_n;
+  ProfScope ps(PROF_UPDATE, (w == 1.f ? 12.0 : 16.0) * n, s);  // read f_c (f_u), x; write x
   LAUNCH(cfg_euler(x, m->ws.fout, w == 1.f ? nullptr : m->ws.fout + n, n, w, sigma_next - sigma_t,
                    s));
   return TRACK_OK;
@@ -760,6 +774,7 @@ static int disagreement_impl(const float* vL, const float* vS, int B, int64_t n,
   const int nblk = disagreement_blocks(n);
   float* scr = stream_scratch(s, (size_t)B * nblk * 2);
   if (scr == nullptr) return fail(TRACK_ENOMEM, "disagreement scratch allocation failed");
+  ProfScope ps(PROF_DIS, 8.0 * B * (double)n, s);  // read p_L, p_S
   LAUNCH(disagreement(vL, vS, B, n, eps, accum, scr, nblk, s));
   return TRACK_OK;
 }
@@ -845,7 +860,7 @@ int track_profile_enable(int enable) {
 int track_profile_read(double* ms, double* flops, int64_t* launches) {
   if (!ms || !flops || !launches) return fail(TRACK_EINVAL, "NULL output");
   std::lock_guard<std::mutex> lk(g_prof_mu);
-  for (int c = 0; c < 3; ++c) {
+  for (int c = 0; c < PROF_NCLASS; ++c) {
     ms[c] = 0;
     flops[c] = 0;
     launches[c] = 0;
@@ -1227,6 +1242,7 @@ int track_calibrate(track_model* large, track_model* small, float* x, int B, con
     TRACK_TRY(denoise_impl(large, x, B, t, cond, uncond, cfg_scale, pL, st));
     TRACK_TRY(denoise_impl(small, x, B, t, cond, uncond, cfg_scale, pS, st));
     TRACK_TRY(disagreement_impl(pL, pS, B, n, eps, r_out + (size_t)k * B, st));
+    ProfScope ps(PROF_UPDATE, 12.0 * B * (double)n, st);  // read x, p_L; write x
     LAUNCH(euler_step(x, pL, (int64_t)B * n, sigmas[k + 1] - sigmas[k], st));
   }
   return TRACK_OK;

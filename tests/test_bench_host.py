@@ -1,0 +1,47 @@
+"""Host-side logic of bench.py (no GPU): the step walk, score-map provenance."""
+import numpy as np
+import pytest
+
+import bench
+import synth
+
+
+def test_window_walks_the_trajectory_and_starts_over():
+    assert bench.window_steps(50, 5, 20) == list(range(5, 25))
+    assert bench.window_steps(4, 3, 6) == [3, 0, 1, 2, 3, 0]
+    assert bench.window_steps(8, 0, 0) == []
+
+
+def test_config_hash_identifies_the_configuration():
+    h = {name: bench.config_hash(wl) for name, wl in synth.WORKLOADS.items()}
+    assert len(set(h.values())) == len(h)                      # every workload its own
+    assert bench.config_hash(synth.WORKLOADS["wan480"]) == h["wan480"]   # stable
+    assert all(0 <= v < 2 ** 64 for v in h.values())
+
+
+def test_host_reader_parses_what_the_library_writes(tmp_path):
+    T = pytest.importorskip("paper_2609_30096_gb300")
+    try:
+        T.lib()
+    except OSError as e:        # no CUDA runtime on this host
+        pytest.skip(str(e))
+    rng = np.random.default_rng(3)
+    r = rng.uniform(0.5, 1.5, size=(3, 7)).astype(np.float32)
+    path = str(tmp_path / "m.trkscore")
+    T.track_score_map_save(path, r, 0x0123456789ABCDEF)
+    rr, q, h = bench.read_score_map(path)
+    assert h == 0x0123456789ABCDEF
+    assert np.array_equal(rr, r)
+    assert np.array_equal(q, T.track_mean_score(r))
+
+
+def test_committed_score_maps_match_their_configuration():
+    import os
+    for name, wl in synth.WORKLOADS.items():
+        path = bench.score_map_path(wl)
+        if not os.path.exists(path):
+            continue
+        r, q, h = bench.read_score_map(path)
+        assert h == bench.config_hash(wl), name
+        assert r.shape == (wl.calib_seeds, wl.steps), name
+        assert np.all(np.isfinite(r)) and np.all(r >= 0), name

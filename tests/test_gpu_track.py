@@ -109,7 +109,31 @@ def test_no_cfg_prediction_parity(T, tiny, calib_inputs):
     assert rel_l2(v[0], ref) < TOL[prec]
 
 
-def test_calibration_scores_and_policy(T, tiny, calib_inputs, oracle_calibration):
+def score_bound(prec, r_ref):
+    """Largest |r_gpu - r_oracle| a calibration score may show.  fp32 mode: the
+    score tolerance.  bf16 mode: with p_L and p_S each within relative L2 e of
+    the oracle's, r = ||p_S - p_L|| / ||p_L|| moves by at most about
+    e (||p_S|| + ||p_L||) / ||p_L|| + e r <= e (2 + 2 r), since ||p_S|| / ||p_L||
+    <= 1 + r."""
+    if prec == "fp32":
+        return SCORE_TOL
+    return TOL["bf16"] * (2.0 + 2.0 * np.asarray(r_ref))
+
+
+def check_policy_rule(T, q_gpu, q_ref, K):
+    """The policy from the GPU's scores equals the oracle's wherever the oracle's
+    K-th and (K+1)-th lowest scores differ by more than the score tolerance.  The
+    workloads' seeds make that gap hold, which is asserted too, so the policy
+    comparison always runs."""
+    srt = np.sort(np.asarray(q_ref, np.float64))
+    gap = float(srt[K] - srt[K - 1])
+    assert gap > SCORE_TOL, gap
+    assert np.array_equal(T.track_policy_topk(np.asarray(q_gpu, np.float32), K),
+                          track.topk_policy(q_ref, K))
+    return gap
+
+
+def test_calibration_scores_and_policy(T, tiny, calib_inputs, oracle_calibration, parity_report):
     prec, P = tiny
     x, c, u = calib_inputs
     sig, traj, r_ref = oracle_calibration
@@ -117,19 +141,18 @@ def test_calibration_scores_and_policy(T, tiny, calib_inputs, oracle_calibration
     r = T.track_calibrate(P.L, P.S, xd, dev(c), dev(u), WL.cfg, sig)
     T.track_sync()
     r_gpu = r.cpu().numpy().T                                  # [M, N]
-    if prec == "fp32":
-        assert np.max(np.abs(r_gpu - r_ref)) < SCORE_TOL
-        # the calibration latents end on the oracle's all-large sample
-        for j in range(len(x)):
-            assert rel_l2(xd[j].cpu().numpy(), traj[j][-1]) < 1e-3
+    dr = np.abs(r_gpu - r_ref)
     q_gpu = T.track_mean_score(r_gpu)
     q_ref = track.mean_score(r_ref)
-    if prec == "fp32":
-        assert np.max(np.abs(q_gpu - q_ref)) < SCORE_TOL
-    # policy identical wherever the oracle's K-th / (K+1)-th gap exceeds the score tolerance
-    srt = np.sort(q_ref)
-    if srt[WL.k] - srt[WL.k - 1] > SCORE_TOL and prec == "fp32":
-        assert np.array_equal(T.track_policy_topk(q_gpu, WL.k), track.topk_policy(q_ref, WL.k))
+    dq = np.abs(q_gpu.astype(np.float64) - q_ref)
+    gap = check_policy_rule(T, q_gpu, q_ref, WL.k)
+    parity_report(precision=prec, max_abs_dr=float(dr.max()), max_abs_dq=float(dq.max()),
+                  oracle_gap_k=gap, K=WL.k)
+    assert np.all(dr <= score_bound(prec, r_ref)), float(dr.max())
+    assert np.max(dq) <= np.max(score_bound(prec, q_ref))
+    # the calibration latents end on the oracle's all-large sample
+    for j in range(len(x)):
+        assert rel_l2(xd[j].cpu().numpy(), traj[j][-1]) < (1e-3 if prec == "fp32" else 5e-2)
 
 
 def test_calibration_trajectory_is_the_all_large_trajectory(T, tiny, calib_inputs):
@@ -274,7 +297,7 @@ def test_timed_graph_brackets_every_kernel(T, tiny):
                 T.track_sync(s.cuda_stream)
                 got = T.track_profile_read()
                 assert torch.equal(xg, xe), call
-                for k in ("gemm", "attention", "norm"):
+                for k in ("gemm", "attention", "layernorm", "norm_rope", "update"):
                     assert got[k][2] == eager[k][2] > 0, (call, k)
                     assert got[k][1] == eager[k][1], (call, k)
                     assert got[k][0] > 0, (call, k)
