@@ -999,13 +999,18 @@ __global__ void __launch_bounds__(PP_THREADS, 1)
           for (int i = 0; i < AT_BN; ++i)
             if (kbase + i >= Lk) sv[i] = __float_as_uint(-INFINITY);
         }
+        // Row maximum: eight running maxima, two new keys each per three-input max.
         float pm[8];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) pm[j] = __uint_as_float(sv[j]);
+        for (int j = 0; j < 8; ++j) pm[j] = fmaxf(__uint_as_float(sv[j]), __uint_as_float(sv[8 + j]));
 #pragma unroll
-        for (int i = 8; i < AT_BN; ++i) pm[i & 7] = fmaxf(pm[i & 7], __uint_as_float(sv[i]));
-        const float rmax = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                                 fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+        for (int i = 16; i < AT_BN; i += 16) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            pm[j] = fmax3(pm[j], __uint_as_float(sv[i + j]), __uint_as_float(sv[i + 8 + j]));
+        }
+        const float rmax =
+            fmaxf(fmax3(pm[0], pm[1], pm[2]), fmax3(fmax3(pm[3], pm[4], pm[5]), pm[6], pm[7]));
         // finite: the first key of every key tile is valid
         const float mt = rmax * scale_log2;
         // Lazy rescaling: the running maximum moves only when it grows by more
@@ -1023,24 +1028,33 @@ __global__ void __launch_bounds__(PP_THREADS, 1)
         } else {
           m = mt;
         }
-        // P = exp2(S * scale - m), keys 16c..16c+15 packed into S columns 8c..8c+7
-        float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-        const float nm = -m;
+        // P = exp2(S * scale - m), keys 16c..16c+15 packed into S columns 8c..8c+7.
+        // The scale-and-shift and the row sum run as packed f32x2 operations on
+        // key pairs (one instruction per pair), four running pair sums.
+        const uint64_t sc2 = f32x2(scale_log2, scale_log2), nm2 = f32x2(-m, -m);
+        uint64_t ps2[4];
 #pragma unroll
         for (int c = 0; c < AT_BN / 16; ++c) {
           uint32_t pk[8];
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
-            const float p0 = exp2_approx(fmaf(__uint_as_float(sv[16 * c + 2 * i]), scale_log2, nm));
-            const float p1 =
-                exp2_approx(fmaf(__uint_as_float(sv[16 * c + 2 * i + 1]), scale_log2, nm));
-            ps[(2 * i) & 7] += p0;
-            ps[(2 * i + 1) & 7] += p1;
+            float x0, x1;
+            f32x2_split(fma_f32x2(f32x2(__uint_as_float(sv[16 * c + 2 * i]),
+                                        __uint_as_float(sv[16 * c + 2 * i + 1])),
+                                  sc2, nm2),
+                        x0, x1);
+            const float p0 = exp2_approx(x0), p1 = exp2_approx(x1);
+            const uint64_t pp = f32x2(p0, p1);
+            ps2[i & 3] = c == 0 && i < 4 ? pp : add_f32x2(ps2[i & 3], pp);
             pk[i] = pack_bf16x2(p0, p1);
           }
           tmem_st8(tS + 8 * c, pk);
         }
-        l += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+        {
+          float a0, a1;
+          f32x2_split(add_f32x2(add_f32x2(ps2[0], ps2[1]), add_f32x2(ps2[2], ps2[3])), a0, a1);
+          l += a0 + a1;
+        }
         if (rescale) {
           // O_t is idle: S_t of this key tile was issued after P V of the
           // previous one, whose completion the s_full wait observed; P V of

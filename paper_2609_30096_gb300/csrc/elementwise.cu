@@ -416,11 +416,62 @@ __global__ void __launch_bounds__(256) k_ln_mod_r(const float* __restrict__ x, i
   }
 }
 
+// Wide rows (d = 16 * blockDim.x, d % 512 == 0, e.g. 5120): one block per row,
+// each thread holding four float4 of it (coalesced: float4 t, t + T, t + 2T,
+// t + 3T), so that a row never leaves registers and several rows share an SM.
+template <typename T>
+__global__ void __launch_bounds__(1024) k_ln_mod_b(const float* __restrict__ x, int M, int d,
+                                                   const float* __restrict__ a,
+                                                   const float* __restrict__ b, int mode,
+                                                   float eps, T* __restrict__ out) {
+  pdl_wait();
+  pdl_release();
+  __shared__ float red[32];
+  const int64_t row = blockIdx.x;
+  const int nt = blockDim.x, t = threadIdx.x;
+  const float4* xr = reinterpret_cast<const float4*>(x + row * d);
+  float4 v[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) v[i] = xr[t + i * nt];
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) s += (v[i].x + v[i].y) + (v[i].z + v[i].w);
+  const float mean = block_sum(s, red) / (float)d;
+  float q = 0.f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    float u;
+    u = v[i].x - mean; q = fmaf(u, u, q);
+    u = v[i].y - mean; q = fmaf(u, u, q);
+    u = v[i].z - mean; q = fmaf(u, u, q);
+    u = v[i].w - mean; q = fmaf(u, u, q);
+  }
+  const float rstd = 1.f / sqrtf(block_sum(q, red) / (float)d + eps);
+  const float4* a4 = reinterpret_cast<const float4*>(a);
+  const float4* b4 = reinterpret_cast<const float4*>(b);
+  T* orow = out + row * d;
+  const float one = mode == 0 ? 1.f : 0.f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int j = t + i * nt;
+    const float4 aa = a4[j], bb = b4[j];
+    store4(orow + 4 * j, fmaf((v[i].x - mean) * rstd, one + aa.x, bb.x),
+           fmaf((v[i].y - mean) * rstd, one + aa.y, bb.y),
+           fmaf((v[i].z - mean) * rstd, one + aa.z, bb.z),
+           fmaf((v[i].w - mean) * rstd, one + aa.w, bb.w));
+  }
+}
+
 template <typename T>
 static cudaError_t ln_dispatch(const float* x, int M, int d, const float* a, const float* b,
                                int mode, float eps, T* out, cudaStream_t s) {
   const int g = (M + 7) / 8;
-  switch (d % 128 == 0 ? d / 128 : 0) {
+  const int c128 = d % 128 == 0 ? d / 128 : 0;  // the warp kernel's instantiations below
+  const bool warp_case = c128 == 1 || c128 == 2 || c128 == 4 || c128 == 6 || c128 == 8 ||
+                         c128 == 12 || c128 == 16 || c128 == 24 || c128 == 32;
+  if (!warp_case && d % 512 == 0 && d / 16 <= 1024)
+    return launch_pdl(k_ln_mod_b<T>, M, d / 16, 0, s, x, M, d, a, b, mode, eps, out);
+  switch (c128) {
 #define LN_CASE(V) \
   case V: return launch_pdl(k_ln_mod_r<T, V>, g, 256, 0, s, x, M, a, b, mode, eps, out);
     LN_CASE(1) LN_CASE(2) LN_CASE(4) LN_CASE(6) LN_CASE(8) LN_CASE(12) LN_CASE(16) LN_CASE(24)
@@ -597,6 +648,43 @@ __global__ void __launch_bounds__(256) k_norm_rope_r(NormRopeArgs a) {
   }
 }
 
+// bf16, wide sections (d = 16 * blockDim.x, d % 512 == 0, e.g. 5120): one block
+// per (row, section), each thread holding two 8-element chunks 8 * blockDim.x
+// elements apart, a whole number of heads when hd divides it (then both
+// chunks share one set of rotation coefficients).
+__global__ void __launch_bounds__(1024) k_norm_rope_b(NormRopeArgs a) {
+  pdl_wait();
+  pdl_release();
+  __shared__ float red[32];
+  const int64_t r = blockIdx.x / a.nsec;
+  const int j = (int)(blockIdx.x % a.nsec);
+  const int l = (int)(r % a.L);
+  const int nt = blockDim.x, t = threadIdx.x;
+  bf16* p = (bf16*)a.buf + r * a.ld + a.off0 + j * a.off_stride;
+  const float* g = a.gain0 + j * a.gain_stride;
+  float v[2][8];
+  load8(p + 8 * t, v[0]);
+  load8(p + 8 * (t + nt), v[1]);
+  float ss = 0.f;
+#pragma unroll
+  for (int c = 0; c < 2; ++c)
+#pragma unroll
+    for (int i = 0; i < 8; ++i) ss = fmaf(v[c][i], v[c][i], ss);
+  const float rstd = 1.f / sqrtf(block_sum(ss, red) / (float)a.d + a.eps);
+  const int pf = l / (a.Hp * a.Wp), ph = (l / a.Wp) % a.Hp, pw = l % a.Wp;
+  float2 cs[4];
+  const bool shared_cs = a.rope && (8 * nt) % a.hd == 0;
+  if (shared_cs) rope_coeffs(cs, (8 * t) % a.hd, a, pf, ph, pw);
+#pragma unroll
+  for (int c = 0; c < 2; ++c) {
+    const int e0 = 8 * (t + c * nt);
+    scale8(v[c], rstd, g + e0);
+    if (shared_cs) rope_apply8(v[c], cs);
+    else if (a.rope) rope8(v[c], e0 % a.hd, a, pf, ph, pw);
+    store8(p + e0, v[c]);
+  }
+}
+
 cudaError_t qk_norm_rope(const NormRopeArgs& a, cudaStream_t s) {
   if (a.nsec <= 0 || a.rows <= 0) return cudaSuccess;
   if (a.d % 8 || a.hd % 8 || a.off0 % 8 || a.off_stride % 8 || a.ld % 8 || a.gain_stride % 8)
@@ -604,8 +692,17 @@ cudaError_t qk_norm_rope(const NormRopeArgs& a, cudaStream_t s) {
   const int64_t warps = (int64_t)a.rows * a.nsec;
   const int g = (int)((warps + 7) / 8);
   cudaError_t e = cudaSuccess;
+  const int c256 = a.d % 256 == 0 ? a.d / 256 : 0;
+  const bool warp_case = c256 == 1 || c256 == 2 || c256 == 3 || c256 == 4 || c256 == 6 ||
+                         c256 == 8 || c256 == 12 || c256 == 16;
+  if (a.dtype == BF16 && !warp_case && a.d % 512 == 0 && a.d / 16 <= 1024 &&
+      (int64_t)a.rows * a.nsec < (1ll << 31)) {
+    e = launch_pdl(k_norm_rope_b, (int)(a.rows * a.nsec), a.d / 16, 0, s, a);
+    count_launch();
+    return e;
+  }
   if (a.dtype == BF16) {
-    switch (a.d % 256 == 0 ? a.d / 256 : 0) {
+    switch (c256) {
 #define NR_CASE(C) \
   case C: e = launch_pdl(k_norm_rope_r<C>, g, 256, 0, s, a); break;
       NR_CASE(1) NR_CASE(2) NR_CASE(3) NR_CASE(4) NR_CASE(6) NR_CASE(8) NR_CASE(12) NR_CASE(16)
@@ -851,66 +948,75 @@ cudaError_t multistep_step(float* x, const float* v, float* xc, float* vp, int64
 }
 
 // ---------------------------------------------------------------- disagreement (Eq. 4)
-// Pass 1: grid (nblk, B); block j of sample b sums (vS - vL)^2 and vL^2 over a fixed
-// strided subset in fp32 and writes both to scratch[(b * nblk + j) * 2 + {0, 1}].
-// Pass 2: one block per sample adds the nblk partials in a fixed order in fp64 and
-// accumulates r_b into accum[b].
+// Grid (nblk, B): block j of sample b sums (vS - vL)^2 and vL^2 over a fixed
+// strided subset in fp32 (four float4 pairs in flight per thread) and writes
+// both to part[(b * nblk + j) * 2 + {0, 1}].  The nblk partials of a sample are
+// then added in a fixed order in fp64 and r_b is accumulated into accum[b].
+// k_dis_fused does both in one launch: the block that finishes its partials
+// last for sample b (a per-sample counter, which that block resets) adds
+// them.  k_dis_partial + k_dis_final do it in two launches (the
+// allocation-free entry point, whose fixed array holds no counters).  Both
+// compute the same bits.
 constexpr int DIS_THREADS = 256;
+constexpr int DIS_UNROLL = 4;
 
-__global__ void __launch_bounds__(DIS_THREADS) k_dis_partial(const float* __restrict__ vL,
-                                                             const float* __restrict__ vS,
-                                                             int64_t n, float* __restrict__ part) {
-  pdl_wait();
-  pdl_release();
-  __shared__ float red[32];
-  const int b = blockIdx.y, nblk = gridDim.x;
-  const float* l = vL + (int64_t)b * n;
-  const float* sp = vS + (int64_t)b * n;
+__device__ __forceinline__ void dis_block_partials(const float* __restrict__ l,
+                                                   const float* __restrict__ sp, int64_t n,
+                                                   int blk, int nblk, float* red, float& td,
+                                                   float& tl) {
   float sd = 0.f, sl = 0.f;
   const int64_t stride = (int64_t)nblk * DIS_THREADS;
   const bool vec = ((((uintptr_t)l) | ((uintptr_t)sp)) & 15) == 0;
   int64_t i0 = 0;
+  auto acc4 = [&](const float4& a, const float4& c) {
+    float t;
+    t = c.x - a.x; sd = fmaf(t, t, sd); sl = fmaf(a.x, a.x, sl);
+    t = c.y - a.y; sd = fmaf(t, t, sd); sl = fmaf(a.y, a.y, sl);
+    t = c.z - a.z; sd = fmaf(t, t, sd); sl = fmaf(a.z, a.z, sl);
+    t = c.w - a.w; sd = fmaf(t, t, sd); sl = fmaf(a.w, a.w, sl);
+  };
   if (vec) {
     const int64_t n4 = n / 4;
-    for (int64_t i = blockIdx.x * (int64_t)DIS_THREADS + threadIdx.x; i < n4; i += stride) {
-      const float4 a = reinterpret_cast<const float4*>(l)[i];
-      const float4 c = reinterpret_cast<const float4*>(sp)[i];
-      float t;
-      t = c.x - a.x; sd = fmaf(t, t, sd); sl = fmaf(a.x, a.x, sl);
-      t = c.y - a.y; sd = fmaf(t, t, sd); sl = fmaf(a.y, a.y, sl);
-      t = c.z - a.z; sd = fmaf(t, t, sd); sl = fmaf(a.z, a.z, sl);
-      t = c.w - a.w; sd = fmaf(t, t, sd); sl = fmaf(a.w, a.w, sl);
+    const float4* l4 = reinterpret_cast<const float4*>(l);
+    const float4* s4 = reinterpret_cast<const float4*>(sp);
+    int64_t i = blk * (int64_t)DIS_THREADS + threadIdx.x;
+    // every load of a group is issued before the group is summed (in index order)
+    for (; i + (DIS_UNROLL - 1) * stride < n4; i += DIS_UNROLL * stride) {
+      float4 a[DIS_UNROLL], c[DIS_UNROLL];
+#pragma unroll
+      for (int u = 0; u < DIS_UNROLL; ++u) {
+        a[u] = l4[i + u * stride];
+        c[u] = s4[i + u * stride];
+      }
+#pragma unroll
+      for (int u = 0; u < DIS_UNROLL; ++u) acc4(a[u], c[u]);
     }
+    for (; i < n4; i += stride) acc4(l4[i], s4[i]);
     i0 = n4 * 4;
   }
-  for (int64_t i = i0 + blockIdx.x * (int64_t)DIS_THREADS + threadIdx.x; i < n; i += stride) {
+  for (int64_t i = i0 + blk * (int64_t)DIS_THREADS + threadIdx.x; i < n; i += stride) {
     const float t = sp[i] - l[i];
     sd = fmaf(t, t, sd);
     sl = fmaf(l[i], l[i], sl);
   }
-  const float td = block_sum(sd, red);
-  const float tl = block_sum(sl, red);
-  if (threadIdx.x == 0) {
-    part[((int64_t)b * nblk + blockIdx.x) * 2 + 0] = td;
-    part[((int64_t)b * nblk + blockIdx.x) * 2 + 1] = tl;
-  }
+  td = block_sum(sd, red);
+  tl = block_sum(sl, red);
 }
 
-__global__ void __launch_bounds__(256) k_dis_final(const float* __restrict__ part, int nblk,
-                                                   float eps, float* __restrict__ accum) {
-  pdl_wait();
-  pdl_release();
-  __shared__ double rd[256], rl[256];
-  const int b = blockIdx.x;
+// Adds sample b's nblk partials in a fixed order in fp64 (all DIS_THREADS
+// threads of the block), then accum[b] += r_b (thread 0).
+__device__ __forceinline__ void dis_combine(const float* part, int nblk, int b, float eps,
+                                            float* accum) {
+  __shared__ double rd[DIS_THREADS], rl[DIS_THREADS];
   double sd = 0.0, sl = 0.0;
-  for (int j = threadIdx.x; j < nblk; j += 256) {
-    sd += (double)part[((int64_t)b * nblk + j) * 2 + 0];
-    sl += (double)part[((int64_t)b * nblk + j) * 2 + 1];
+  for (int j = threadIdx.x; j < nblk; j += DIS_THREADS) {
+    sd += (double)__ldcg(part + ((int64_t)b * nblk + j) * 2 + 0);
+    sl += (double)__ldcg(part + ((int64_t)b * nblk + j) * 2 + 1);
   }
   rd[threadIdx.x] = sd;
   rl[threadIdx.x] = sl;
   __syncthreads();
-  for (int w = 128; w > 0; w >>= 1) {
+  for (int w = DIS_THREADS / 2; w > 0; w >>= 1) {
     if (threadIdx.x < w) {
       rd[threadIdx.x] += rd[threadIdx.x + w];
       rl[threadIdx.x] += rl[threadIdx.x + w];
@@ -921,6 +1027,54 @@ __global__ void __launch_bounds__(256) k_dis_final(const float* __restrict__ par
     const double den = fmax(sqrt(rl[0]), (double)eps);
     accum[b] += (float)(sqrt(rd[0]) / den);
   }
+}
+
+__global__ void __launch_bounds__(DIS_THREADS) k_dis_partial(const float* __restrict__ vL,
+                                                             const float* __restrict__ vS,
+                                                             int64_t n, float* __restrict__ part) {
+  pdl_wait();
+  pdl_release();
+  __shared__ float red[32];
+  const int b = blockIdx.y, nblk = gridDim.x;
+  float td, tl;
+  dis_block_partials(vL + (int64_t)b * n, vS + (int64_t)b * n, n, blockIdx.x, nblk, red, td, tl);
+  if (threadIdx.x == 0) {
+    part[((int64_t)b * nblk + blockIdx.x) * 2 + 0] = td;
+    part[((int64_t)b * nblk + blockIdx.x) * 2 + 1] = tl;
+  }
+}
+
+__global__ void __launch_bounds__(DIS_THREADS) k_dis_final(const float* __restrict__ part,
+                                                           int nblk, float eps,
+                                                           float* __restrict__ accum) {
+  pdl_wait();
+  pdl_release();
+  dis_combine(part, nblk, blockIdx.x, eps, accum);
+}
+
+__global__ void __launch_bounds__(DIS_THREADS) k_dis_fused(const float* __restrict__ vL,
+                                                           const float* __restrict__ vS, int64_t n,
+                                                           float* __restrict__ part,
+                                                           int* __restrict__ cnt, float eps,
+                                                           float* __restrict__ accum) {
+  pdl_wait();
+  pdl_release();
+  __shared__ float red[32];
+  __shared__ int last;
+  const int b = blockIdx.y, nblk = gridDim.x;
+  float td, tl;
+  dis_block_partials(vL + (int64_t)b * n, vS + (int64_t)b * n, n, blockIdx.x, nblk, red, td, tl);
+  if (threadIdx.x == 0) {
+    part[((int64_t)b * nblk + blockIdx.x) * 2 + 0] = td;
+    part[((int64_t)b * nblk + blockIdx.x) * 2 + 1] = tl;
+    __threadfence();  // the partials are visible before this block counts in
+    last = atomicAdd(cnt + b, 1) == nblk - 1 ? 1 : 0;
+  }
+  __syncthreads();
+  if (!last) return;
+  __threadfence();  // every other block's partials are visible to the loads below
+  dis_combine(part, nblk, b, eps, accum);
+  if (threadIdx.x == 0) cnt[b] = 0;  // every block has counted in: ready for the next call
 }
 
 int disagreement_blocks(int64_t n_per_sample) {
@@ -936,9 +1090,20 @@ cudaError_t disagreement(const float* vL, const float* vS, int B, int64_t n, flo
   if (B <= 0) return cudaSuccess;
   cudaError_t e = launch_pdl(k_dis_partial, dim3(nblk, B), DIS_THREADS, 0, s, vL, vS, n, scratch);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(k_dis_final, B, 256, 0, s, scratch, nblk, eps, accum);
+  e = launch_pdl(k_dis_final, B, DIS_THREADS, 0, s, scratch, nblk, eps, accum);
   if (e != cudaSuccess) return e;
   count_launch(2);
+  return cudaGetLastError();
+}
+
+cudaError_t disagreement_fused(const float* vL, const float* vS, int B, int64_t n, float eps,
+                               float* accum, float* scratch, int* counters, int nblk,
+                               cudaStream_t s) {
+  if (B <= 0) return cudaSuccess;
+  cudaError_t e = launch_pdl(k_dis_fused, dim3(nblk, B), DIS_THREADS, 0, s, vL, vS, n, scratch,
+                             counters, eps, accum);
+  if (e != cudaSuccess) return e;
+  count_launch();
   return cudaGetLastError();
 }
 

@@ -173,6 +173,11 @@ cudaError_t band_disagreement(const float* vL, const float* vS, int B, int C, in
 int disagreement_blocks(int64_t n_per_sample);
 cudaError_t disagreement(const float* vL, const float* vS, int B, int64_t n, float eps,
                          float* accum, float* scratch, int nblk, cudaStream_t s);
+// The same computation (same bits) in one launch; counters: B ints, zero before
+// the call, left at zero by it.
+cudaError_t disagreement_fused(const float* vL, const float* vS, int B, int64_t n, float eps,
+                               float* accum, float* scratch, int* counters, int nblk,
+                               cudaStream_t s);
 
 int num_sms();
 

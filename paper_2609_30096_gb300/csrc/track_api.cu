@@ -769,13 +769,44 @@ static int band_impl(const float* vL, const float* vS, int B, int C, int F, int 
   return TRACK_OK;
 }
 
+// Per-sample completion counters of the one-launch Eq. 4 reduction, one array
+// per (device, stream), zeroed when allocated; every call leaves them at zero.
+static std::mutex g_cnt_mu;
+static std::map<std::pair<int, cudaStream_t>, std::pair<int*, int>> g_dis_cnt;
+
+static int* dis_counters(cudaStream_t s, int B) {
+  const int dev = current_device();
+  std::lock_guard<std::mutex> lk(g_cnt_mu);
+  auto& slot = g_dis_cnt[std::make_pair(dev, s)];
+  if (slot.second >= B) return slot.first;
+  if (slot.first) {
+    cudaStreamSynchronize(s);
+    cudaFree(slot.first);
+  }
+  slot.first = nullptr;
+  slot.second = 0;
+  const int n = B > 64 ? B : 64;
+  int* p = nullptr;
+  if (dev_malloc((void**)&p, n * sizeof(int)) != cudaSuccess ||
+      cudaMemsetAsync(p, 0, n * sizeof(int), s) != cudaSuccess) {
+    cudaGetLastError();
+    cudaFree(p);
+    return nullptr;
+  }
+  slot.first = p;
+  slot.second = n;
+  return p;
+}
+
 static int disagreement_impl(const float* vL, const float* vS, int B, int64_t n, float eps,
                              float* accum, cudaStream_t s) {
   const int nblk = disagreement_blocks(n);
   float* scr = stream_scratch(s, (size_t)B * nblk * 2);
   if (scr == nullptr) return fail(TRACK_ENOMEM, "disagreement scratch allocation failed");
+  int* cnt = dis_counters(s, B);
+  if (cnt == nullptr) return fail(TRACK_ENOMEM, "disagreement counter allocation failed");
   ProfScope ps(PROF_DIS, 8.0 * B * (double)n, s);  // read p_L, p_S
-  LAUNCH(disagreement(vL, vS, B, n, eps, accum, scr, nblk, s));
+  LAUNCH(disagreement_fused(vL, vS, B, n, eps, accum, scr, cnt, nblk, s));
   return TRACK_OK;
 }
 

@@ -45,3 +45,18 @@ def test_committed_score_maps_match_their_configuration():
         assert h == bench.config_hash(wl), name
         assert r.shape == (wl.calib_seeds, wl.steps), name
         assert np.all(np.isfinite(r)) and np.all(r >= 0), name
+
+
+def test_timed_window_has_the_policys_split():
+    rng = np.random.default_rng(0)
+    for n, k, count, warm in ((50, 25, 20, 5), (30, 15, 20, 5), (50, 25, 7, 3), (4, 2, 20, 5)):
+        for _ in range(5):
+            pol = np.zeros(n, np.uint8)
+            pol[rng.choice(n, k, replace=False)] = 1
+            w = bench.timed_window(pol, warm, count)
+            assert warm <= w < warm + n
+            got = sum(int(pol[i]) for i in bench.window_steps(n, w, count))
+            best = min(abs(sum(int(pol[i]) for i in bench.window_steps(n, v, count))
+                           - round(count * k / n)) for v in range(warm, warm + n))
+            assert abs(got - round(count * k / n)) == best
+    assert bench.timed_window(np.zeros(10, np.uint8), 3, 4) == 3      # all-large: any window

@@ -456,6 +456,24 @@ def test_disagreement(T, B, n):
     assert torch.equal(acc, again)                                # deterministic
 
 
+@pytest.mark.parametrize("B,n", [(1, 3), (3, 2_096_641), (64, 40_000), (2, 4 * 2_096_640)])
+def test_disagreement_one_launch_equals_two_launches(T, B, n):
+    # track_disagreement runs Eq. 4 in one launch (the last block of a sample adds
+    # the partials); the allocation-free entry point runs the same partials and the
+    # same fixed-order combine in two launches: the bits must agree, call after call
+    # (the one-launch kernel's counters are reset by each call).
+    rng = np.random.default_rng(B + n)
+    pl = dev_f32(rng.normal(size=(B, n)).astype(np.float32))
+    ps = dev_f32(rng.normal(size=(B, n)).astype(np.float32))
+    for _ in range(3):
+        one = torch.full((B,), 0.125, device=DEV)
+        two = torch.full((B,), 0.125, device=DEV)
+        T.track_disagreement(pl, ps, one)
+        T.track_disagreement_static(pl, ps, two)
+        T.track_sync()
+        assert torch.equal(one, two)
+
+
 def test_disagreement_special_cases(T):
     pl = np.random.default_rng(1).normal(size=(2, 1000)).astype(np.float32)
     acc = torch.zeros(2, device=DEV)

@@ -101,6 +101,24 @@ def test_per_step_prediction_parity(T, tiny, calib_inputs, oracle_calibration):
                 assert err < TOL[prec], (prec, om.name, k, j, err)
 
 
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+@pytest.mark.parametrize("dim,heads", [(2560, 20)])
+def test_wide_model_prediction_parity(T, prec, dim, heads):
+    """Rows of 2560 features take the block-per-row LayerNorm and RMSNorm/RoPE
+    kernels (one block of threads per row, as the 14B shape's 5120 does in the
+    full-shape tests); one guided evaluation of a one-block model of that width
+    against the oracle."""
+    arch = synth.Arch(dim=dim, layers=1, heads=heads, ffn=1024, text_dim=256, text_len=32,
+                      frames=2, height=8, width=16)
+    w = synth.make_weights(arch, 4242)
+    m = T.track_model_create(arch, list(w.values()), T.FP32 if prec == "fp32" else T.BF16)
+    x, c, u = synth.evaluation_inputs(arch, 0, 1, with_uncond=True)
+    v = T.track_denoise(m, dev(x), 700.0, dev(c), dev(u), 5.0).cpu().numpy()
+    m.close()
+    ref = track.guided_prediction(dit.DiT(arch, w, prec), x[0], 0.7, c[0], u[0], 5.0)
+    assert rel_l2(v[0], ref) < TOL[prec]
+
+
 def test_no_cfg_prediction_parity(T, tiny, calib_inputs):
     prec, P = tiny
     x, c, _ = calib_inputs
