@@ -503,7 +503,7 @@ def class_summary(prof, peaks):
         if not n:
             continue
         rec = {"ms": ms, "launches": int(n), "avg_launch_ms": ms / n}
-        if k in ("gemm", "attention"):
+        if k in ("gemm", "attention", "cross_attention"):
             rec["tflops"] = work / (ms / 1e3) / 1e12 if ms else None
             rec["frac_of_sustained"] = rec["tflops"] / peaks["bf16_tflops_sustained"] if ms else None
         else:
@@ -634,10 +634,10 @@ def run_window(args):
         classes["disagreement"] = class_summary(prof_calib, peaks)["disagreement"]
     dominant = max(("gemm", "attention"), key=lambda c: classes.get(c, {}).get("ms", 0.0))
     dm, dwork, dn = prof[dominant]
-    kname = "k_gemm_tc" if dominant == "gemm" else "k_attn_pp"
+    kname = "k_gemm_tc" if dominant == "gemm" else "k_attn_pp (self-attention)"
     achieved = dwork / (dm / 1e3) / 1e12
     peak = peaks["bf16_tflops_sustained"]
-    traffic, traffic_src = measured_traffic(kname, wl.name, dwork / dn)
+    traffic, traffic_src = measured_traffic(kname.split()[0], wl.name, dwork / dn)
     roof = {"bound": "tensor", "kernel": kname, "achieved": achieved, "peak": peak,
             "unit": "TFLOP/s", "frac": achieved / peak, "traffic": traffic,
             "peak_source": f"{src} bf16 sustained (a step lasts seconds under the power cap; "
@@ -949,7 +949,7 @@ def run_trajectories(args):
 
     peaks, src = load_peaks()
     gm, gf, gn = prof["gemm"]
-    am, af, an = prof["attention"]
+    am, af, an = (a + b for a, b in zip(prof["attention"], prof["cross_attention"]))
     nm = prof["layernorm"][0] + prof["norm_rope"][0]
     nb = prof["layernorm"][1] + prof["norm_rope"][1]
     nn = prof["layernorm"][2] + prof["norm_rope"][2]
@@ -1123,21 +1123,17 @@ def run_hbm(args, T, torch):
         if kind == "disagreement":
             acc = torch.zeros(B, device="cuda")
             return lambda: T.track_disagreement(fc.view(B, -1), fu.view(B, -1), acc)
-        if kind == "disagreement_static":
-            acc = torch.zeros(B, device="cuda")
-            return lambda: T.track_disagreement_static(fc.view(B, -1), fu.view(B, -1), acc)
         bo = torch.empty(B, 6, device="cuda")
         bl, bs = fc.view(B, 16, 21, 60, 104), fu.view(B, 16, 21, 60, 104)
         return lambda: T.track_band_disagreement(bl, bs, out=bo)
 
-    per_elem = {"cfg_euler": 16.0, "multistep": 28.0, "disagreement": 8.0,
-                "disagreement_static": 8.0, "band_split": 8.0}
+    per_elem = {"cfg_euler": 16.0, "multistep": 28.0, "disagreement": 8.0, "band_split": 8.0}
     resident = {"cfg_euler": 12.0, "multistep": 28.0, "disagreement": 12.0,
-                "disagreement_static": 12.0, "band_split": 12.0}   # bytes allocated per element
+                "band_split": 12.0}   # bytes allocated per element
     out = []
     for label, B in (("one 480p request (latent 16x21x60x104)", 1),
                      ("serving batch of 4 480p requests", 4)):
-        for kind in ("cfg_euler", "multistep", "disagreement", "disagreement_static", "band_split"):
+        for kind in ("cfg_euler", "multistep", "disagreement", "band_split"):
             if kind == "band_split" and B != 1:
                 continue
             nk = B * n480                # latent elements of the step (per model prediction)

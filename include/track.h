@@ -118,15 +118,15 @@ int track_fail_next_allocations(int n);
  * and Eq. 4 launches inside track_denoise/track_denoise_step/track_calibrate/
  * track_sample are bracketed by CUDA events on their stream.
  * track_profile_read synchronizes those events and returns, per class (0 =
- * GEMM, 1 = attention, 2 = LayerNorm-modulate, 3 = RMSNorm of q/k with RoPE,
- * 4 = guidance combine and scheduler update, 5 = Eq. 4 reduction), the summed
- * event time in ms, the summed algorithmic work (FLOPs for classes 0 and 1,
- * bytes moved for the others) and the number of launches, then clears the
+ * GEMM, 1 = self-attention, 2 = LayerNorm-modulate, 3 = RMSNorm of q/k with
+ * RoPE, 4 = guidance combine and scheduler update, 5 = Eq. 4 reduction, 6 =
+ * cross-attention), the summed event time in ms, the summed algorithmic work
+ * (FLOPs for classes 0, 1 and 6, bytes moved for the others) and the number of launches, then clears the
  * records.  Arrays are host, length TRACK_PROFILE_CLASSES.  In a graph
  * recorded by track_sample_graph while timing is enabled, the brackets are
  * event-record nodes of the graph: each replay re-records the same events, so
  * read after every replay. */
-#define TRACK_PROFILE_CLASSES 6
+#define TRACK_PROFILE_CLASSES 7
 int track_profile_enable(int enable);
 int track_profile_read(double* ms, double* flops, int64_t* launches);
 

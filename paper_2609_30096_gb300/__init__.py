@@ -186,12 +186,13 @@ def track_profile_enable(enable: bool):
     _check(lib().track_profile_enable(int(bool(enable))))
 
 
-PROFILE_CLASSES = ("gemm", "attention", "layernorm", "norm_rope", "update", "disagreement")
+PROFILE_CLASSES = ("gemm", "attention", "layernorm", "norm_rope", "update", "disagreement",
+                   "cross_attention")
 
 
 def track_profile_read():
     """{class: (ms, work, launches)} since the last read, for the classes of
-    PROFILE_CLASSES; work is FLOPs for gemm and attention, bytes for the rest."""
+    PROFILE_CLASSES; work is FLOPs for gemm and the attention classes, bytes for the rest."""
     k = len(PROFILE_CLASSES)
     ms = (ctypes.c_double * k)()
     fl = (ctypes.c_double * k)()

@@ -605,6 +605,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
 // Schedules, the stream-K combine and the bounded waits are those of the
 // one-tile kernel above, with items of 256 rows.
 constexpr int PP_THREADS = 320;  // warp 0 TMA, warp 1 MMA, warps 2-5 / 6-9 softmax of tile 0 / 1
+// Of every 8 key pairs of a row, this many take their exponentials on the FMA
+// pipe (exp2_poly_x2) instead of the special-function unit.
+#ifndef ATTN_POLY_PAIRS
+#define ATTN_POLY_PAIRS 0
+#endif
 
 template <int HD>
 struct PpShape {
@@ -1043,7 +1048,13 @@ __global__ void __launch_bounds__(PP_THREADS, 1)
                                         __uint_as_float(sv[16 * c + 2 * i + 1])),
                                   sc2, nm2),
                         x0, x1);
-            const float p0 = exp2_approx(x0), p1 = exp2_approx(x1);
+            float p0, p1;
+            if (ATTN_POLY_PAIRS > 0 && (i & 7) >= 8 - ATTN_POLY_PAIRS) {
+              f32x2_split(exp2_poly_x2(x0, x1), p0, p1);  // FMA pipe (see exp2_poly_x2)
+            } else {
+              p0 = exp2_approx(x0);
+              p1 = exp2_approx(x1);
+            }
             const uint64_t pp = f32x2(p0, p1);
             ps2[i & 3] = c == 0 && i < 4 ? pp : add_f32x2(ps2[i & 3], pp);
             pk[i] = pack_bf16x2(p0, p1);

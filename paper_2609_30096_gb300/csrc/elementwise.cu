@@ -648,10 +648,12 @@ __global__ void __launch_bounds__(256) k_norm_rope_r(NormRopeArgs a) {
   }
 }
 
-// bf16, wide sections (d = 16 * blockDim.x, d % 512 == 0, e.g. 5120): one block
-// per (row, section), each thread holding two 8-element chunks 8 * blockDim.x
-// elements apart, a whole number of heads when hd divides it (then both
-// chunks share one set of rotation coefficients).
+// bf16, wide sections (d = 8 * CPT * blockDim.x, e.g. 5120 with CPT = 4 and 160
+// threads): one block per (row, section), each thread holding CPT 8-element
+// chunks 8 * blockDim.x elements apart - a whole number of heads when hd
+// divides that, and then all of a thread's chunks share one set of rotation
+// coefficients.  CPT chunks per thread keep 16 * CPT bytes per thread in flight.
+template <int CPT>
 __global__ void __launch_bounds__(1024) k_norm_rope_b(NormRopeArgs a) {
   pdl_wait();
   pdl_release();
@@ -662,12 +664,12 @@ __global__ void __launch_bounds__(1024) k_norm_rope_b(NormRopeArgs a) {
   const int nt = blockDim.x, t = threadIdx.x;
   bf16* p = (bf16*)a.buf + r * a.ld + a.off0 + j * a.off_stride;
   const float* g = a.gain0 + j * a.gain_stride;
-  float v[2][8];
-  load8(p + 8 * t, v[0]);
-  load8(p + 8 * (t + nt), v[1]);
+  float v[CPT][8];
+#pragma unroll
+  for (int c = 0; c < CPT; ++c) load8(p + 8 * (t + c * nt), v[c]);
   float ss = 0.f;
 #pragma unroll
-  for (int c = 0; c < 2; ++c)
+  for (int c = 0; c < CPT; ++c)
 #pragma unroll
     for (int i = 0; i < 8; ++i) ss = fmaf(v[c][i], v[c][i], ss);
   const float rstd = 1.f / sqrtf(block_sum(ss, red) / (float)a.d + a.eps);
@@ -676,7 +678,7 @@ __global__ void __launch_bounds__(1024) k_norm_rope_b(NormRopeArgs a) {
   const bool shared_cs = a.rope && (8 * nt) % a.hd == 0;
   if (shared_cs) rope_coeffs(cs, (8 * t) % a.hd, a, pf, ph, pw);
 #pragma unroll
-  for (int c = 0; c < 2; ++c) {
+  for (int c = 0; c < CPT; ++c) {
     const int e0 = 8 * (t + c * nt);
     scale8(v[c], rstd, g + e0);
     if (shared_cs) rope_apply8(v[c], cs);
@@ -697,7 +699,9 @@ cudaError_t qk_norm_rope(const NormRopeArgs& a, cudaStream_t s) {
                          c256 == 8 || c256 == 12 || c256 == 16;
   if (a.dtype == BF16 && !warp_case && a.d % 512 == 0 && a.d / 16 <= 1024 &&
       (int64_t)a.rows * a.nsec < (1ll << 31)) {
-    e = launch_pdl(k_norm_rope_b, (int)(a.rows * a.nsec), a.d / 16, 0, s, a);
+    const int blocks = (int)(a.rows * a.nsec);
+    e = a.d % 1024 == 0 ? launch_pdl(k_norm_rope_b<4>, blocks, a.d / 32, 0, s, a)
+                        : launch_pdl(k_norm_rope_b<2>, blocks, a.d / 16, 0, s, a);
     count_launch();
     return e;
   }

@@ -291,6 +291,38 @@ __device__ __forceinline__ uint64_t add_f32x2(uint64_t a, uint64_t b) {
   asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
 }
+__device__ __forceinline__ uint64_t sub_f32x2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+// 2^x for two values on the FMA and integer pipes instead of the special-function
+// unit.  Range reduction as in Cody and Waite: n = round(x) by adding the
+// shifter 1.5 * 2^23 (n then sits in the low mantissa bits of the sum), f = x - n
+// in [-1/2, 1/2]; 2^f by a degree-3 polynomial whose coefficients minimise the
+// maximum relative error on [-1/2, 1/2] (Remez exchange; 7.5e-5 for results
+// above 2^-125, below bf16's 2^-9 rounding of P); then n is added to the
+// exponent field.  x is clamped at
+// -126 (2^-126: nothing below it survives P's bf16 rounding next to the row's
+// maximum, which is 1).
+constexpr float EXP2_C0 = 0.99992805719375610f, EXP2_C1 = 0.69326096773147583f,
+                EXP2_C2 = 0.24261112511157990f, EXP2_C3 = 0.05517166852951050f;
+__device__ __forceinline__ uint64_t exp2_poly_x2(float x0, float x1) {
+  const uint64_t shifter = f32x2(12582912.f, 12582912.f);
+  const uint64_t x = f32x2(fmaxf(x0, -126.f), fmaxf(x1, -126.f));
+  const uint64_t j = add_f32x2(x, shifter);
+  const uint64_t f = sub_f32x2(x, sub_f32x2(j, shifter));
+  uint64_t p = fma_f32x2(f, f32x2(EXP2_C3, EXP2_C3), f32x2(EXP2_C2, EXP2_C2));
+  p = fma_f32x2(p, f, f32x2(EXP2_C1, EXP2_C1));
+  p = fma_f32x2(p, f, f32x2(EXP2_C0, EXP2_C0));
+  uint32_t j0, j1, p0, p1;
+  asm("mov.b64 {%0, %1}, %2;" : "=r"(j0), "=r"(j1) : "l"(j));
+  asm("mov.b64 {%0, %1}, %2;" : "=r"(p0), "=r"(p1) : "l"(p));
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "r"(p0 + (j0 << 23)), "r"(p1 + (j1 << 23)));
+  return r;
+}
+
 // max(a, b, c) in one instruction.
 __device__ __forceinline__ float fmax3(float a, float b, float c) {
   float d;

@@ -101,11 +101,12 @@ int* device_error_word() {
 // algorithmic bytes for the others.
 enum ProfClass {
   PROF_GEMM = 0,
-  PROF_ATTN = 1,
+  PROF_ATTN = 1,    // self-attention
   PROF_LN = 2,      // LayerNorm-modulate (and the cross-attention LayerNorm)
   PROF_NORM = 3,    // RMSNorm of q/k with 3-D RoPE, in place
   PROF_UPDATE = 4,  // guidance combine and scheduler updates (Eq. 1, Eq. 2)
   PROF_DIS = 5,     // Eq. 4 reduction
+  PROF_XATTN = 6,   // cross-attention to the text tokens
   PROF_NCLASS = TRACK_PROFILE_CLASSES
 };
 struct ProfRec {
@@ -540,7 +541,7 @@ static int run_gemm(const track_model* m, const void* A, const void* W, int M, i
 static int run_attention(const track_model* m, const AttnOperand& Q, const AttnOperand& K,
                          const AttnOperand& V, void* O, int S, int Lq, int Lk, cudaStream_t s) {
   const int H = m->a.heads, hd = m->hd;
-  ProfScope ps(PROF_ATTN, 4.0 * S * H * (double)Lq * Lk * hd, s);
+  ProfScope ps(Lq == Lk ? PROF_ATTN : PROF_XATTN, 4.0 * S * H * (double)Lq * Lk * hd, s);
   cudaError_t e = m->dtype == BF16 ? attention_bf16(Q, K, V, O, S, H, Lq, Lk, hd, s)
                                    : attention_f32(Q, K, V, (float*)O, S, H, Lq, Lk, hd, s);
   if (e != cudaSuccess)

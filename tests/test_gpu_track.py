@@ -315,7 +315,8 @@ def test_timed_graph_brackets_every_kernel(T, tiny):
                 T.track_sync(s.cuda_stream)
                 got = T.track_profile_read()
                 assert torch.equal(xg, xe), call
-                for k in ("gemm", "attention", "layernorm", "norm_rope", "update"):
+                for k in ("gemm", "attention", "cross_attention", "layernorm", "norm_rope",
+                          "update"):
                     assert got[k][2] == eager[k][2] > 0, (call, k)
                     assert got[k][1] == eager[k][1], (call, k)
                     assert got[k][0] > 0, (call, k)
