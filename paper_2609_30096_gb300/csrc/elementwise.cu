@@ -961,8 +961,30 @@ cudaError_t multistep_step(float* x, const float* v, float* xc, float* vp, int64
 // them.  k_dis_partial + k_dis_final do it in two launches (the
 // allocation-free entry point, whose fixed array holds no counters).  Both
 // compute the same bits.
-constexpr int DIS_THREADS = 256;
+constexpr int DIS_THREADS = 512;
 constexpr int DIS_UNROLL = 4;
+
+// Block-wide sums of two floats per thread in one pass (blockDim.x ==
+// DIS_THREADS): warp shuffles, then warp 0 adds the per-warp sums in order.
+__device__ __forceinline__ void block_sum2(float& a, float& b, float* red) {
+  for (int o = 16; o > 0; o >>= 1) {
+    a += __shfl_xor_sync(0xffffffffu, a, o);
+    b += __shfl_xor_sync(0xffffffffu, b, o);
+  }
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  if (l == 0) {
+    red[w] = a;
+    red[32 + w] = b;
+  }
+  __syncthreads();
+  float ta = 0.f, tb = 0.f;
+  for (int i = 0; i < DIS_THREADS / 32; ++i) {  // same order in every thread
+    ta += red[i];
+    tb += red[32 + i];
+  }
+  a = ta;
+  b = tb;
+}
 
 __device__ __forceinline__ void dis_block_partials(const float* __restrict__ l,
                                                    const float* __restrict__ sp, int64_t n,
@@ -1003,33 +1025,40 @@ __device__ __forceinline__ void dis_block_partials(const float* __restrict__ l,
     sd = fmaf(t, t, sd);
     sl = fmaf(l[i], l[i], sl);
   }
-  td = block_sum(sd, red);
-  tl = block_sum(sl, red);
+  block_sum2(sd, sl, red);
+  td = sd;
+  tl = sl;
 }
 
 // Adds sample b's nblk partials in a fixed order in fp64 (all DIS_THREADS
-// threads of the block), then accum[b] += r_b (thread 0).
+// threads of the block: strided per-thread sums, warp shuffles, then thread 0
+// adds the warps' sums in order), then accum[b] += r_b (thread 0).
 __device__ __forceinline__ void dis_combine(const float* part, int nblk, int b, float eps,
                                             float* accum) {
-  __shared__ double rd[DIS_THREADS], rl[DIS_THREADS];
+  __shared__ double rd[DIS_THREADS / 32], rl[DIS_THREADS / 32];
   double sd = 0.0, sl = 0.0;
   for (int j = threadIdx.x; j < nblk; j += DIS_THREADS) {
-    sd += (double)__ldcg(part + ((int64_t)b * nblk + j) * 2 + 0);
-    sl += (double)__ldcg(part + ((int64_t)b * nblk + j) * 2 + 1);
+    const float2 v = __ldcg(reinterpret_cast<const float2*>(part) + (int64_t)b * nblk + j);
+    sd += (double)v.x;
+    sl += (double)v.y;
   }
-  rd[threadIdx.x] = sd;
-  rl[threadIdx.x] = sl;
+  for (int o = 16; o > 0; o >>= 1) {
+    sd += __shfl_xor_sync(0xffffffffu, sd, o);
+    sl += __shfl_xor_sync(0xffffffffu, sl, o);
+  }
+  if ((threadIdx.x & 31) == 0) {
+    rd[threadIdx.x >> 5] = sd;
+    rl[threadIdx.x >> 5] = sl;
+  }
   __syncthreads();
-  for (int w = DIS_THREADS / 2; w > 0; w >>= 1) {
-    if (threadIdx.x < w) {
-      rd[threadIdx.x] += rd[threadIdx.x + w];
-      rl[threadIdx.x] += rl[threadIdx.x + w];
-    }
-    __syncthreads();
-  }
   if (threadIdx.x == 0) {
-    const double den = fmax(sqrt(rl[0]), (double)eps);
-    accum[b] += (float)(sqrt(rd[0]) / den);
+    double td = 0.0, tl = 0.0;
+    for (int i = 0; i < DIS_THREADS / 32; ++i) {
+      td += rd[i];
+      tl += rl[i];
+    }
+    const double den = fmax(sqrt(tl), (double)eps);
+    accum[b] += (float)(sqrt(td) / den);
   }
 }
 
@@ -1038,7 +1067,7 @@ __global__ void __launch_bounds__(DIS_THREADS) k_dis_partial(const float* __rest
                                                              int64_t n, float* __restrict__ part) {
   pdl_wait();
   pdl_release();
-  __shared__ float red[32];
+  __shared__ float red[64];
   const int b = blockIdx.y, nblk = gridDim.x;
   float td, tl;
   dis_block_partials(vL + (int64_t)b * n, vS + (int64_t)b * n, n, blockIdx.x, nblk, red, td, tl);
@@ -1063,7 +1092,7 @@ __global__ void __launch_bounds__(DIS_THREADS) k_dis_fused(const float* __restri
                                                            float* __restrict__ accum) {
   pdl_wait();
   pdl_release();
-  __shared__ float red[32];
+  __shared__ float red[64];
   __shared__ int last;
   const int b = blockIdx.y, nblk = gridDim.x;
   float td, tl;

@@ -3,10 +3,14 @@
 // Persistent, warp-specialised kernel, one CTA per SM.  A CTA follows one of
 // two schedules:
 //   data-parallel  CTA w takes output tiles w, w + G, ... (whole K loop);
-//   stream-K       the tiles' k-blocks form one sequence of U units and CTA w
-//                  takes the contiguous share [w U / G, (w+1) U / G), so every
-//                  CTA does the same number of k-blocks whatever the tile
-//                  count.  A tile split across CTAs is finished by whichever
+//   stream-K       tiles of all full waves but the last are taken whole and
+//                  round-robin; the remaining tiles' k-blocks form one
+//                  sequence of U units and CTA w takes the contiguous share
+//                  [w U / G, (w+1) U / G), so every CTA does the same number
+//                  of k-blocks whatever the tile count (sharing out every tile
+//                  this way would scatter the tiles in flight over the whole
+//                  output and defeat L2 reuse of A and W at large sizes).  A
+//                  tile split across CTAs is finished by whichever
 //                  ends its part last: the others write their fp32 partial
 //                  sums to a workspace slot and count in on a per-(tile, warp)
 //                  counter; the last one adds the parts in k order (a fixed
@@ -72,7 +76,8 @@ __device__ __forceinline__ uint32_t pack2(float a, float b) {
 struct SkArgs {
   int* cnt;
   float* ws;
-  int64_t units;  // work tiles * k-blocks
+  int64_t units;  // k-blocks of the stream-K tiles (tiles dp_tiles .. end)
+  int dp_tiles;   // leading tiles taken whole, round-robin
 };
 
 constexpr int SK_MAX_PARTS = 4;     // the host only picks stream-K when no tile spans more workers
@@ -180,7 +185,7 @@ __global__ void __launch_bounds__(192, 1)
       uint32_t armed[STAGES];
 #pragma unroll
       for (int i = 0; i < STAGES; ++i) armed[i] = 0;
-      SegIter it(use_sk, sk.units, num_tiles, nk, worker, workers);
+      SegIter it(use_sk, sk.units, num_tiles, nk, worker, workers, sk.dp_tiles);
       int pre = 0;  // k-blocks of the first segment whose W tile is already requested
       if (g.w_static) {
         SegIter first = it;
@@ -243,7 +248,7 @@ __global__ void __launch_bounds__(192, 1)
       constexpr uint32_t idesc = idesc_bf16(BM, BN);
       int stage = 0, acc = 0;
       uint32_t phase = 0, acc_phase = 0;
-      SegIter it(use_sk, sk.units, num_tiles, nk, worker, workers);
+      SegIter it(use_sk, sk.units, num_tiles, nk, worker, workers, sk.dp_tiles);
       int tile, kb0, kb1;
       while (it.next(tile, kb0, kb1)) {
         if (!mbar_wait(su32(&acce[acc]), acc_phase ^ 1, abort_flag, g.err, 2)) break;
@@ -287,7 +292,7 @@ __global__ void __launch_bounds__(192, 1)
     uint32_t acc_phase = 0;
     const int64_t U = sk.units;
     constexpr int SLOT = BM * BN;  // floats per partial-sum slot
-    SegIter it(use_sk, U, num_tiles, nk, worker, workers);
+    SegIter it(use_sk, U, num_tiles, nk, worker, workers, sk.dp_tiles);
     int tile, kb0, kb1;
     while (it.next(tile, kb0, kb1)) {
       int mu, nt;
@@ -318,13 +323,13 @@ __global__ void __launch_bounds__(192, 1)
       // segment, 2w+1 for its last.
       auto slot_of = [&](int i) -> float4* {
         const int wi = w_first + i;
-        const int first_tile = (int)(((int64_t)wi * U / workers) / nk);
+        const int first_tile = sk.dp_tiles + (int)(((int64_t)wi * U / workers) / nk);
         const int s = 2 * wi + (first_tile == tile ? 0 : 1);
         return reinterpret_cast<float4*>(sk.ws + (size_t)s * SLOT);
       };
       const int rowq = quarter * 32 + lane;  // this thread's row within the tile
       if (kb0 != 0 || kb1 != nk) {
-        const int64_t tu = (int64_t)tile * nk;
+        const int64_t tu = (int64_t)(tile - sk.dp_tiles) * nk;  // the tile's first unit
         w_first = sk_worker_of(tu, U, workers);
         nparts = sk_worker_of(tu + nk - 1, U, workers) - w_first + 1;
         part = worker - w_first;
@@ -600,13 +605,18 @@ cudaError_t launch_tc(const void* A, const void* W, const GemmArgs& g_in, bool s
   const int tiles = m_units * ((g.N + BN - 1) / BN);
   const int wmax = max_workers();
   int workers = tiles < wmax ? tiles : wmax;
-  SkArgs sk = {nullptr, nullptr, 0};
+  SkArgs sk = {nullptr, nullptr, 0, 0};
   if (stream_k) {
-    sk.units = (int64_t)tiles * (g.K / BK);
+    // All but the last full wave and the partial one are taken whole and
+    // round-robin (the tiles in flight stay neighbours in the raster order, so
+    // their A and W blocks are shared in L2); stream-K evens out the rest.
+    const int full = tiles / wmax;
+    sk.dp_tiles = full > 1 ? (full - 1) * wmax : 0;
+    sk.units = (int64_t)(tiles - sk.dp_tiles) * (g.K / BK);
     if (sk_scratch(s, (size_t)4 * tiles, (size_t)2 * wmax * BM * BN, &sk.cnt, &sk.ws))
       workers = wmax;
     else
-      sk = {nullptr, nullptr, 0};
+      sk = {nullptr, nullptr, 0, 0};
   }
   count_launch();
   return launch_pdl(k_gemm_tc<BN, STAGES>, workers, 192, S::SMEM, s, ta, tb, tc, g, sk);

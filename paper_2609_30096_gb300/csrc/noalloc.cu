@@ -29,7 +29,6 @@ __device__ __align__(256) float g_dis_scratch[kMaxSamples * kMaxBlocks * 2];
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
 float* g_scratch_ptr[kMaxDevices] = {};  // device address of g_dis_scratch, per device
-int g_sm_count[kMaxDevices] = {};
 
 int err(int code, const std::string& msg) {
   return report_error(code, ("track_disagreement_static: " + msg).c_str());
@@ -63,7 +62,6 @@ extern "C" int track_disagreement_static(const float* v_L, const float* v_S, int
                                    ", not to the current device " + std::to_string(dev));
   }
   float* scratch = nullptr;
-  int sms = 0;
   {
     // One-time set-up per device, with that device current: the host-side name
     // g_dis_scratch is only a stand-in, so its device address is looked up here.
@@ -73,21 +71,14 @@ extern "C" int track_disagreement_static(const float* v_L, const float* v_S, int
       cudaError_t e = cudaGetSymbolAddress(&p, g_dis_scratch);
       if (e != cudaSuccess) return err(TRACK_ECUDA, std::string("cudaGetSymbolAddress: ") +
                                                       cudaGetErrorString(e));
-      int n = 0;
-      e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-      if (e != cudaSuccess || n <= 0) return err(TRACK_ECUDA, "cannot read the SM count");
       g_scratch_ptr[dev] = (float*)p;
-      g_sm_count[dev] = n;
     }
     scratch = g_scratch_ptr[dev];
-    sms = g_sm_count[dev];
   }
-  // Same partition as track_disagreement (blocks of 256 threads x 16 elements, at
-  // most two blocks per SM), capped by the array's size.
-  int64_t nblk = (n_per_sample + 256 * 16 - 1) / (256 * 16);
-  if (nblk > 2 * (int64_t)sms) nblk = 2 * (int64_t)sms;
+  // Same partition as track_disagreement (so both give the same bits), capped
+  // by the array's size.
+  int64_t nblk = disagreement_blocks(n_per_sample);
   if (nblk > kMaxBlocks) nblk = kMaxBlocks;
-  if (nblk < 1) nblk = 1;
   // Every partial slot the reduction reads is written earlier in the same call,
   // so nothing needs clearing between calls.
   cudaError_t e = disagreement(v_L, v_S, B, n_per_sample, eps, score_accum, scratch, (int)nblk,

@@ -340,34 +340,40 @@ __device__ __forceinline__ int sk_worker_of(int64_t u, int64_t U, int G) {
 // Segment sequence of worker w of G: (work tile, first k-block, end k-block).
 struct SegIter {
   int64_t u, u1;
-  int tile, stride, num_tiles, nk;
+  int tile, stride, num_tiles, nk, dp_end;
   bool sk;
-  __device__ SegIter(bool sk_, int64_t U, int num_tiles_, int nk_, int w, int G) {
+  // Without stream-K, worker w takes tiles w, w + G, ...  With stream-K, the
+  // first dp_tiles tiles (a multiple of G) still go round-robin, keeping the
+  // tiles in flight at a time close together in the tile order, and only the
+  // U units of the remaining tiles are shared out contiguously.
+  __device__ SegIter(bool sk_, int64_t U, int num_tiles_, int nk_, int w, int G, int dp_tiles = 0) {
     sk = sk_;
     num_tiles = num_tiles_;
     nk = nk_;
+    dp_end = sk ? dp_tiles : num_tiles;
     u = (int64_t)w * U / G;
     u1 = (int64_t)(w + 1) * U / G;
     tile = w;
     stride = G;
   }
   // True once the segment just returned is the worker's last.
-  __device__ bool done() const { return sk ? u >= u1 : tile >= num_tiles; }
+  __device__ bool done() const { return tile >= dp_end && (!sk || u >= u1); }
+  // Tile t (absolute), k-blocks [k0, k1).  Stream-K tiles are numbered from dp_end.
   __device__ bool next(int& t, int& k0, int& k1) {
-    if (sk) {
-      if (u >= u1) return false;
-      t = (int)(u / nk);
-      k0 = (int)(u - (int64_t)t * nk);
-      const int64_t left = u1 - u;
-      k1 = left < (int64_t)(nk - k0) ? k0 + (int)left : nk;
-      u += k1 - k0;
+    if (tile < dp_end) {
+      t = tile;
+      k0 = 0;
+      k1 = nk;
+      tile += stride;
       return true;
     }
-    if (tile >= num_tiles) return false;
-    t = tile;
-    k0 = 0;
-    k1 = nk;
-    tile += stride;
+    if (!sk || u >= u1) return false;
+    const int64_t tt = u / nk;
+    t = dp_end + (int)tt;
+    k0 = (int)(u - tt * nk);
+    const int64_t left = u1 - u;
+    k1 = left < (int64_t)(nk - k0) ? k0 + (int)left : nk;
+    u += k1 - k0;
     return true;
   }
 };

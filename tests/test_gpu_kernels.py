@@ -84,12 +84,15 @@ def test_linear_bf16_tcgen05(T, M, N, K, epi):
 
 # Stream-K forced where the shape allows it: a ragged 32-column last tile and
 # ragged rows (three CTAs per tile), the output projection at 3510 tokens (two),
-# wide N, and K = 4096 over 52 tiles, where a tile spans four CTAs.
+# wide N, K = 4096 over 52 tiles, where a tile spans four CTAs, and two shapes of
+# several waves, whose leading waves are taken whole before the stream-K tail.
 SK_SHAPES = [
     (2000, 1568, 1536),
     (3510, 1536, 1536),
     (600, 8960, 1536),
     (1664, 1024, 4096),
+    (8250, 1536, 512),     # 390 tiles: one wave taken whole, the rest stream-K
+    (16300, 2048, 256),    # 1024 tiles: five waves whole, ragged rows
 ]
 
 
