@@ -649,6 +649,10 @@ def run_window(args):
             "measured_in": f"the first {n_prof} timed steps run again with a CUDA event "
                            "before and after every kernel of the classes below"}
 
+    # the update and Eq. 4 kernels at this workload's size, graph-timed (a call lasts
+    # microseconds: a CUDA event pair around one call would mostly time the launch)
+    hbm = workload_hbm_kernels(T, torch, stream, B, wl.large.latent_numel, peaks)
+
     # e2e: the same steps through the C ABI with the latent on the host between steps
     x_host.copy_(x_at_window)
     ms_e2e, _, _ = run(idx, lambda i: step_e2e(i, policy))
@@ -716,6 +720,7 @@ def run_window(args):
                             "seconds": sum(b["seconds"] for b in prov.get("batches", [])) or None,
                             "q": [float(v) for v in q], "step_ms": calib_step_ms},
             "kernels": classes,
+            "hbm_kernels": hbm,
             "roofline": roof,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": "steps/s",
@@ -1096,6 +1101,55 @@ def run_forward(args):
 L2_BYTES = 126 * 2 ** 20
 
 
+def graph_rate(T, torch, stream, make_call, bytes_call, resident_bytes, replays, peaks):
+    """Rate of a microsecond-scale HBM kernel: calls recorded back to back in a CUDA
+    graph on `stream`, cycling through enough copies of their buffers (make_call()
+    makes one) to exceed L2 three times; the replay time over the calls."""
+    copies = max(2, math.ceil(3 * L2_BYTES / resident_bytes))
+    fns = [make_call() for _ in range(copies)]
+    for f in fns:
+        f()
+    torch.cuda.synchronize()
+    reps = max(1, math.ceil(60 / copies))
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for _ in range(reps):
+            for f in fns:
+                f()
+    for _ in range(2):
+        g.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(replays):
+        g.replay()
+    e1.record(stream)
+    T.track_sync(stream.cuda_stream)
+    ms = e0.elapsed_time(e1) / (replays * reps * copies)
+    gbs = bytes_call / (ms / 1e3) / 1e9
+    del fns, g
+    torch.cuda.empty_cache()
+    return {"us_per_call": ms * 1e3, "gb_per_s": gbs, "frac_of_hbm": gbs / peaks["hbm_gbs"],
+            "bytes_per_call": bytes_call,
+            "timing": f"CUDA graph of {reps * copies} calls over {copies} buffer sets"}
+
+
+def workload_hbm_kernels(T, torch, stream, B, n, peaks):
+    """The guidance + Euler update (16 B/elem) and Eq. 4 (8 B/elem) at a workload's
+    size (B samples of n latent elements), graph-timed as graph_rate does."""
+    def upd():
+        fc, fu, xx = (torch.randn(B * n, device="cuda") for _ in range(3))
+        return lambda: T.track_cfg_step(xx, fc, fu, 5.0, 0.5, 0.45, stream=stream.cuda_stream)
+
+    def dis():
+        pl, ps = (torch.randn(B, n, device="cuda") for _ in range(2))
+        acc = torch.zeros(B, device="cuda")
+        return lambda: T.track_disagreement(pl, ps, acc, stream=stream.cuda_stream)
+
+    return {"cfg_euler": graph_rate(T, torch, stream, upd, 16.0 * B * n, 12.0 * B * n, 10, peaks),
+            "disagreement": graph_rate(T, torch, stream, dis, 8.0 * B * n, 8.0 * B * n, 10, peaks)}
+
+
 def run_hbm(args, T, torch):
     """The HBM-bound kernels of the C ABI at the sizes the workloads give them, with
     their algorithmic bytes per call: fused guidance + Euler update 16 B/elem (read
@@ -1138,36 +1192,10 @@ def run_hbm(args, T, torch):
                 continue
             nk = B * n480                # latent elements of the step (per model prediction)
             Bk = B if kind not in ("cfg_euler", "multistep") else 1
-            bytes_call = per_elem[kind] * nk
-            copies = max(2, math.ceil(3 * L2_BYTES / (resident[kind] * nk)))
-            fns = [make(kind, nk, Bk) for _ in range(copies)]
-            for f in fns:
-                f()
-            torch.cuda.synchronize()
-            reps = max(1, math.ceil(60 / copies))
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g, stream=stream):
-                for _ in range(reps):
-                    for f in fns:
-                        f()
-            for _ in range(2):
-                g.replay()
-            torch.cuda.synchronize()
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            for _ in range(args.steps):
-                g.replay()
-            e1.record(stream)
-            T.track_sync(stream.cuda_stream)
-            ms = e0.elapsed_time(e1) / (args.steps * reps * copies)
-            gbs = bytes_call / (ms / 1e3) / 1e9
+            rec = graph_rate(T, torch, stream, lambda: make(kind, nk, Bk), per_elem[kind] * nk,
+                             resident[kind] * nk, args.steps, peaks)
             out.append({"kernel": kind, "shape": f"{label}: {nk} elements"
-                        + (f", B={Bk}" if Bk > 1 else ""), "us_per_call": ms * 1e3,
-                        "gb_per_s": gbs, "frac_of_hbm": gbs / peaks["hbm_gbs"],
-                        "timing": f"CUDA graph of {reps * copies} calls over {copies} buffer sets",
-                        "peak_source": src})
-            del fns, g
-            torch.cuda.empty_cache()
+                        + (f", B={Bk}" if Bk > 1 else ""), **rec, "peak_source": src})
     n = 1 << 30
     for kind in ("cfg_euler", "multistep", "disagreement"):
         f = make(kind, n, 8)

@@ -1110,9 +1110,12 @@ __global__ void __launch_bounds__(DIS_THREADS) k_dis_fused(const float* __restri
   if (threadIdx.x == 0) cnt[b] = 0;  // every block has counted in: ready for the next call
 }
 
-int disagreement_blocks(int64_t n_per_sample) {
+int disagreement_blocks(int64_t n_per_sample, int B) {
+  // At most two blocks per SM over all B samples: one wave, each thread with
+  // several float4 loads of both inputs in flight.
   int64_t want = (n_per_sample + DIS_THREADS * 16 - 1) / (DIS_THREADS * 16);
-  const int cap = 2 * num_sms();
+  int cap = 2 * num_sms() / (B > 0 ? B : 1);
+  if (cap < 1) cap = 1;
   if (want < 1) want = 1;
   if (want > cap) want = cap;
   return (int)want;

@@ -170,7 +170,7 @@ cudaError_t band_disagreement(const float* vL, const float* vS, int B, int C, in
                               float eps, float* out, float* scratch, cudaStream_t s);
 
 // Eq. 4: partial sums then a fixed-order final combine; scratch holds B*nblk*2 floats.
-int disagreement_blocks(int64_t n_per_sample);
+int disagreement_blocks(int64_t n_per_sample, int B);
 cudaError_t disagreement(const float* vL, const float* vS, int B, int64_t n, float eps,
                          float* accum, float* scratch, int nblk, cudaStream_t s);
 // The same computation (same bits) in one launch; counters: B ints, zero before

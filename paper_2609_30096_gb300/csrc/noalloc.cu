@@ -77,7 +77,7 @@ extern "C" int track_disagreement_static(const float* v_L, const float* v_S, int
   }
   // Same partition as track_disagreement (so both give the same bits), capped
   // by the array's size.
-  int64_t nblk = disagreement_blocks(n_per_sample);
+  int64_t nblk = disagreement_blocks(n_per_sample, B);
   if (nblk > kMaxBlocks) nblk = kMaxBlocks;
   // Every partial slot the reduction reads is written earlier in the same call,
   // so nothing needs clearing between calls.

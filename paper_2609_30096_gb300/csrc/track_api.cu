@@ -801,7 +801,7 @@ static int* dis_counters(cudaStream_t s, int B) {
 
 static int disagreement_impl(const float* vL, const float* vS, int B, int64_t n, float eps,
                              float* accum, cudaStream_t s) {
-  const int nblk = disagreement_blocks(n);
+  const int nblk = disagreement_blocks(n, B);
   float* scr = stream_scratch(s, (size_t)B * nblk * 2);
   if (scr == nullptr) return fail(TRACK_ENOMEM, "disagreement scratch allocation failed");
   int* cnt = dis_counters(s, B);
