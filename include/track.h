@@ -370,8 +370,7 @@ int track_gemm_schedule(int mode);
  * varying fastest inside a group, then the 128-to-256-column tile.  The tiles
  * running at one time then share few A and W blocks, which stay in L2 while
  * they are reused.  A group at least as large as the row-unit count is plain
- * column order.  0 restores the default: column order for outputs of at most
- * 32 column tiles, groups of 32 above.  Data-parallel results do not depend
+ * column order.  0 restores the default, groups of 32.  Data-parallel results do not depend
  * on the order; under stream-K it moves the split points between tiles (fp32
  * rounding only).  EINVAL outside 0..65536. */
 int track_gemm_raster(int group);

@@ -1005,19 +1005,22 @@ __device__ __forceinline__ void dis_block_partials(const float* __restrict__ l,
     const int64_t n4 = n / 4;
     const float4* l4 = reinterpret_cast<const float4*>(l);
     const float4* s4 = reinterpret_cast<const float4*>(sp);
-    int64_t i = blk * (int64_t)DIS_THREADS + threadIdx.x;
-    // every load of a group is issued before the group is summed (in index order)
-    for (; i + (DIS_UNROLL - 1) * stride < n4; i += DIS_UNROLL * stride) {
+    // Every load of a group of DIS_UNROLL strided float4 pairs is issued before the
+    // group is summed (in index order); slots past the end read as zeros, which
+    // leave the sums unchanged (fma(0, 0, s) = s), so a thread's last, partial
+    // group costs one memory latency like the others.
+    const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int64_t i = blk * (int64_t)DIS_THREADS + threadIdx.x; i < n4; i += DIS_UNROLL * stride) {
       float4 a[DIS_UNROLL], c[DIS_UNROLL];
 #pragma unroll
       for (int u = 0; u < DIS_UNROLL; ++u) {
-        a[u] = l4[i + u * stride];
-        c[u] = s4[i + u * stride];
+        const int64_t k = i + u * stride;
+        a[u] = k < n4 ? l4[k] : z;
+        c[u] = k < n4 ? s4[k] : z;
       }
 #pragma unroll
       for (int u = 0; u < DIS_UNROLL; ++u) acc4(a[u], c[u]);
     }
-    for (; i < n4; i += stride) acc4(l4[i], s4[i]);
     i0 = n4 * 4;
   }
   for (int64_t i = i0 + blk * (int64_t)DIS_THREADS + threadIdx.x; i < n; i += stride) {
@@ -1100,12 +1103,15 @@ __global__ void __launch_bounds__(DIS_THREADS) k_dis_fused(const float* __restri
   if (threadIdx.x == 0) {
     part[((int64_t)b * nblk + blockIdx.x) * 2 + 0] = td;
     part[((int64_t)b * nblk + blockIdx.x) * 2 + 1] = tl;
-    __threadfence();  // the partials are visible before this block counts in
-    last = atomicAdd(cnt + b, 1) == nblk - 1 ? 1 : 0;
+    // Release: the partials are visible before this block counts in; acquire:
+    // the last block sees every other block's partials.
+    int prev;
+    asm volatile("atom.add.acq_rel.gpu.global.s32 %0, [%1], 1;" : "=r"(prev) : "l"(cnt + b) : "memory");
+    last = prev == nblk - 1 ? 1 : 0;
   }
   __syncthreads();
   if (!last) return;
-  __threadfence();  // every other block's partials are visible to the loads below
+  __threadfence();  // the acquire of thread 0 extends to the block's loads below
   dis_combine(part, nblk, b, eps, accum);
   if (threadIdx.x == 0) cnt[b] = 0;  // every block has counted in: ready for the next call
 }

@@ -93,12 +93,11 @@ constexpr double SK_FIXUP = 10000.0;
 // reused, instead of one column of up to all row units, which streams all of A
 // from DRAM once per column tile when A is larger than L2.  With at most
 // `group` row units (3510 tokens: 28) this is the plain column order.
-// Measured at 32760 rows and K 5120 (14B shapes): groups of 32 made the FFN
-// up-projection (54 column tiles) 21 % faster than column order, but the 20-
-// column-tile projections 20-30 % slower; the default therefore keeps column
-// order up to RASTER_NARROW column tiles and groups of 32 above.
+// Measured at 65520 rows (the 14B shapes with CFG): groups of 32 made every
+// projection 13-25 % faster than column order (qkv 1813, out_proj 1542,
+// cross_q 1623, ffn_up 1610, ffn_down 1534 TFLOP/s), and were the best or
+// within 1 % of the best of 4, 8, 16, 32 and 64.
 constexpr int RASTER_DEFAULT = 32;
-constexpr int RASTER_NARROW = 32;
 
 __device__ __forceinline__ void tile_coords(int tile, int m_units, int n_tiles, int group, int& mu,
                                             int& nt) {
@@ -585,7 +584,7 @@ cudaError_t launch_tc(const void* A, const void* W, const GemmArgs& g_in, bool s
   using S = TcShape<BN, STAGES>;
   GemmArgs g = g_in;
   g.raster = g_gemm_raster.load();
-  if (g.raster <= 0) g.raster = (g.N + BN - 1) / BN <= RASTER_NARROW ? (1 << 30) : RASTER_DEFAULT;
+  if (g.raster <= 0) g.raster = RASTER_DEFAULT;
   static_assert(S::SMEM <= 232448, "shared memory budget");
   CUtensorMap ta, tb, tc;
   const CUtensorMapDataType BF = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
