@@ -658,6 +658,18 @@ def run_window(args):
     ms_e2e, _, _ = run(idx, lambda i: step_e2e(i, policy))
     e2e_value = world * B * args.steps / (ms_e2e / 1e3)
 
+    # without the whole trajectories: the same number of steps of the all-large
+    # trajectory from the window's first step, for the routed / all-large ratio
+    all_large_window = None
+    if args.no_trajectories:
+        xa = x_at_window.clone()
+        ms_al, _, _ = run(idx, lambda i: step(i, all_l, xa))
+        del xa
+        all_large_window = {"steps_per_s": world * B * args.steps / (ms_al / 1e3),
+                            "ms_per_step": ms_al / args.steps,
+                            "routed_speedup": ms_al / ms,
+                            "note": "the timed window's steps run with the large model only"}
+
     # whole trajectories, end to end (text projection included): routed and all-large
     traj = {}
     if not args.no_trajectories:
@@ -716,6 +728,7 @@ def run_window(args):
                        "launch": "eager, one track_sample call per step"},
             "dit_tflops": tflops, "dit_frac_of_sustained": tflops / peaks["bf16_tflops_sustained"],
             "trajectory": traj or None,
+            "all_large_window": all_large_window,
             "calibration": {"score_map": os.path.relpath(score_map_path(wl), ROOT), "seeds": M,
                             "seconds": sum(b["seconds"] for b in prov.get("batches", [])) or None,
                             "q": [float(v) for v in q], "step_ms": calib_step_ms},
@@ -1146,8 +1159,16 @@ def workload_hbm_kernels(T, torch, stream, B, n, peaks):
         acc = torch.zeros(B, device="cuda")
         return lambda: T.track_disagreement(pl, ps, acc, stream=stream.cuda_stream)
 
+    def dis_upd():
+        pl, ps, xx = (torch.randn(B, n, device="cuda") for _ in range(3))
+        acc = torch.zeros(B, device="cuda")
+        return lambda: T.track_disagreement_update(pl, ps, acc, xx, 0.5, 0.45,
+                                                   stream=stream.cuda_stream)
+
     return {"cfg_euler": graph_rate(T, torch, stream, upd, 16.0 * B * n, 12.0 * B * n, 10, peaks),
-            "disagreement": graph_rate(T, torch, stream, dis, 8.0 * B * n, 8.0 * B * n, 10, peaks)}
+            "disagreement": graph_rate(T, torch, stream, dis, 8.0 * B * n, 8.0 * B * n, 10, peaks),
+            "disagreement_update": graph_rate(T, torch, stream, dis_upd, 16.0 * B * n,
+                                              12.0 * B * n, 10, peaks)}
 
 
 def run_hbm(args, T, torch):
@@ -1177,17 +1198,22 @@ def run_hbm(args, T, torch):
         if kind == "disagreement":
             acc = torch.zeros(B, device="cuda")
             return lambda: T.track_disagreement(fc.view(B, -1), fu.view(B, -1), acc)
+        if kind == "disagreement_update":
+            acc = torch.zeros(B, device="cuda")
+            return lambda: T.track_disagreement_update(fc.view(B, -1), fu.view(B, -1), acc,
+                                                       xx.view(B, -1), 0.5, 0.45)
         bo = torch.empty(B, 6, device="cuda")
         bl, bs = fc.view(B, 16, 21, 60, 104), fu.view(B, 16, 21, 60, 104)
         return lambda: T.track_band_disagreement(bl, bs, out=bo)
 
-    per_elem = {"cfg_euler": 16.0, "multistep": 28.0, "disagreement": 8.0, "band_split": 8.0}
+    per_elem = {"cfg_euler": 16.0, "multistep": 28.0, "disagreement": 8.0,
+                "disagreement_update": 16.0, "band_split": 8.0}
     resident = {"cfg_euler": 12.0, "multistep": 28.0, "disagreement": 12.0,
-                "band_split": 12.0}   # bytes allocated per element
+                "disagreement_update": 12.0, "band_split": 12.0}   # bytes allocated per element
     out = []
     for label, B in (("one 480p request (latent 16x21x60x104)", 1),
                      ("serving batch of 4 480p requests", 4)):
-        for kind in ("cfg_euler", "multistep", "disagreement", "band_split"):
+        for kind in ("cfg_euler", "multistep", "disagreement", "disagreement_update", "band_split"):
             if kind == "band_split" and B != 1:
                 continue
             nk = B * n480                # latent elements of the step (per model prediction)
@@ -1197,7 +1223,7 @@ def run_hbm(args, T, torch):
             out.append({"kernel": kind, "shape": f"{label}: {nk} elements"
                         + (f", B={Bk}" if Bk > 1 else ""), **rec, "peak_source": src})
     n = 1 << 30
-    for kind in ("cfg_euler", "multistep", "disagreement"):
+    for kind in ("cfg_euler", "multistep", "disagreement", "disagreement_update"):
         f = make(kind, n, 8)
         for _ in range(args.warmup):
             f()
@@ -1210,7 +1236,7 @@ def run_hbm(args, T, torch):
         T.track_sync(stream.cuda_stream)
         ms = e0.elapsed_time(e1) / args.steps
         gbs = per_elem[kind] * n / (ms / 1e3) / 1e9
-        out.append({"kernel": kind, "shape": f"1 Gi elements{', B=8' if kind == 'disagreement' else ''}",
+        out.append({"kernel": kind, "shape": f"1 Gi elements{', B=8' if 'disagree' in kind else ''}",
                     "us_per_call": ms * 1e3, "gb_per_s": gbs, "frac_of_hbm": gbs / peaks["hbm_gbs"],
                     "timing": "eager launches", "peak_source": src})
         del f

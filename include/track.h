@@ -221,6 +221,17 @@ int track_cfg_step(float* x, const float* f_c, const float* f_u, int64_t n, floa
 int track_disagreement(const float* v_L, const float* v_S, int B, int64_t n_per_sample,
                        float eps, float* score_accum, track_stream s);
 
+/* One step of the calibration trajectory after both predictions (Sec. 3.2.1):
+ * adds Eq. 4's r_b of (v_L, v_S) to score_accum[b] exactly as
+ * track_disagreement does (same bits), and advances the trajectory by the large
+ * model's prediction, x[b] += (sigma_next - sigma_t) * v_L[b] (Eq. 2, Euler,
+ * the bits of track_step), in one pass that reads v_L once for both.
+ * x: device fp32 [B, n_per_sample], in/out, must not overlap v_L or v_S
+ * (EINVAL).  Same scratch, stream and determinism rules as track_disagreement. */
+int track_disagreement_update(const float* v_L, const float* v_S, int B, int64_t n_per_sample,
+                              float eps, float* score_accum, float* x, float sigma_t,
+                              float sigma_next, track_stream s);
+
 /* Eq. 5 on the host: q[k] = (1/M) sum_j r[j*N + k] (r host [M, N]), summed in j
  * order in double and rounded to float. */
 int track_mean_score(const float* r, int M, int N, float* q_out);

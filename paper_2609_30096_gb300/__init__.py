@@ -83,6 +83,7 @@ def lib():
         "track_step": (_I, [_P, _P, _L, _F, _F, _P]),
         "track_cfg_step": (_I, [_P, _P, _P, _L, _F, _F, _F, _P]),
         "track_disagreement": (_I, [_P, _P, _I, _L, _F, _P, _P]),
+        "track_disagreement_update": (_I, [_P, _P, _I, _L, _F, _P, _P, _F, _F, _P]),
         "track_disagreement_static": (_I, [_P, _P, _I, _L, _F, _P, _P]),
         "track_mean_score": (_I, [_P, _I, _I, _P]),
         "track_policy_topk": (_I, [_P, _I, _I, _P]),
@@ -329,6 +330,17 @@ def track_disagreement(v_L, v_S, score_accum, eps=1e-8, stream=None):
     B = v_L.shape[0]
     _check(lib().track_disagreement(_ptr(v_L), _ptr(v_S), B, v_L.numel() // B, eps,
                                     _ptr(score_accum), _stream(stream)))
+    return score_accum
+
+
+def track_disagreement_update(v_L, v_S, score_accum, x, sigma_t, sigma_next, eps=1e-8,
+                              stream=None):
+    """Eq. 4 into score_accum and the calibration trajectory's Euler update
+    x += (sigma_next - sigma_t) * v_L, in one pass (x: same shape as v_L)."""
+    B = v_L.shape[0]
+    _check(lib().track_disagreement_update(_ptr(v_L), _ptr(v_S), B, v_L.numel() // B, eps,
+                                           _ptr(score_accum), _ptr(x), float(sigma_t),
+                                           float(sigma_next), _stream(stream)))
     return score_accum
 
 

@@ -960,7 +960,9 @@ cudaError_t multistep_step(float* x, const float* v, float* xc, float* vp, int64
 // last for sample b (a per-sample counter, which that block resets) adds
 // them.  k_dis_partial + k_dis_final do it in two launches (the
 // allocation-free entry point, whose fixed array holds no counters).  Both
-// compute the same bits.
+// compute the same bits.  k_dis_fused<true> also advances the latent of the
+// calibration trajectory by the large model's prediction (Eq. 2, Euler) in
+// the same pass, x += dsig * vL, reading each element of vL once for both.
 constexpr int DIS_THREADS = 512;
 constexpr int DIS_UNROLL = 4;
 
@@ -986,13 +988,15 @@ __device__ __forceinline__ void block_sum2(float& a, float& b, float* red) {
   b = tb;
 }
 
+template <bool UPD>
 __device__ __forceinline__ void dis_block_partials(const float* __restrict__ l,
-                                                   const float* __restrict__ sp, int64_t n,
+                                                   const float* __restrict__ sp,
+                                                   float* __restrict__ x, float dsig, int64_t n,
                                                    int blk, int nblk, float* red, float& td,
                                                    float& tl) {
   float sd = 0.f, sl = 0.f;
   const int64_t stride = (int64_t)nblk * DIS_THREADS;
-  const bool vec = ((((uintptr_t)l) | ((uintptr_t)sp)) & 15) == 0;
+  const bool vec = ((((uintptr_t)l) | ((uintptr_t)sp) | (UPD ? (uintptr_t)x : 0)) & 15) == 0;
   int64_t i0 = 0;
   auto acc4 = [&](const float4& a, const float4& c) {
     float t;
@@ -1010,58 +1014,102 @@ __device__ __forceinline__ void dis_block_partials(const float* __restrict__ l,
     // leave the sums unchanged (fma(0, 0, s) = s), so a thread's last, partial
     // group costs one memory latency like the others.
     const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+    float4* x4 = reinterpret_cast<float4*>(x);
     for (int64_t i = blk * (int64_t)DIS_THREADS + threadIdx.x; i < n4; i += DIS_UNROLL * stride) {
-      float4 a[DIS_UNROLL], c[DIS_UNROLL];
+      float4 a[DIS_UNROLL], c[DIS_UNROLL], xv[DIS_UNROLL];
 #pragma unroll
       for (int u = 0; u < DIS_UNROLL; ++u) {
         const int64_t k = i + u * stride;
         a[u] = k < n4 ? l4[k] : z;
         c[u] = k < n4 ? s4[k] : z;
+        if (UPD) xv[u] = k < n4 ? x4[k] : z;
       }
 #pragma unroll
       for (int u = 0; u < DIS_UNROLL; ++u) acc4(a[u], c[u]);
+      if (UPD) {
+#pragma unroll
+        for (int u = 0; u < DIS_UNROLL; ++u) {
+          const int64_t k = i + u * stride;
+          if (k < n4)
+            x4[k] = make_float4(euler_val(xv[u].x, a[u].x, dsig), euler_val(xv[u].y, a[u].y, dsig),
+                                euler_val(xv[u].z, a[u].z, dsig), euler_val(xv[u].w, a[u].w, dsig));
+        }
+      }
     }
     i0 = n4 * 4;
   }
   for (int64_t i = i0 + blk * (int64_t)DIS_THREADS + threadIdx.x; i < n; i += stride) {
-    const float t = sp[i] - l[i];
+    const float li = l[i];
+    const float t = sp[i] - li;
     sd = fmaf(t, t, sd);
-    sl = fmaf(l[i], l[i], sl);
+    sl = fmaf(li, li, sl);
+    if (UPD) x[i] = euler_val(x[i], li, dsig);
   }
   block_sum2(sd, sl, red);
   td = sd;
   tl = sl;
 }
 
-// Adds sample b's nblk partials in a fixed order in fp64 (all DIS_THREADS
-// threads of the block: strided per-thread sums, warp shuffles, then thread 0
-// adds the warps' sums in order), then accum[b] += r_b (thread 0).
+// Compensated fp32 ("double-float") addition: (h, l) += (bh, bl), where each
+// pair stands for the unevaluated sum h + l with |l| <= ulp(h) / 2.  The
+// rounding error of h + bh is recovered exactly by Knuth's TwoSum, added to the
+// low parts, and the result renormalized by Dekker's FastTwoSum.  About 48
+// significant bits, on the FP32 pipe.  Commutative bit for bit (TwoSum's error
+// term is exact whichever operand comes first).
+__device__ __forceinline__ void df_add(float& h, float& l, float bh, float bl) {
+  const float s = __fadd_rn(h, bh);
+  const float bb = __fsub_rn(s, h);
+  const float e = __fadd_rn(__fsub_rn(h, __fsub_rn(s, bb)), __fsub_rn(bh, bb));
+  const float t = __fadd_rn(__fadd_rn(l, bl), e);
+  h = __fadd_rn(s, t);
+  l = __fsub_rn(t, __fsub_rn(h, s));
+}
+
+// Adds sample b's nblk partials in a fixed order with double-float sums (all
+// DIS_THREADS threads of the block: strided per-thread sums, warp shuffles,
+// then warp 0 adds the warps' sums by shuffles), then accum[b] += r_b (thread
+// 0, IEEE sqrt and division in fp32).  The combine runs on one SM after every
+// other block has finished, so it avoids fp64 arithmetic, whose rate on this
+// GPU made a double-precision combine the longest part of the launch.
 __device__ __forceinline__ void dis_combine(const float* part, int nblk, int b, float eps,
                                             float* accum) {
-  __shared__ double rd[DIS_THREADS / 32], rl[DIS_THREADS / 32];
-  double sd = 0.0, sl = 0.0;
+  __shared__ float rs[4][DIS_THREADS / 32];
+  float dh = 0.f, dl = 0.f, lh = 0.f, ll = 0.f;
   for (int j = threadIdx.x; j < nblk; j += DIS_THREADS) {
     const float2 v = __ldcg(reinterpret_cast<const float2*>(part) + (int64_t)b * nblk + j);
-    sd += (double)v.x;
-    sl += (double)v.y;
+    df_add(dh, dl, v.x, 0.f);
+    df_add(lh, ll, v.y, 0.f);
   }
   for (int o = 16; o > 0; o >>= 1) {
-    sd += __shfl_xor_sync(0xffffffffu, sd, o);
-    sl += __shfl_xor_sync(0xffffffffu, sl, o);
+    const float a = __shfl_xor_sync(0xffffffffu, dh, o), c = __shfl_xor_sync(0xffffffffu, dl, o);
+    const float e = __shfl_xor_sync(0xffffffffu, lh, o), f = __shfl_xor_sync(0xffffffffu, ll, o);
+    df_add(dh, dl, a, c);
+    df_add(lh, ll, e, f);
   }
-  if ((threadIdx.x & 31) == 0) {
-    rd[threadIdx.x >> 5] = sd;
-    rl[threadIdx.x >> 5] = sl;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) {
+    rs[0][w] = dh;
+    rs[1][w] = dl;
+    rs[2][w] = lh;
+    rs[3][w] = ll;
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    double td = 0.0, tl = 0.0;
-    for (int i = 0; i < DIS_THREADS / 32; ++i) {
-      td += rd[i];
-      tl += rl[i];
+  if (w == 0) {
+    constexpr int NW = DIS_THREADS / 32;
+    dh = lane < NW ? rs[0][lane] : 0.f;
+    dl = lane < NW ? rs[1][lane] : 0.f;
+    lh = lane < NW ? rs[2][lane] : 0.f;
+    ll = lane < NW ? rs[3][lane] : 0.f;
+    for (int o = NW / 2; o > 0; o >>= 1) {
+      const float a = __shfl_xor_sync(0xffffffffu, dh, o), c = __shfl_xor_sync(0xffffffffu, dl, o);
+      const float e = __shfl_xor_sync(0xffffffffu, lh, o), f = __shfl_xor_sync(0xffffffffu, ll, o);
+      df_add(dh, dl, a, c);
+      df_add(lh, ll, e, f);
     }
-    const double den = fmax(sqrt(tl), (double)eps);
-    accum[b] += (float)(sqrt(td) / den);
+    if (lane == 0) {
+      const float den = fmaxf(__fsqrt_rn(__fadd_rn(lh, ll)), eps);
+      accum[b] = __fadd_rn(accum[b], __fdiv_rn(__fsqrt_rn(__fadd_rn(dh, dl)), den));
+    }
   }
 }
 
@@ -1073,7 +1121,8 @@ __global__ void __launch_bounds__(DIS_THREADS) k_dis_partial(const float* __rest
   __shared__ float red[64];
   const int b = blockIdx.y, nblk = gridDim.x;
   float td, tl;
-  dis_block_partials(vL + (int64_t)b * n, vS + (int64_t)b * n, n, blockIdx.x, nblk, red, td, tl);
+  dis_block_partials<false>(vL + (int64_t)b * n, vS + (int64_t)b * n, nullptr, 0.f, n,
+                            blockIdx.x, nblk, red, td, tl);
   if (threadIdx.x == 0) {
     part[((int64_t)b * nblk + blockIdx.x) * 2 + 0] = td;
     part[((int64_t)b * nblk + blockIdx.x) * 2 + 1] = tl;
@@ -1088,18 +1137,22 @@ __global__ void __launch_bounds__(DIS_THREADS) k_dis_final(const float* __restri
   dis_combine(part, nblk, blockIdx.x, eps, accum);
 }
 
+template <bool UPD>
 __global__ void __launch_bounds__(DIS_THREADS) k_dis_fused(const float* __restrict__ vL,
                                                            const float* __restrict__ vS, int64_t n,
                                                            float* __restrict__ part,
                                                            int* __restrict__ cnt, float eps,
-                                                           float* __restrict__ accum) {
+                                                           float* __restrict__ accum,
+                                                           float* __restrict__ x, float dsig) {
   pdl_wait();
   pdl_release();
   __shared__ float red[64];
   __shared__ int last;
   const int b = blockIdx.y, nblk = gridDim.x;
   float td, tl;
-  dis_block_partials(vL + (int64_t)b * n, vS + (int64_t)b * n, n, blockIdx.x, nblk, red, td, tl);
+  dis_block_partials<UPD>(vL + (int64_t)b * n, vS + (int64_t)b * n,
+                          UPD ? x + (int64_t)b * n : nullptr, dsig, n, blockIdx.x, nblk, red, td,
+                          tl);
   if (threadIdx.x == 0) {
     part[((int64_t)b * nblk + blockIdx.x) * 2 + 0] = td;
     part[((int64_t)b * nblk + blockIdx.x) * 2 + 1] = tl;
@@ -1119,7 +1172,7 @@ __global__ void __launch_bounds__(DIS_THREADS) k_dis_fused(const float* __restri
 int disagreement_blocks(int64_t n_per_sample, int B) {
   // At most two blocks per SM over all B samples: one wave, each thread with
   // several float4 loads of both inputs in flight.
-  int64_t want = (n_per_sample + DIS_THREADS * 16 - 1) / (DIS_THREADS * 16);
+  int64_t want = (n_per_sample + DIS_THREADS * 8 - 1) / (DIS_THREADS * 8);
   int cap = 2 * num_sms() / (B > 0 ? B : 1);
   if (cap < 1) cap = 1;
   if (want < 1) want = 1;
@@ -1140,10 +1193,14 @@ cudaError_t disagreement(const float* vL, const float* vS, int B, int64_t n, flo
 
 cudaError_t disagreement_fused(const float* vL, const float* vS, int B, int64_t n, float eps,
                                float* accum, float* scratch, int* counters, int nblk,
-                               cudaStream_t s) {
+                               cudaStream_t s, float* x, float dsig) {
   if (B <= 0) return cudaSuccess;
-  cudaError_t e = launch_pdl(k_dis_fused, dim3(nblk, B), DIS_THREADS, 0, s, vL, vS, n, scratch,
-                             counters, eps, accum);
+  cudaError_t e =
+      x != nullptr
+          ? launch_pdl(k_dis_fused<true>, dim3(nblk, B), DIS_THREADS, 0, s, vL, vS, n, scratch,
+                       counters, eps, accum, x, dsig)
+          : launch_pdl(k_dis_fused<false>, dim3(nblk, B), DIS_THREADS, 0, s, vL, vS, n, scratch,
+                       counters, eps, accum, (float*)nullptr, 0.f);
   if (e != cudaSuccess) return e;
   count_launch();
   return cudaGetLastError();

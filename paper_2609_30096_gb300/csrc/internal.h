@@ -174,10 +174,11 @@ int disagreement_blocks(int64_t n_per_sample, int B);
 cudaError_t disagreement(const float* vL, const float* vS, int B, int64_t n, float eps,
                          float* accum, float* scratch, int nblk, cudaStream_t s);
 // The same computation (same bits) in one launch; counters: B ints, zero before
-// the call, left at zero by it.
+// the call, left at zero by it.  With x non-null the same pass also applies the
+// Euler update x[b] += dsig * vL[b] (x must not alias vL or vS).
 cudaError_t disagreement_fused(const float* vL, const float* vS, int B, int64_t n, float eps,
                                float* accum, float* scratch, int* counters, int nblk,
-                               cudaStream_t s);
+                               cudaStream_t s, float* x = nullptr, float dsig = 0.f);
 
 int num_sms();
 

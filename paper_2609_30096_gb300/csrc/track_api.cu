@@ -799,15 +799,18 @@ static int* dis_counters(cudaStream_t s, int B) {
   return p;
 }
 
+// Eq. 4 into accum; with x non-null also x += dsig * vL (Euler, Eq. 2) in the
+// same pass.
 static int disagreement_impl(const float* vL, const float* vS, int B, int64_t n, float eps,
-                             float* accum, cudaStream_t s) {
+                             float* accum, cudaStream_t s, float* x = nullptr, float dsig = 0.f) {
   const int nblk = disagreement_blocks(n, B);
   float* scr = stream_scratch(s, (size_t)B * nblk * 2);
   if (scr == nullptr) return fail(TRACK_ENOMEM, "disagreement scratch allocation failed");
   int* cnt = dis_counters(s, B);
   if (cnt == nullptr) return fail(TRACK_ENOMEM, "disagreement counter allocation failed");
-  ProfScope ps(PROF_DIS, 8.0 * B * (double)n, s);  // read p_L, p_S
-  LAUNCH(disagreement_fused(vL, vS, B, n, eps, accum, scr, cnt, nblk, s));
+  // read p_L, p_S (and x, written back)
+  ProfScope ps(PROF_DIS, (x != nullptr ? 16.0 : 8.0) * B * (double)n, s);
+  LAUNCH(disagreement_fused(vL, vS, B, n, eps, accum, scr, cnt, nblk, s, x, dsig));
   return TRACK_OK;
 }
 
@@ -1118,6 +1121,21 @@ int track_disagreement(const float* v_L, const float* v_S, int B, int64_t n_per_
   return disagreement_impl(v_L, v_S, B, n_per_sample, eps, score_accum, (cudaStream_t)s);
 }
 
+int track_disagreement_update(const float* v_L, const float* v_S, int B, int64_t n_per_sample,
+                              float eps, float* score_accum, float* x, float sigma_t,
+                              float sigma_next, track_stream s) {
+  if (!v_L || !v_S || !score_accum || !x || B < 0 || n_per_sample <= 0 || !(eps > 0.f))
+    return fail(TRACK_EINVAL, "bad arguments");
+  if (B == 0) return TRACK_OK;
+  const uintptr_t xb = (uintptr_t)x, xe = xb + (uintptr_t)B * n_per_sample * sizeof(float);
+  for (const float* v : {v_L, v_S}) {
+    const uintptr_t vb = (uintptr_t)v, ve = vb + (uintptr_t)B * n_per_sample * sizeof(float);
+    if (xb < ve && vb < xe) return fail(TRACK_EINVAL, "x overlaps v_L or v_S");
+  }
+  return disagreement_impl(v_L, v_S, B, n_per_sample, eps, score_accum, (cudaStream_t)s, x,
+                           sigma_next - sigma_t);
+}
+
 int track_mean_score(const float* r, int M, int N, float* q_out) {
   if (!r || !q_out || M < 1 || N < 1) return fail(TRACK_EINVAL, "bad arguments");
   for (int k = 0; k < N; ++k) {
@@ -1273,9 +1291,9 @@ int track_calibrate(track_model* large, track_model* small, float* x, int B, con
     const float t = 1000.f * sigmas[k];
     TRACK_TRY(denoise_impl(large, x, B, t, cond, uncond, cfg_scale, pL, st));
     TRACK_TRY(denoise_impl(small, x, B, t, cond, uncond, cfg_scale, pS, st));
-    TRACK_TRY(disagreement_impl(pL, pS, B, n, eps, r_out + (size_t)k * B, st));
-    ProfScope ps(PROF_UPDATE, 12.0 * B * (double)n, st);  // read x, p_L; write x
-    LAUNCH(euler_step(x, pL, (int64_t)B * n, sigmas[k + 1] - sigmas[k], st));
+    // Eq. 4 and the trajectory's Euler update by p_L in one pass
+    TRACK_TRY(disagreement_impl(pL, pS, B, n, eps, r_out + (size_t)k * B, st, x,
+                                sigmas[k + 1] - sigmas[k]));
   }
   return TRACK_OK;
 }

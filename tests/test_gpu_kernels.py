@@ -477,6 +477,38 @@ def test_disagreement_one_launch_equals_two_launches(T, B, n):
         assert torch.equal(one, two)
 
 
+@pytest.mark.parametrize("B,n", [(1, 3), (2, 4097), (1, 2_096_640), (3, 2_096_641),
+                                 (4, 2_096_640)])
+def test_disagreement_update_equals_separate_calls(T, B, n):
+    # Calibration's per-step call: Eq. 4 and the Euler update of the trajectory by
+    # p_L in one pass.  Its score must have the bits of track_disagreement and its
+    # latent those of track_step, call after call; both also against the oracle.
+    rng = np.random.default_rng(7 * B + n)
+    pl = rng.normal(size=(B, n)).astype(np.float32)
+    ps = (pl + 0.2 * rng.normal(size=(B, n))).astype(np.float32)
+    x = rng.normal(size=(B, n)).astype(np.float32)
+    s0, s1 = 0.8333333, 0.625
+    pld, psd = dev_f32(pl), dev_f32(ps)
+    xa, xb = dev_f32(x), dev_f32(x)
+    acc_a = torch.full((B,), 0.5, device=DEV)
+    acc_b = torch.full((B,), 0.5, device=DEV)
+    for _ in range(2):
+        T.track_disagreement(pld, psd, acc_a)
+        T.track_step(xa, pld, s0, s1)
+        T.track_disagreement_update(pld, psd, acc_b, xb, s0, s1)
+        T.track_sync()
+        assert torch.equal(acc_a, acc_b)
+        assert torch.equal(xa, xb)
+    ref_r = [track.disagreement(pl[b], ps[b]) for b in range(B)]
+    assert np.max(np.abs((acc_b.cpu().numpy() - 0.5) / 2 - ref_r)) < 1e-5
+    ref_x = x
+    for _ in range(2):
+        ref_x = track.euler_update(ref_x, pl, np.float32(s0), np.float32(s1))
+    assert rel_l2(xb.cpu().numpy(), ref_x) < 1e-6
+    with pytest.raises(T.TrackError):
+        T.track_disagreement_update(pld, psd, acc_b, pld, s0, s1)  # x aliases p_L
+
+
 def test_disagreement_special_cases(T):
     pl = np.random.default_rng(1).normal(size=(2, 1000)).astype(np.float32)
     acc = torch.zeros(2, device=DEV)
