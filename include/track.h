@@ -119,7 +119,8 @@ int track_fail_next_allocations(int n);
  * track_sample are bracketed by CUDA events on their stream.
  * track_profile_read synchronizes those events and returns, per class (0 =
  * GEMM, 1 = self-attention, 2 = LayerNorm-modulate, 3 = RMSNorm of q/k with
- * RoPE, 4 = guidance combine and scheduler update, 5 = Eq. 4 reduction, 6 =
+ * RoPE, 4 = guidance combine and scheduler update, 5 = Eq. 4 reduction (in
+ * track_calibrate fused with the trajectory's Euler update), 6 =
  * cross-attention), the summed event time in ms, the summed algorithmic work
  * (FLOPs for classes 0, 1 and 6, bytes moved for the others) and the number of launches, then clears the
  * records.  Arrays are host, length TRACK_PROFILE_CLASSES.  In a graph
