@@ -302,11 +302,12 @@ def block_flops(arch, tokens):
 class OracleSample:
     """The oracle on a bounded sample of the workload: one DiT block of each model
     (fp64 numpy) over the first `frames` latent frames of the workload's latent
-    (all of them when frames is None), timed and extrapolated to one full-size
-    forward of one sequence by algorithmic FLOPs (block FLOPs at the full token
-    count over those at the sample's) times the model's depth."""
+    (all of them when frames is None), or over the first `rows` token rows of
+    its first frame, timed and extrapolated to one full-size forward of one
+    sequence by algorithmic FLOPs (block FLOPs at the full token count over
+    those at the sample's) times the model's depth."""
 
-    def __init__(self, wl, frames=None):
+    def __init__(self, wl, frames=None, rows=None):
         from oracle import dit
 
         self.wl = wl
@@ -315,7 +316,10 @@ class OracleSample:
         for which, arch, seed in (("large", wl.large, synth.SEED_LARGE),
                                   ("small", wl.small, synth.SEED_SMALL)):
             f = arch.frames if frames is None else min(frames, arch.frames)
-            sample = synth.Arch(**{**arch.__dict__, "layers": 1, "frames": f})
+            if rows is not None:
+                f = 1
+            hgt = arch.height if rows is None else min(arch.height, 2 * rows)
+            sample = synth.Arch(**{**arch.__dict__, "layers": 1, "frames": f, "height": hgt})
             specs = [s for s in synth.weight_specs(arch)
                      if not s.name.startswith("blk") or s.name.startswith("blk0.")]
             w = {s.name: synth.make_tensor(s, seed) for s in specs}
@@ -392,7 +396,9 @@ def run_reference(args):
         idx = window_steps(wl.steps, timed_window(pol, args.warmup, args.steps), args.steps)
         n_small = int(sum(int(pol[i]) for i in idx))
         mix = (args.steps - n_small, n_small)
-        sampler = OracleSample(wl, frames=1)
+        # warm-up + timed steps each run a sample: 8 token rows of the first frame
+        # (416 tokens at 480p) keep the whole run to a few minutes on the host
+        sampler = OracleSample(wl, rows=8)
     else:
         pol = None
         n_small = wl.k
