@@ -198,3 +198,25 @@ def test_score_map_rejects_bad_files_and_scores(T, tmp_path):
         assert e.value.code == T.TRACK_EINVAL
     with pytest.raises(T.TrackError):
         T.track_score_map_save(tmp_path / "no_such_dir" / "x.trk", r)
+
+
+def test_disagreement_update_checks_arguments_on_the_host(T):
+    # Host-side checks only: every call below is rejected before anything is
+    # launched, so the addresses are never dereferenced.
+    lib = T.lib()
+    n, B = 1024, 2
+    base = 1 << 30                                   # stand-in addresses, 16-byte aligned
+    vL, vS, acc = base, base + 4 * B * n, base + 8 * B * n
+    x_ok = base + 16 * B * n
+    cases = [
+        (0, vS, B, n, 1e-8, acc, x_ok),              # NULL v_L
+        (vL, vS, B, n, 1e-8, acc, 0),                # NULL x
+        (vL, vS, B, 0, 1e-8, acc, x_ok),             # empty samples
+        (vL, vS, B, n, 0.0, acc, x_ok),              # eps not positive
+        (vL, vS, B, n, 1e-8, acc, vL),               # x is v_L
+        (vL, vS, B, n, 1e-8, acc, vS + 4 * n),       # x overlaps the second sample of v_S
+        (vL, vS, B, n, 1e-8, acc, vL - 4 * n),       # x's second sample overlaps v_L
+    ]
+    for a, b, bb, nn, eps, ac, x in cases:
+        rc = lib.track_disagreement_update(a, b, bb, nn, eps, ac, x, 0.5, 0.25, None)
+        assert rc == T.TRACK_EINVAL, (a, b, bb, nn, eps, ac, x)
