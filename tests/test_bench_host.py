@@ -67,3 +67,16 @@ def test_timed_window_has_the_policys_split():
                            - round(count * k / n)) for v in range(warm, warm + n))
             assert abs(got - round(count * k / n)) == best
     assert bench.timed_window(np.zeros(10, np.uint8), 3, 4) == 3      # all-large: any window
+
+
+def test_event_timed_classes_carry_their_graph_timed_rate():
+    classes = {"gemm": {"ms": 1.0}, "update": {"ms": 0.1, "frac_of_hbm": 0.47},
+               "disagreement": {"ms": 0.01, "frac_of_hbm": 0.2}}
+    hbm = {"cfg_euler": {"frac_of_hbm": 0.73, "gb_per_s": 4960.0},
+           "disagreement": {"frac_of_hbm": 0.34, "gb_per_s": 2300.0},
+           "disagreement_update": {"frac_of_hbm": 0.55, "gb_per_s": 3700.0}}
+    out = bench.annotate_event_timed(classes, hbm)
+    assert out["update"]["graph_timed_frac_of_hbm"] == 0.73
+    assert out["disagreement"]["graph_timed_frac_of_hbm"] == 0.55
+    assert "graph_timed_frac_of_hbm" not in out["gemm"]
+    assert bench.annotate_event_timed({}, hbm) == {}
